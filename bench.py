@@ -1,0 +1,391 @@
+"""Benchmark of the masked secure linear layer on GB300.
+
+One step = one pass of the whole per-call path of Pi_Sec-Linear over one
+batch of l tokens: Init X (PRG masks R, T_i, E_x and U_x, K), rotation +
+encode + mask-add of X, the server's ring product Z = X' [W'; P]^T over
+Z_{2^32}, and the unmask + decode.  Init W (public chains and the masked
+weights) is one-time and is timed apart (``init_w_s``).
+
+Default workload: the attention projection at 7B shape (X 512 x 4096,
+W 4096 x 4096, Example 3.1 parameters).  Inputs are seeded synthetic
+(activations ~ N(0,1), weights ~ N(0,0.02)).  L2 is flushed (256 MiB write)
+between timed steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
+
+Prints one JSON line (rank 0).  With N > 1 (torchrun), every rank runs an
+independent replica on its own GPU (weak scaling, no data-path collective).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2607_29221_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "masked ring-GEMM effective TOPS (Z_2^32) and masked-layer tokens/s; % of roofline"
+L2_FLUSH_BYTES = 256 << 20
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="mine", choices=["mine", "reference"])
+    ap.add_argument("--workload", default="attn_proj_7b_512x4096x4096")
+    ap.add_argument("--variant", default="auto", choices=["auto", "tc", "mma", "imad"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget-s", type=float, default=12.0)
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,utilization.gpu,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(self.index), "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, util, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[0])); smax.append(float(parts[1])); util.append(float(parts[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        loaded = [s for s, u in zip(sm, util) if u > 0] or sm
+        return {"sm_mhz": float(np.median(loaded)), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm), "samples_under_load": len(loaded)}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def run_mine(args, rank, world):
+    import torch
+    import __graft_entry__ as G
+    from paper_2607_29221_gb300 import mosaic as M
+    from paper_2607_29221_gb300 import protocol as PR
+
+    G.build()
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    wk = wl.WORKLOADS[args.workload]
+    lin = wk.linears[0]
+    m, n, l = lin.m, lin.n, wk.l
+    n_pad = PR.pad_width(n)
+    variant = {"auto": M.GEMM_AUTO, "tc": M.GEMM_TC, "mma": M.GEMM_MMA_S8, "imad": M.GEMM_IMAD}[args.variant]
+    if variant == M.GEMM_AUTO:
+        variant = M.GEMM_TC if M.mosaic_gemm_variant_available(M.GEMM_TC) else M.GEMM_IMAD
+    key = wl.mask_key()
+    proto = PR.Protocol(key, M.default_params(), variant=variant)
+    Sr = proto.sum_r
+
+    W = torch.from_numpy(wl.weights(m, n, std=lin.w_std)).to(dev)
+    b = torch.from_numpy(wl.bias(m)).to(dev)
+    X_host = torch.from_numpy(wl.activations(l, n, seed=wl.SEED_X + rank)).pin_memory()
+    X = X_host.to(dev)
+
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    chains = PR.Chains(proto, n_pad)
+    layer = PR.SecureLinear(proto, W, 1, chains, bias=b)
+    torch.cuda.synchronize()
+    init_w_s = time.perf_counter() - t0
+
+    # persistent per-step buffers
+    Xp = torch.empty(l, n_pad, dtype=torch.int32, device=dev)
+    s_x = torch.empty(l, dtype=torch.float32, device=dev)
+    Xpl = torch.empty(4, l, n_pad, dtype=torch.int16, device=dev) if layer.use_planes else None
+    Z = torch.empty(l, m + Sr, dtype=torch.int32, device=dev)
+    Y = torch.empty(l, m, dtype=torch.float32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    gemm_ev = []
+
+    def step(i, record=False):
+        mp = layer.init_x(l, 1000 * rank + i)
+        layer.mask_input(X, mp, Xp, s_x, Xpl)
+        if record:
+            e0 = torch.cuda.Event(enable_timing=True); e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+        layer.server(Xp, Xpl, Z)
+        if record:
+            e1.record(stream)
+            gemm_ev.append((e0, e1))
+        layer.unmask(Z, mp, s_x, Y)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(_smi_index(dev.index))
+    sampler.start()
+    time.sleep(0.3)
+    _barrier(world)
+    torch.cuda.synchronize()
+    evs = []
+    for i in range(args.steps):
+        flush.fill_(i & 0xFF)
+        s0 = torch.cuda.Event(enable_timing=True); s1 = torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        step(args.warmup + i, record=True)
+        s1.record(stream)
+        evs.append((s0, s1))
+    torch.cuda.synchronize()
+    _barrier(world)
+    step_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    gemm_ms = float(np.mean([a.elapsed_time(b) for a, b in gemm_ev]))
+
+    # end to end through the public API with host buffers
+    Y_host = torch.empty(l, m, dtype=torch.float32).pin_memory()
+    e2e = []
+    for i in range(max(3, args.steps // 2)):
+        flush.fill_(i & 0xFF)
+        a = torch.cuda.Event(enable_timing=True); c = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        X.copy_(X_host, non_blocking=True)
+        step(10_000 + i)
+        Y_host.copy_(Y, non_blocking=True)
+        c.record(stream)
+        e2e.append((a, c))
+    torch.cuda.synchronize()
+    e2e_ms = float(np.mean([a.elapsed_time(c) for a, c in e2e]))
+    clocks = sampler.stop()
+
+    step_ms_max = _max_over_ranks(step_ms, world, dev)
+    e2e_ms_max = _max_over_ranks(e2e_ms, world, dev)
+    if rank != 0:
+        return
+
+    hbm, bf16, bf16_sus, peak_src = _peaks()
+    ring_macs = l * (m + Sr) * n_pad                       # server product Z = X' [W'; P]^T
+    tokens_s = world * l / (step_ms_max / 1e3)
+    ring_tops = 2 * ring_macs / (gemm_ms / 1e3) / 1e12
+    if variant == M.GEMM_TC:
+        achieved = 10 * 2 * ring_macs / (gemm_ms / 1e3) / 1e12      # bf16 digit-pair flops
+        roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": bf16, "unit": "TFLOP/s",
+                "frac": round(achieved / bf16, 4), "traffic": None,
+                "kernel": "ring_gemm_tc (10 bf16 digit-pair products per ring MAC)",
+                "peak_source": f"{peak_src} bf16 dense burst"}
+    else:
+        imad_peak = 152 * 64 * 2 * 2.07e9 / 1e12               # ring-ops/s: 64 IMAD/clk/SM, 2 ops each
+        roof = {"bound": "alu", "achieved": round(ring_tops, 3), "peak": round(imad_peak, 2),
+                "unit": "TOPS", "frac": round(ring_tops / imad_peak, 4), "traffic": None,
+                "kernel": "ring_gemm_imad", "peak_source": "derived: 152 SMs x 64 IMAD/clk x 2070 MHz"}
+    launches_per_step = _launches_per_step(proto.d, layer.use_planes)
+    out = {
+        "metric": METRIC, "value": round(tokens_s, 1), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms_max, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+        "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights)",
+        "config": {"workload": args.workload, "l": l, "m": m, "n": n, "n_pad": n_pad,
+                   "params": "Example 3.1: d=3, r=1536/1024/652, t=80/80, sigma=0.5, b=16",
+                   "gemm_variant": {M.GEMM_TC: "tc", M.GEMM_IMAD: "imad", M.GEMM_MMA_S8: "mma_s8"}[variant],
+                   "l2": "flushed between timed steps (256 MiB write)",
+                   "parallelism": f"replicas x{world}"},
+        "ring_tops": round(ring_tops, 2),
+        "gemm_ms": round(gemm_ms, 4),
+        "init_w_s": round(init_w_s, 3),
+        "roofline": roof,
+        "e2e": {"value": round(world * l / (e2e_ms_max / 1e3), 1), "unit": "tokens/s",
+                "h2d_bytes_per_step": l * n * 4, "d2h_bytes_per_step": l * m * 4},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(wk, args.cpu_budget_s)
+    print(json.dumps(out), flush=True)
+
+
+def _launches_per_step(d: int, planes: bool) -> int:
+    # Init X: R, E_x, (d-1) sparse T, U_x product, K product, 2 sparse gathers (d > 1)
+    init_x = 4 + (d - 1) + (2 if d > 1 else 0)
+    return init_x + 1 + (1 if planes else 1) + 2      # encode, server product, unmask (2)
+
+
+def _smi_index(dev_index: int) -> int:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    parts = [p for p in vis.split(",") if p.strip()]
+    if parts and all(p.strip().isdigit() for p in parts) and dev_index < len(parts):
+        return int(parts[dev_index])
+    return dev_index
+
+
+def _barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def _max_over_ranks(v, world, dev):
+    if world == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle as baseline / reference arm
+# ---------------------------------------------------------------------------
+def _oracle_setup(wk):
+    import oracle as O
+    lin = wk.linears[0]
+    m, n = lin.m, lin.n
+    n_pad = 1 << max(0, (n - 1).bit_length())
+    key = wl.mask_key()
+    p = O.Params()
+    t0 = time.perf_counter()
+    P, C = O.chains(key, p, n_pad)
+    W = wl.weights(m, n, std=lin.w_std)
+    ws = O.init_w(key, p, W, 1, P, C, n_pad)
+    return O, key, p, P, C, ws, time.perf_counter() - t0
+
+
+def _oracle_step(O, key, p, P, C, ws, X, pass_id, b):
+    ps = O.init_x(key, p, X.shape[1], pass_id, C, ws.J, ws.n_pad)
+    _, s_x, Xm = O.mask_input(X, ws, ps.U_x)
+    Ym, Q = O.server(ws, P, Xm)
+    Yh = O.unmask(p, ws, ps, Ym, Q)
+    return O.decode(Yh, ws.s_w, s_x, b)
+
+
+def cpu_baseline(wk, budget_s, tokens=None):
+    O, key, p, P, C, ws, init_s = _oracle_setup(wk)
+    l = wk.l if tokens is None else tokens
+    X = wl.activations(l, wk.linears[0].n).T.copy()
+    b = wl.bias(wk.linears[0].m)
+    done, t0 = 0, time.perf_counter()
+    while True:
+        _oracle_step(O, key, p, P, C, ws, X, 500 + done, b)
+        done += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": round(done * l / dt, 2), "unit": "tokens/s", "cores": O.num_threads(),
+            "kind": "oracle",
+            "sample": f"{done} full per-call steps of {l} tokens ({wk.name}); one-time chains + Init W "
+                      f"({init_s:.1f} s) excluded like the GPU value",
+            "init_w_s": round(init_s, 2)}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    wk = wl.WORKLOADS[args.workload]
+    O, key, p, P, C, ws, init_s = _oracle_setup(wk)
+    lin = wk.linears[0]
+    l = min(wk.l, 64)               # bounded sample of the workload's tokens per step
+    X = wl.activations(l, lin.n).T.copy()
+    b = wl.bias(lin.m)
+    for i in range(args.warmup):
+        _oracle_step(O, key, p, P, C, ws, X, 900 + i, b)
+    times = []
+    for i in range(args.steps):
+        t0 = time.perf_counter()
+        _oracle_step(O, key, p, P, C, ws, X, 950 + i, b)
+        times.append(time.perf_counter() - t0)
+    sec = float(np.mean(times))
+    val = l / sec
+    out = {"impl": "reference", "metric": METRIC, "value": round(val, 2), "unit": "tokens/s",
+           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(sec * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+           "config": {"workload": args.workload, "l": wk.l, "m": lin.m, "n": lin.n,
+                      "params": "Example 3.1"},
+           "cpu_baseline": {"value": round(val, 2), "unit": "tokens/s", "cores": O.num_threads(),
+                            "kind": "oracle",
+                            "sample": f"{l} of {wk.l} tokens per step; one-time chains + Init W "
+                                      f"({init_s:.1f} s) excluded"},
+           "e2e": {"value": round(val, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        dist.init_process_group("nccl")
+    try:
+        run_mine(args, rank, world)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,302 @@
+/*
+ * mosaic.h -- C ABI of the GB300 masked ring-matmul library (libmosaic.so).
+ *
+ * The library computes the data-parallel hot path of MOSAIC's secure linear
+ * layer: the random Hadamard rotation and fixed-point encoding of
+ * Pi_Sec-Linear (Sec. 4 protocol box), the LWE/LPN masks of
+ * Pi_Sec-Approx-MatMul (Sec. 3.2 protocol box, Init W and Init X), the
+ * server's product over Z_{2^32} (Online step 3) and the client's unmask and
+ * decode (Online step 5 and Pi_Sec-Linear Online step 3).
+ *
+ * Conventions shared by every entry point
+ *  - Every matrix pointer is a DEVICE pointer owned by the caller; the
+ *    library never allocates, frees or retains memory.  Scratch memory comes
+ *    in `ws` (size from mosaic_workspace_bytes) and must not overlap any
+ *    other argument.
+ *  - Every call is asynchronous on `stream` (a cudaStream_t passed as void*;
+ *    NULL is the legacy default stream).  A status of MOSAIC_OK means the
+ *    work was validated and enqueued; faults inside a kernel surface at the
+ *    caller's next synchronisation as a CUDA error.
+ *  - Matrices are row-major with an explicit leading dimension (elements).
+ *    Activations are TOKEN-MAJOR: the paper's X (n x l) is stored as
+ *    X_tm = X^T (l x n), and Y (m x l) as Y_tm (l x m).  Every ring product is
+ *    "NT": C[i][j] = sum_k A[i][k] * B[j][k] mod 2^32.
+ *  - Ring elements are uint32_t (kappa = 32: Z_{2^32}, two's complement for
+ *    signed values).  Float inputs must be finite unless stated otherwise.
+ *  - Host pointers (mosaic_params*, mosaic_key*) are read during the call
+ *    only.
+ *  - Errors are returned, never thrown or printed; no entry point exits.
+ */
+#ifndef MOSAIC_H
+#define MOSAIC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MOSAIC_OK = 0,
+    MOSAIC_ERR_ARG = 1,          /* null pointer, bad enum, bad parameter value      */
+    MOSAIC_ERR_SHAPE = 2,        /* size out of range, n_pad not a power of two, ... */
+    MOSAIC_ERR_ALIGN = 3,        /* pointer or leading dimension misaligned          */
+    MOSAIC_ERR_UNSUPPORTED = 4,  /* valid request this build does not implement      */
+    MOSAIC_ERR_CUDA = 5,         /* a CUDA runtime call or launch failed             */
+    MOSAIC_ERR_WORKSPACE = 6,    /* ws too small (see mosaic_workspace_bytes)        */
+    MOSAIC_ERR_TIMEOUT = 7       /* a bounded device wait expired (tensor GEMM)      */
+} mosaic_status;
+
+/* Protocol parameters (Example 3.1 defaults, lambda = 140).
+ * d       nesting depth of the LWE + LPN mask, 1..3 (Sec. 3.2)
+ * r[i-1]  rank r_i, i = 1..d (1536, 1024, 652); r_1 > r_2 > ... is not required
+ * t[i-1]  Hamming weight t_i of each row of S_i and each column of T_i,
+ *         i = 2..d (t[0] is unused; 80, 80); 1 <= t_i <= r_{i-1} / 2
+ * sigma   Gaussian parameter of E_w, E_x: Pr[k] ~ exp(-k^2 / (2 sigma^2)),
+ *         0 <= sigma <= 8 (0 disables the noise)
+ * qbits   signed operand width b of Pi_Sec-Linear (16); the operand window is
+ *         q_max = min(2^(b-1) - 1, floor(sqrt(2^31 / n_pad)))
+ * rounds  ChaCha rounds of the PRG (20; 8 and 12 accepted)
+ * kappa   ring width, must be 32                                           */
+typedef struct {
+    uint32_t kappa;
+    uint32_t d;
+    uint32_t r[3];
+    uint32_t t[3];
+    float sigma;
+    uint32_t qbits;
+    uint32_t rounds;
+} mosaic_params;
+
+/* 256-bit PRG key (8 little-endian words). */
+typedef struct {
+    uint32_t key[8];
+} mosaic_key;
+
+/* Fills `p` with the Example 3.1 parameters (d = 3, r = 1536/1024/652,
+ * t = 80/80, sigma = 0.5, b = 16, 20 rounds, kappa = 32). */
+void mosaic_default_params(mosaic_params *p);
+
+/* Human-readable name of a status code (static string). */
+const char *mosaic_status_string(mosaic_status s);
+
+/* q_max for a rotation width n_pad (Sec. 4 straw-man paragraph: each entry of
+ * W_hat X_hat is at most n q_max^2, and n q_max^2 <= 2^(kappa-1)).  Returns 0
+ * if n_pad is not a power of two in [32, 32768] or qbits is outside [2, 16]. */
+int32_t mosaic_qmax(int64_t n_pad, uint32_t qbits);
+
+/* Writes the inversion table of the discrete Gaussian with parameter sigma
+ * (Sec. 3.1: Pr[k] ~ exp(-k^2 / (2 sigma^2)) on [-B, B], B = ceil(12 sigma)):
+ * table[j] = floor(2^64 CDF(j - B)) computed in long double, last entry
+ * 2^64 - 1.  Host-only.  Returns B, or -1 if sigma is outside (0, 8] or
+ * capacity < 2B + 1. */
+int mosaic_gaussian_table(float sigma, uint64_t *table, int capacity);
+
+/* ------------------------------------------------------------------------ */
+/* PRG and samplers (Sec. 3.2 box: "C samples ...").  The generator is       */
+/* ChaCha in counter mode (RFC 8439 block layout): stream (tag, stream_id)   */
+/* uses nonce = (tag, stream_id low 32 bits, stream_id high 32 bits); word w */
+/* of the stream is word w mod 16 of block floor(w / 16).                    */
+/* Tags: kind in bits 0..7, level i in bits 8..15.                           */
+/* ------------------------------------------------------------------------ */
+enum {
+    MOSAIC_TAG_M = 1,     /* public M_i        (stream_id: the chain id, n_pad by convention) */
+    MOSAIC_TAG_N = 2,     /* public N_i                                                        */
+    MOSAIC_TAG_L = 3,     /* secret L           (stream_id: matrix id)                         */
+    MOSAIC_TAG_S = 4,     /* secret sparse S_i                                                  */
+    MOSAIC_TAG_EW = 5,    /* weight noise E_w                                                   */
+    MOSAIC_TAG_R = 6,     /* per-pass R         (stream_id: pass id)                            */
+    MOSAIC_TAG_T = 7,     /* per-pass sparse T_i                                                */
+    MOSAIC_TAG_EX = 8,    /* activation noise E_x                                               */
+    MOSAIC_TAG_SIGN = 9   /* rotation signs d   (stream_id: matrix id)                          */
+};
+
+/* out[i * ldo + j] = stream word i * cols + j: uniform elements of Z_{2^32}.
+ * rows, cols >= 0; rows * cols < 2^36; ldo >= cols. */
+mosaic_status mosaic_prg_uniform(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
+                                 uint32_t rounds, int64_t rows, int64_t cols, uint32_t *out,
+                                 int64_t ldo, void *stream);
+
+/* out[e], e < count: discrete Gaussian ring elements (two's complement).
+ * Element e reads u = word(2e) | word(2e+1) << 32 and returns the smallest
+ * k in [-B, B] (B = ceil(12 sigma)) with u < floor(2^64 CDF(k)), else B.
+ * sigma = 0 writes zeros.  count < 2^35. */
+mosaic_status mosaic_prg_gaussian(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
+                                  uint32_t rounds, float sigma, int64_t count, uint32_t *out,
+                                  void *stream);
+
+/* rows sparse vectors over [0, r), exactly t nonzeros each (LPN noise of
+ * Hamming weight t, Example 3.1).  Row j reads its own window of 65536
+ * stream words starting at word j * 65536: positions p = (w * r) >> 32 in
+ * draw order, repeats skipped, then the next nonzero words as values.
+ * idx, val: rows x t row-major.  rows < 2^20, 1 <= t <= min(r/2, 1024).
+ * `fail` (device, nullable) is set to 1 if a row exhausts its window
+ * (probability below 2^-1000 within these limits). */
+mosaic_status mosaic_prg_sparse(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
+                                uint32_t rounds, int64_t rows, uint32_t r, uint32_t t,
+                                uint32_t *idx, uint32_t *val, uint32_t *fail, void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Rotation and encoding (Pi_Sec-Linear box; Sec. 4 "Random Hadamard        */
+/* rotation").                                                               */
+/* ------------------------------------------------------------------------ */
+
+/* y = rows of H D x (Sec. 4: R = H D, H the normalised Walsh-Hadamard
+ * matrix in Sylvester order, D = diag(d)).  Each row of x (length n, leading
+ * dimension ldx) is zero-padded to n_pad, negated where bit c of
+ * sign_words[c / 32] is set (sign_words: n_pad / 32 device words, NULL for
+ * D = I), transformed by butterflies (a, b) -> (a + b, a - b) in fp32 with
+ * stages h = 1, 2, ..., n_pad / 2 in that order, then multiplied by
+ * fl32(1 / sqrt(n_pad)).  y: rows x n_pad (leading dimension n_pad); y must
+ * not overlap x.  n_pad a power of two in [32, 32768], 1 <= n <= n_pad.
+ * x, y 16-byte aligned; ldx a multiple of 4. */
+mosaic_status mosaic_hadamard(const float *x, int64_t ldx, float *y, int64_t rows, int64_t n,
+                              int64_t n_pad, const uint32_t *sign_words, void *stream);
+
+/* Fused rotation + per-row quantisation + mask-add (Pi_Sec-Linear Online
+ * step 1 for activation rows, Init W step 2 for weight rows; Approx-MatMul
+ * Online step 2).  For each row: v = H D x as in mosaic_hadamard when
+ * `rotate` is 1 (v = x zero-padded when 0); s = max|v| / qmax (fp32);
+ * code = clamp(rint(v / s), -qmax, qmax) (IEEE division, ties to even),
+ * 0 when s = 0; a row with a non-finite value gets s = NaN and code 0.
+ * out[row][c] = code + mask[row][c] mod 2^32 (mask nullable: no add);
+ * scale[row] = s.  `planes` (nullable) additionally receives the signed
+ * base-2^8 digits of out as bf16 digit planes, layout [4][rows][n_pad]
+ * (see mosaic_digit_split).  out: rows x ldo; mask: rows x ldm.
+ * 1 <= qmax <= 32767.  Alignment as mosaic_hadamard; ldo, ldm multiples of 4. */
+mosaic_status mosaic_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, int64_t n_pad,
+                            int32_t qmax, int rotate, const uint32_t *sign_words,
+                            const uint32_t *mask, int64_t ldm, uint32_t *out, int64_t ldo,
+                            float *scale, uint16_t *planes, void *stream);
+
+/* Signed base-2^8 digit split of ring elements (Sec. 5.2 "Emulation
+ * approach", re-designed with signed digits): with b = a + 0x80808080,
+ * digit i is (int)((b >> 8i) & 0xff) - 128 in [-128, 127], so that
+ * a = sum_i digit_i 2^(8i) mod 2^32.  Each digit is written exactly as a
+ * bf16 value into planes[i][row][col] (layout [4][rows][cols], bf16 bits in
+ * uint16_t).  cols a multiple of 8; lda a multiple of 4; 16-byte aligned. */
+mosaic_status mosaic_digit_split(const uint32_t *a, int64_t lda, int64_t rows, int64_t cols,
+                                 uint16_t *planes, void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Ring product (Approx-MatMul Online step 3; Sec. 5.2 emulation).           */
+/* ------------------------------------------------------------------------ */
+typedef enum {
+    MOSAIC_GEMM_AUTO = 0,     /* fastest available variant for the shape                    */
+    MOSAIC_GEMM_TC = 1,       /* tcgen05 kind::f16: 10 exact bf16 digit-pair products, TMEM  */
+    MOSAIC_GEMM_MMA_S8 = 2,   /* legacy mma.sync s8 digit-pair products, int32 accumulators */
+    MOSAIC_GEMM_IMAD = 3      /* CUDA-core 32-bit multiply-add                               */
+} mosaic_gemm_variant;
+
+/* 1 if this build implements `variant` on the current device (host-only
+ * query of the build and of the device's compute capability), else 0. */
+int mosaic_gemm_variant_available(int variant);
+
+/* C[i][j] = sum_{k<K} A[i][k] B[j][k] mod 2^32, i < M, j < N.
+ * A: M x K (lda), B: N x K (ldb), C: M x N (ldc); C must not overlap A or B.
+ * M, N, K >= 0, K <= 2^20.  The TC and MMA_S8 variants split A and B into
+ * digit planes in `ws` (mosaic_workspace_bytes(MOSAIC_OP_RING_GEMM, ...));
+ * IMAD needs no workspace.  TC requires lda, ldb multiples of 4 and 16-byte
+ * aligned A, B. */
+mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb,
+                               uint32_t *C, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                               int variant, void *ws, size_t ws_bytes, void *stream);
+
+/* Same product from pre-split bf16 digit planes (layout [4][rows][K] with a
+ * plane stride of rows_alloc * ldp elements, see mosaic_digit_split /
+ * mosaic_encode).  A planes: M rows (plane stride a_plane), B planes: N rows
+ * (plane stride b_plane); ldpa, ldpb leading dimensions in elements,
+ * multiples of 8; 16-byte aligned.  Variant TC or MMA_S8. */
+mosaic_status mosaic_ring_gemm_planes(const uint16_t *A_planes, int64_t ldpa, int64_t a_plane,
+                                      const uint16_t *B_planes, int64_t ldpb, int64_t b_plane,
+                                      uint32_t *C, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                                      int variant, void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Masks (Sec. 3.2 protocol box).  Sr = r_1 + ... + r_d.                      */
+/* ------------------------------------------------------------------------ */
+
+/* Public chains for input width n_pad (Init W steps 1-3, 5): samples
+ * M_i (r_i x r_{i-1}, element (a,b) = word a r_{i-1} + b of (M, level i))
+ * and N_i (r_{i-1} x r_i, element (a,b) = word a r_i + b of (N, level i)),
+ * r_0 = n_pad, from stream `chain_id`, and writes
+ *   P  (Sr x n_pad): rows [P_1; P_2; ...; P_d], P_i = M_i ... M_1
+ *   C  (n_pad x Sr): columns [C_1 | ... | C_d], C_i = N_1 ... N_i
+ *   CT (Sr x n_pad): C transposed.
+ * ws: mosaic_workspace_bytes(MOSAIC_OP_MASK_CHAINS, 0, n_pad, 0, p). */
+mosaic_status mosaic_mask_chains(const mosaic_params *p, const mosaic_key *key,
+                                 uint64_t chain_id, int64_t n_pad, uint32_t *P, uint32_t *C,
+                                 uint32_t *CT, void *ws, size_t ws_bytes, void *stream);
+
+/* Init W of Pi_Sec-Linear and Pi_Sec-Approx-MatMul for one weight matrix
+ * W (m x n float, leading dimension ldw) with matrix id `matrix_id`:
+ *   sign_words (n_pad/32)  d of R = H D           (stream (SIGN, matrix_id))
+ *   W_hat, s_w (m)          rows of W R^T quantised (mosaic_encode)
+ *   L (m x r_d)             uniform                 (stream (L, matrix_id))
+ *   S_idx, S_val            S_{i+1}, i = 1..d-1: m x t_{i+1} each, stored
+ *                           level after level        (stream (S, level i+1))
+ *   E_w (m x n_pad)         Gaussian                (stream (EW, matrix_id))
+ *   Wp ((m + Sr) x n_pad)   rows [0, m):   W' = W_hat + L P_d + sum S_{i+1} P_i + E_w
+ *                           rows [m, m+Sr): a copy of P (server-side operand)
+ *   J (m x Sr)              columns [J_1 | ... | J_d], J_i = (W_hat + E_w) C_i
+ * Wp_planes (nullable): bf16 digit planes of Wp ([4][m + Sr][n_pad]).
+ * ws: mosaic_workspace_bytes(MOSAIC_OP_MASK_WEIGHT, m, n_pad, 0, p). */
+mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key,
+                                 uint64_t matrix_id, const float *W, int64_t ldw, int64_t m,
+                                 int64_t n, int64_t n_pad, const uint32_t *P, const uint32_t *CT,
+                                 uint32_t *sign_words, float *s_w, uint32_t *L, uint32_t *S_idx,
+                                 uint32_t *S_val, uint32_t *Wp, uint16_t *Wp_planes, uint32_t *J,
+                                 int variant, void *ws, size_t ws_bytes, void *stream);
+
+/* Init X (per pass, independent of X): samples R^T (l x r_d, stream (R,
+ * pass_id)), T_{i+1} (column k = sparse row k, stream (T, level i+1)) and
+ * E_x^T (l x n_pad, stream (EX, pass_id)) and writes
+ *   Ux_tm (l x n_pad) = (C_d R + sum_i C_i T_{i+1} + E_x)^T
+ *   K_tm  (l x m)     = (J_d R + sum_i J_i T_{i+1})^T
+ * from C (n_pad x Sr) and J (m x Sr).
+ * ws: mosaic_workspace_bytes(MOSAIC_OP_MASK_ACTIVATION, m, n_pad, l, p). */
+mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *key,
+                                     uint64_t pass_id, int64_t m, int64_t n_pad, int64_t l,
+                                     const uint32_t *C, const uint32_t *J, uint32_t *Ux_tm,
+                                     uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
+                                     void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Unmask and decode (Approx-MatMul Online step 5; Pi_Sec-Linear Online      */
+/* step 3).                                                                  */
+/* ------------------------------------------------------------------------ */
+
+/* Z (l x ldz) is the server output X'_tm Wp^T: columns [0, m) hold Y'_tm,
+ * columns [m, m + Sr) hold [Q_1 | ... | Q_d]_tm.  Computes
+ *   Y_hat = Y' - K - L Q_d - sum_{i<d} S_{i+1} Q_i      (mod 2^32)
+ *   Y[k][j] = ((float)(int32)Y_hat[k][j] * s_w[j]) * s_x[k] + bias[j]
+ * (fp32, two roundings of the products, no fused multiply-add; bias
+ * nullable).  Y: l x m fp32 (ldy); Yhat (nullable): l x m uint32 (ldy).
+ * ws: mosaic_workspace_bytes(MOSAIC_OP_UNMASK, m, 0, l, p). */
+mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z,
+                            int64_t ldz, const uint32_t *K_tm, const uint32_t *L,
+                            const uint32_t *S_idx, const uint32_t *S_val, const float *s_w,
+                            const float *s_x, const float *bias, float *Y, uint32_t *Yhat,
+                            int64_t ldy, int variant, void *ws, size_t ws_bytes, void *stream);
+
+/* Workspace sizes. */
+typedef enum {
+    MOSAIC_OP_RING_GEMM = 1,        /* M = rows of A, n_pad = rows of B (N), l = K */
+    MOSAIC_OP_MASK_CHAINS = 2,
+    MOSAIC_OP_MASK_WEIGHT = 3,
+    MOSAIC_OP_MASK_ACTIVATION = 4,
+    MOSAIC_OP_UNMASK = 5
+} mosaic_op;
+
+/* Bytes of `ws` the op needs for the given sizes and variant-independent
+ * worst case (0 on invalid arguments).  Arguments unused by an op are
+ * ignored. */
+size_t mosaic_workspace_bytes(int op, int64_t m, int64_t n_pad, int64_t l,
+                              const mosaic_params *p);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOSAIC_H */

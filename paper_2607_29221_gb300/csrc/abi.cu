@@ -1,0 +1,454 @@
+// extern "C" entry points of libmosaic.so: argument validation, workspace
+// carving and the composition of kernels into the protocol steps of
+// Pi_Sec-Approx-MatMul (Sec. 3.2 protocol box) and Pi_Sec-Linear (Sec. 4
+// protocol box).  See include/mosaic.h for the contract of each call.
+#include <math.h>
+#include <string.h>
+
+#include "mosaic_internal.cuh"
+
+using namespace mosaic;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+size_t up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
+
+// Bump allocator over the caller's workspace.
+struct Carve {
+    char *base;
+    size_t cap, used;
+    template <class T>
+    T *take(size_t count) {
+        const size_t bytes = up(count * sizeof(T));
+        if (used + bytes > cap) return nullptr;
+        T *p = reinterpret_cast<T *>(base + used);
+        used += bytes;
+        return p;
+    }
+};
+
+bool rounds_ok(uint32_t r) { return r == 8 || r == 12 || r == 20; }
+
+mosaic_status check_params(const mosaic_params *p) {
+    if (!p) return MOSAIC_ERR_ARG;
+    if (p->kappa != 32) return MOSAIC_ERR_UNSUPPORTED;
+    if (p->d < 1 || p->d > 3) return MOSAIC_ERR_ARG;
+    for (uint32_t i = 0; i < p->d; i++)
+        if (p->r[i] < 2 || p->r[i] > 65536) return MOSAIC_ERR_ARG;
+    for (uint32_t i = 1; i < p->d; i++) {
+        const uint32_t t = p->t[i], r = p->r[i - 1];
+        if (t < 1 || t > 1024 || t > r / 2) return MOSAIC_ERR_ARG;
+    }
+    if (!(p->sigma >= 0.0f && p->sigma <= 8.0f)) return MOSAIC_ERR_ARG;
+    if (p->qbits < 2 || p->qbits > 16) return MOSAIC_ERR_ARG;
+    if (!rounds_ok(p->rounds)) return MOSAIC_ERR_ARG;
+    return MOSAIC_OK;
+}
+
+int64_t sum_r(const mosaic_params *p) {
+    int64_t s = 0;
+    for (uint32_t i = 0; i < p->d; i++) s += p->r[i];
+    return s;
+}
+// Column / row offset of level i (1-based) inside the stacked chains.
+int64_t off_r(const mosaic_params *p, uint32_t i) {
+    int64_t s = 0;
+    for (uint32_t q = 1; q < i; q++) s += p->r[q - 1];
+    return s;
+}
+uint32_t tag_of(uint32_t kind, uint32_t level) { return kind | (level << 8); }
+bool npad_ok(int64_t n_pad) { return is_pow2(n_pad) && n_pad >= 32 && n_pad <= 32768; }
+
+// ring product dispatch for the internal compositions (uint32 operands)
+mosaic_status gemm_u32(int variant, const uint32_t *A, int64_t sai, int64_t sak, const uint32_t *B,
+                       int64_t sbj, int64_t sbk, uint32_t *C, int64_t ldc, const uint32_t *Cin,
+                       int64_t ldcin, int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st) {
+    (void)variant;
+    return ring_gemm_imad(A, sai, sak, B, sbj, sbk, C, ldc, Cin, ldcin, sgn, M, N, K, st);
+}
+
+size_t ws_chains(int64_t n_pad, const mosaic_params *p) {
+    size_t s = 0;
+    int64_t prev = n_pad;
+    for (uint32_t i = 1; i <= p->d; i++) {
+        const int64_t ri = p->r[i - 1];
+        if (i >= 2) s += up(sizeof(uint32_t) * (size_t)(ri * prev)) * 2;   // M_i and N_i
+        prev = ri;
+    }
+    return s;
+}
+size_t ws_weight(int64_t m, int64_t n_pad, const mosaic_params *) {
+    return up(sizeof(uint32_t) * (size_t)(m * n_pad));
+}
+size_t ws_activation(int64_t l, int64_t n_pad, const mosaic_params *p) {
+    (void)n_pad;
+    size_t s = up(sizeof(uint32_t) * (size_t)(l * p->r[p->d - 1]));
+    for (uint32_t i = 2; i <= p->d; i++) s += 2 * up(sizeof(uint32_t) * (size_t)(l * p->t[i - 1]));
+    return s;
+}
+size_t ws_unmask(int64_t m, int64_t l, const mosaic_params *) {
+    return up(sizeof(uint32_t) * (size_t)(l * m));
+}
+size_t ws_gemm(int64_t M, int64_t N, int64_t K) {
+    return up(8 * (size_t)(M * K)) + up(8 * (size_t)(N * K));
+}
+
+}  // namespace
+
+extern "C" {
+
+void mosaic_default_params(mosaic_params *p) {
+    if (!p) return;
+    memset(p, 0, sizeof *p);
+    p->kappa = 32;
+    p->d = 3;
+    p->r[0] = 1536; p->r[1] = 1024; p->r[2] = 652;
+    p->t[0] = 0; p->t[1] = 80; p->t[2] = 80;
+    p->sigma = 0.5f;
+    p->qbits = 16;
+    p->rounds = 20;
+}
+
+const char *mosaic_status_string(mosaic_status s) {
+    switch (s) {
+        case MOSAIC_OK: return "ok";
+        case MOSAIC_ERR_ARG: return "invalid argument";
+        case MOSAIC_ERR_SHAPE: return "invalid shape";
+        case MOSAIC_ERR_ALIGN: return "misaligned pointer or leading dimension";
+        case MOSAIC_ERR_UNSUPPORTED: return "unsupported by this build";
+        case MOSAIC_ERR_CUDA: return "CUDA error";
+        case MOSAIC_ERR_WORKSPACE: return "workspace too small";
+        case MOSAIC_ERR_TIMEOUT: return "device wait timed out";
+    }
+    return "unknown status";
+}
+
+int32_t mosaic_qmax(int64_t n_pad, uint32_t qbits) {
+    if (!npad_ok(n_pad) || qbits < 2 || qbits > 16) return 0;
+    const int64_t cap = ((int64_t)1 << (qbits - 1)) - 1;
+    const int64_t lim = ((int64_t)1 << 31) / n_pad;
+    int64_t q = (int64_t)sqrt((double)lim);
+    while (q * q > lim) q--;
+    while ((q + 1) * (q + 1) <= lim) q++;
+    return (int32_t)(q < cap ? q : cap);
+}
+
+int mosaic_gaussian_table(float sigma, uint64_t *table, int capacity) {
+    if (!(sigma > 0.0f && sigma <= 8.0f) || !table) return -1;
+    unsigned long long t[2 * kMaxGaussBound + 1];
+    const int B = gaussian_table_host(sigma, t);
+    if (capacity < 2 * B + 1) return -1;
+    for (int i = 0; i < 2 * B + 1; i++) table[i] = t[i];
+    return B;
+}
+
+mosaic_status mosaic_prg_uniform(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
+                                 uint32_t rounds, int64_t rows, int64_t cols, uint32_t *out,
+                                 int64_t ldo, void *stream) {
+    if (!key || !rounds_ok(rounds)) return MOSAIC_ERR_ARG;
+    if (rows < 0 || cols < 0 || ldo < cols) return MOSAIC_ERR_SHAPE;
+    if (rows * cols >= ((int64_t)1 << 36)) return MOSAIC_ERR_SHAPE;
+    if (rows * cols == 0) return MOSAIC_OK;
+    if (!out) return MOSAIC_ERR_ARG;
+    return prg_uniform(to_key(key), tag, stream_id, (int)rounds, rows, cols, out, ldo,
+                       as_stream(stream));
+}
+
+mosaic_status mosaic_prg_gaussian(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
+                                  uint32_t rounds, float sigma, int64_t count, uint32_t *out,
+                                  void *stream) {
+    if (!key || !rounds_ok(rounds)) return MOSAIC_ERR_ARG;
+    if (!(sigma >= 0.0f && sigma <= 8.0f)) return MOSAIC_ERR_ARG;
+    if (count < 0 || count >= ((int64_t)1 << 35)) return MOSAIC_ERR_SHAPE;
+    if (count == 0) return MOSAIC_OK;
+    if (!out) return MOSAIC_ERR_ARG;
+    return prg_gaussian(to_key(key), tag, stream_id, (int)rounds, sigma, count, out,
+                        as_stream(stream));
+}
+
+mosaic_status mosaic_prg_sparse(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
+                                uint32_t rounds, int64_t rows, uint32_t r, uint32_t t,
+                                uint32_t *idx, uint32_t *val, uint32_t *fail, void *stream) {
+    if (!key || !rounds_ok(rounds)) return MOSAIC_ERR_ARG;
+    if (rows < 0 || rows >= ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
+    if (t < 1 || t > 1024 || r < 2 || t > r / 2) return MOSAIC_ERR_ARG;
+    if (rows == 0) return MOSAIC_OK;
+    if (!idx || !val) return MOSAIC_ERR_ARG;
+    return prg_sparse(to_key(key), tag, stream_id, (int)rounds, rows, r, t, idx, val, fail,
+                      as_stream(stream));
+}
+
+mosaic_status mosaic_hadamard(const float *x, int64_t ldx, float *y, int64_t rows, int64_t n,
+                              int64_t n_pad, const uint32_t *sign_words, void *stream) {
+    if (!npad_ok(n_pad) || n < 1 || n > n_pad || rows < 0 || ldx < n) return MOSAIC_ERR_SHAPE;
+    if (rows == 0) return MOSAIC_OK;
+    if (!x || !y) return MOSAIC_ERR_ARG;
+    if (!aligned16(y)) return MOSAIC_ERR_ALIGN;
+    return fwht_encode(x, ldx, rows, n, n_pad, sign_words, 1, 0, y, 0, nullptr, 0, nullptr, 0,
+                       nullptr, nullptr, as_stream(stream));
+}
+
+mosaic_status mosaic_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, int64_t n_pad,
+                            int32_t qmax, int rotate, const uint32_t *sign_words,
+                            const uint32_t *mask, int64_t ldm, uint32_t *out, int64_t ldo,
+                            float *scale, uint16_t *planes, void *stream) {
+    if (!npad_ok(n_pad) || n < 1 || n > n_pad || rows < 0 || ldx < n || ldo < n_pad)
+        return MOSAIC_ERR_SHAPE;
+    if (mask && ldm < n_pad) return MOSAIC_ERR_SHAPE;
+    if (qmax < 1 || qmax > 32767 || (rotate != 0 && rotate != 1)) return MOSAIC_ERR_ARG;
+    if (rows == 0) return MOSAIC_OK;
+    if (!x || !out || !scale) return MOSAIC_ERR_ARG;
+    if (!aligned16(out) || ldo % 4 || (mask && (!aligned16(mask) || ldm % 4)) ||
+        (planes && !aligned16(planes)))
+        return MOSAIC_ERR_ALIGN;
+    return fwht_encode(x, ldx, rows, n, n_pad, sign_words, rotate, 1, nullptr, qmax, mask, ldm, out,
+                       ldo, scale, planes, as_stream(stream));
+}
+
+mosaic_status mosaic_digit_split(const uint32_t *a, int64_t lda, int64_t rows, int64_t cols,
+                                 uint16_t *planes, void *stream) {
+    if (rows < 0 || cols < 0 || cols % 8 || lda < cols) return MOSAIC_ERR_SHAPE;
+    if (rows == 0 || cols == 0) return MOSAIC_OK;
+    if (!a || !planes) return MOSAIC_ERR_ARG;
+    if (!aligned16(a) || !aligned16(planes) || lda % 4) return MOSAIC_ERR_ALIGN;
+    return digit_split(a, lda, rows, cols, planes, cols, rows * cols, as_stream(stream));
+}
+
+int mosaic_gemm_variant_available(int variant) {
+    switch (variant) {
+        case MOSAIC_GEMM_AUTO: return 1;
+        case MOSAIC_GEMM_IMAD: return 1;
+        case MOSAIC_GEMM_TC: return tc_available() ? 1 : 0;
+        case MOSAIC_GEMM_MMA_S8: return mma_s8_available() ? 1 : 0;
+    }
+    return 0;
+}
+
+mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb,
+                               uint32_t *C, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                               int variant, void *ws, size_t ws_bytes, void *stream) {
+    if (M < 0 || N < 0 || K < 0 || K > ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
+    if (lda < K || ldb < K || ldc < N) return MOSAIC_ERR_SHAPE;
+    if (variant < MOSAIC_GEMM_AUTO || variant > MOSAIC_GEMM_IMAD) return MOSAIC_ERR_ARG;
+    if (M == 0 || N == 0) return MOSAIC_OK;
+    if (!A || !B || !C) return MOSAIC_ERR_ARG;
+    cudaStream_t st = as_stream(stream);
+    if (variant == MOSAIC_GEMM_IMAD || (variant == MOSAIC_GEMM_AUTO && !tc_available()))
+        return ring_gemm_imad(A, lda, 1, B, ldb, 1, C, ldc, nullptr, 0, 1, M, N, K, st);
+    if (variant == MOSAIC_GEMM_MMA_S8)
+        return ring_gemm_mma_s8(A, lda, B, ldb, C, ldc, nullptr, 0, 1, M, N, K, st);
+    // Tensor-core variant: split both operands into digit planes in ws.
+    if (!tc_available()) return MOSAIC_ERR_UNSUPPORTED;
+    const int64_t Kp = (K + 7) / 8 * 8;
+    if (!aligned16(A) || !aligned16(B) || lda % 4 || ldb % 4) return MOSAIC_ERR_ALIGN;
+    if (K % 8) return MOSAIC_ERR_SHAPE;
+    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    uint16_t *Ap = cv.take<uint16_t>((size_t)(4 * M * Kp));
+    uint16_t *Bp = cv.take<uint16_t>((size_t)(4 * N * Kp));
+    if (!Ap || !Bp) return MOSAIC_ERR_WORKSPACE;
+    MOSAIC_TRY(digit_split(A, lda, M, K, Ap, Kp, M * Kp, st));
+    MOSAIC_TRY(digit_split(B, ldb, N, K, Bp, Kp, N * Kp, st));
+    return ring_gemm_tc_planes(Ap, Kp, M * Kp, Bp, Kp, N * Kp, C, ldc, nullptr, 0, 1, M, N, K, st);
+}
+
+mosaic_status mosaic_ring_gemm_planes(const uint16_t *A_planes, int64_t ldpa, int64_t a_plane,
+                                      const uint16_t *B_planes, int64_t ldpb, int64_t b_plane,
+                                      uint32_t *C, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                                      int variant, void *stream) {
+    if (M < 0 || N < 0 || K < 0 || K > ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
+    if (ldpa < K || ldpb < K || ldc < N || a_plane < M * ldpa || b_plane < N * ldpb)
+        return MOSAIC_ERR_SHAPE;
+    if (variant != MOSAIC_GEMM_TC && variant != MOSAIC_GEMM_AUTO) return MOSAIC_ERR_UNSUPPORTED;
+    if (M == 0 || N == 0) return MOSAIC_OK;
+    if (!A_planes || !B_planes || !C) return MOSAIC_ERR_ARG;
+    if (!aligned16(A_planes) || !aligned16(B_planes) || ldpa % 8 || ldpb % 8 || a_plane % 8 ||
+        b_plane % 8)
+        return MOSAIC_ERR_ALIGN;
+    if (!tc_available()) return MOSAIC_ERR_UNSUPPORTED;
+    return ring_gemm_tc_planes(A_planes, ldpa, a_plane, B_planes, ldpb, b_plane, C, ldc, nullptr, 0,
+                               1, M, N, K, as_stream(stream));
+}
+
+size_t mosaic_workspace_bytes(int op, int64_t m, int64_t n_pad, int64_t l, const mosaic_params *p) {
+    if (m < 0 || n_pad < 0 || l < 0) return 0;
+    switch (op) {
+        case MOSAIC_OP_RING_GEMM: return ws_gemm(m, n_pad, l);
+        case MOSAIC_OP_MASK_CHAINS: return check_params(p) == MOSAIC_OK ? ws_chains(n_pad, p) : 0;
+        case MOSAIC_OP_MASK_WEIGHT: return check_params(p) == MOSAIC_OK ? ws_weight(m, n_pad, p) : 0;
+        case MOSAIC_OP_MASK_ACTIVATION:
+            return check_params(p) == MOSAIC_OK ? ws_activation(l, n_pad, p) : 0;
+        case MOSAIC_OP_UNMASK: return check_params(p) == MOSAIC_OK ? ws_unmask(m, l, p) : 0;
+    }
+    return 0;
+}
+
+mosaic_status mosaic_mask_chains(const mosaic_params *p, const mosaic_key *key, uint64_t chain_id,
+                                 int64_t n_pad, uint32_t *P, uint32_t *C, uint32_t *CT, void *ws,
+                                 size_t ws_bytes, void *stream) {
+    MOSAIC_TRY(check_params(p));
+    if (!key) return MOSAIC_ERR_ARG;
+    if (!is_pow2(n_pad) || n_pad > 32768 || n_pad < 32) return MOSAIC_ERR_SHAPE;
+    if (!P || !C || !CT) return MOSAIC_ERR_ARG;
+    if (ws_bytes < ws_chains(n_pad, p)) return MOSAIC_ERR_WORKSPACE;
+    cudaStream_t st = as_stream(stream);
+    const Key k = to_key(key);
+    const int R = (int)p->rounds;
+    const int64_t Sr = sum_r(p);
+    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    // Level 1: M_1 (r_1 x n_pad) is P_1; N_1 (n_pad x r_1) is C_1.
+    MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_M, 1), chain_id, R, p->r[0], n_pad, P, n_pad, st));
+    MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_N, 1), chain_id, R, n_pad, p->r[0], C, Sr, st));
+    for (uint32_t i = 2; i <= p->d; i++) {
+        const int64_t ri = p->r[i - 1], rp = p->r[i - 2];
+        const int64_t oi = off_r(p, i), op = off_r(p, i - 1);
+        uint32_t *Mi = cv.take<uint32_t>((size_t)(ri * rp));
+        uint32_t *Ni = cv.take<uint32_t>((size_t)(rp * ri));
+        if (!Mi || !Ni) return MOSAIC_ERR_WORKSPACE;
+        MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_M, i), chain_id, R, ri, rp, Mi, rp, st));
+        MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_N, i), chain_id, R, rp, ri, Ni, ri, st));
+        // P_i = M_i P_{i-1}:  C(a, c) = sum_b M_i[a][b] P_{i-1}[b][c]
+        MOSAIC_TRY(ring_gemm_imad(Mi, rp, 1, P + op * n_pad, 1, n_pad, P + oi * n_pad, n_pad,
+                                  nullptr, 0, 1, ri, n_pad, rp, st));
+        // C_i = C_{i-1} N_i:  C(c, b) = sum_a C_{i-1}[c][a] N_i[a][b]
+        MOSAIC_TRY(ring_gemm_imad(C + op, Sr, 1, Ni, 1, ri, C + oi, Sr, nullptr, 0, 1, n_pad, ri,
+                                  rp, st));
+    }
+    return transpose_u32(C, Sr, n_pad, Sr, CT, n_pad, st);
+}
+
+mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, uint64_t matrix_id,
+                                 const float *W, int64_t ldw, int64_t m, int64_t n, int64_t n_pad,
+                                 const uint32_t *P, const uint32_t *CT, uint32_t *sign_words,
+                                 float *s_w, uint32_t *L, uint32_t *S_idx, uint32_t *S_val,
+                                 uint32_t *Wp, uint16_t *Wp_planes, uint32_t *J, int variant,
+                                 void *ws, size_t ws_bytes, void *stream) {
+    MOSAIC_TRY(check_params(p));
+    if (!key) return MOSAIC_ERR_ARG;
+    if (!npad_ok(n_pad) || n < 1 || n > n_pad || m < 1 || ldw < n || m >= ((int64_t)1 << 20))
+        return MOSAIC_ERR_SHAPE;
+    if (!W || !P || !CT || !sign_words || !s_w || !L || !Wp || !J) return MOSAIC_ERR_ARG;
+    if (p->d > 1 && (!S_idx || !S_val)) return MOSAIC_ERR_ARG;
+    if (!aligned16(Wp) || (Wp_planes && !aligned16(Wp_planes))) return MOSAIC_ERR_ALIGN;
+    if (ws_bytes < ws_weight(m, n_pad, p)) return MOSAIC_ERR_WORKSPACE;
+    cudaStream_t st = as_stream(stream);
+    const Key k = to_key(key);
+    const int R = (int)p->rounds;
+    const uint32_t d = p->d;
+    const int64_t Sr = sum_r(p), rd = p->r[d - 1], od = off_r(p, d);
+    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    uint32_t *WE = cv.take<uint32_t>((size_t)(m * n_pad));
+    if (!WE) return MOSAIC_ERR_WORKSPACE;
+
+    // Pi_Sec-Linear Init W: d, then rows of W R^T quantised into W_hat (rows [0, m) of Wp).
+    MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_SIGN, 0), matrix_id, R, 1, n_pad / 32, sign_words,
+                           n_pad / 32, st));
+    const int32_t qmax = mosaic_qmax(n_pad, p->qbits);
+    MOSAIC_TRY(fwht_encode(W, ldw, m, n, n_pad, sign_words, 1, 1, nullptr, qmax, nullptr, 0, Wp,
+                           n_pad, s_w, nullptr, st));
+    // E_w and W_hat + E_w.
+    MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EW, 0), matrix_id, R, p->sigma, m * n_pad, WE, st));
+    MOSAIC_TRY(add_u32(Wp, n_pad, WE, n_pad, WE, n_pad, m, n_pad, st));
+    // J_i = (W_hat + E_w) C_i for all i at once: J = WE CT^T (m x Sr).
+    MOSAIC_TRY(gemm_u32(variant, WE, n_pad, 1, CT, n_pad, 1, J, Sr, nullptr, 0, 1, m, Sr, n_pad, st));
+    // L, S_{i+1}.
+    MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_L, 0), matrix_id, R, m, rd, L, rd, st));
+    SparseLevel lev[2];
+    int64_t soff = 0;
+    for (uint32_t i = 1; i < d; i++) {
+        const uint32_t t = p->t[i], ri = p->r[i - 1];
+        MOSAIC_TRY(prg_sparse(k, tag_of(MOSAIC_TAG_S, i + 1), matrix_id, R, m, ri, t, S_idx + soff,
+                              S_val + soff, nullptr, st));
+        lev[i - 1] = SparseLevel{S_idx + soff, S_val + soff, (int)t, off_r(p, i), ri};
+        soff += m * t;
+    }
+    // W' = (W_hat + E_w) + L P_d + sum_i S_{i+1} P_i.
+    MOSAIC_TRY(gemm_u32(variant, L, rd, 1, P + od * n_pad, 1, n_pad, Wp, n_pad, WE, n_pad, 1, m,
+                        n_pad, rd, st));
+    if (d > 1)
+        MOSAIC_TRY(sparse_rowgather(P, n_pad, lev, (int)d - 1, m, n_pad, Wp, n_pad, Wp, n_pad, st));
+    // The server operand carries the public chains below W'.
+    if (cudaMemcpyAsync(Wp + m * n_pad, P, sizeof(uint32_t) * (size_t)(Sr * n_pad),
+                        cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+        return MOSAIC_ERR_CUDA;
+    if (Wp_planes)
+        MOSAIC_TRY(digit_split(Wp, n_pad, m + Sr, n_pad, Wp_planes, n_pad, (m + Sr) * n_pad, st));
+    return MOSAIC_OK;
+}
+
+mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *key,
+                                     uint64_t pass_id, int64_t m, int64_t n_pad, int64_t l,
+                                     const uint32_t *C, const uint32_t *J, uint32_t *Ux_tm,
+                                     uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
+                                     void *stream) {
+    MOSAIC_TRY(check_params(p));
+    if (!key) return MOSAIC_ERR_ARG;
+    if (!npad_ok(n_pad) || m < 1 || l < 0 || l >= ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
+    if (l == 0) return MOSAIC_OK;
+    if (!C || !J || !Ux_tm || !K_tm) return MOSAIC_ERR_ARG;
+    if (ws_bytes < ws_activation(l, n_pad, p)) return MOSAIC_ERR_WORKSPACE;
+    cudaStream_t st = as_stream(stream);
+    const Key k = to_key(key);
+    const int R = (int)p->rounds;
+    const uint32_t d = p->d;
+    const int64_t Sr = sum_r(p), rd = p->r[d - 1], od = off_r(p, d);
+    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    uint32_t *Rt = cv.take<uint32_t>((size_t)(l * rd));
+    if (!Rt) return MOSAIC_ERR_WORKSPACE;
+    MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_R, 0), pass_id, R, l, rd, Rt, rd, st));
+    SparseLevel lev[2];
+    for (uint32_t i = 1; i < d; i++) {
+        const uint32_t t = p->t[i], ri = p->r[i - 1];
+        uint32_t *ti = cv.take<uint32_t>((size_t)(l * t));
+        uint32_t *tv = cv.take<uint32_t>((size_t)(l * t));
+        if (!ti || !tv) return MOSAIC_ERR_WORKSPACE;
+        MOSAIC_TRY(prg_sparse(k, tag_of(MOSAIC_TAG_T, i + 1), pass_id, R, l, ri, t, ti, tv, nullptr, st));
+        lev[i - 1] = SparseLevel{ti, tv, (int)t, off_r(p, i), ri};
+    }
+    // U_x^T = E_x^T + R^T C_d^T + sum_i T_{i+1}^T C_i^T.
+    MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EX, 0), pass_id, R, p->sigma, l * n_pad, Ux_tm, st));
+    MOSAIC_TRY(gemm_u32(variant, Rt, rd, 1, C + od, Sr, 1, Ux_tm, n_pad, Ux_tm, n_pad, 1, l, n_pad,
+                        rd, st));
+    if (d > 1)
+        MOSAIC_TRY(sparse_gather(C, Sr, 0, od, n_pad, l, false, lev, (int)d - 1, Ux_tm, n_pad,
+                                 nullptr, 0, 1, Ux_tm, n_pad, st));
+    // K^T = R^T J_d^T + sum_i T_{i+1}^T J_i^T.
+    MOSAIC_TRY(gemm_u32(variant, Rt, rd, 1, J + od, Sr, 1, K_tm, m, nullptr, 0, 1, l, m, rd, st));
+    if (d > 1)
+        MOSAIC_TRY(sparse_gather(J, Sr, 0, od, m, l, false, lev, (int)d - 1, K_tm, m, nullptr, 0, 1,
+                                 K_tm, m, st));
+    return MOSAIC_OK;
+}
+
+mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z,
+                            int64_t ldz, const uint32_t *K_tm, const uint32_t *L,
+                            const uint32_t *S_idx, const uint32_t *S_val, const float *s_w,
+                            const float *s_x, const float *bias, float *Y, uint32_t *Yhat,
+                            int64_t ldy, int variant, void *ws, size_t ws_bytes, void *stream) {
+    MOSAIC_TRY(check_params(p));
+    const uint32_t d = p->d;
+    const int64_t Sr = sum_r(p), rd = p->r[d - 1], od = off_r(p, d);
+    if (l < 0 || m < 1 || ldz < m + Sr || ldy < m) return MOSAIC_ERR_SHAPE;
+    if (l == 0) return MOSAIC_OK;
+    if (!Z || !K_tm || !L || !s_w || !s_x || !Y) return MOSAIC_ERR_ARG;
+    if (d > 1 && (!S_idx || !S_val)) return MOSAIC_ERR_ARG;
+    if (ws_bytes < ws_unmask(m, l, p)) return MOSAIC_ERR_WORKSPACE;
+    cudaStream_t st = as_stream(stream);
+    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    uint32_t *tmp = cv.take<uint32_t>((size_t)(l * m));
+    if (!tmp) return MOSAIC_ERR_WORKSPACE;
+    // tmp = K + Q_d L^T  (token-major: Q_d^T is the column block [m + od, m + Sr) of Z).
+    MOSAIC_TRY(gemm_u32(variant, Z + m + od, ldz, 1, L, rd, 1, tmp, m, K_tm, m, 1, l, m, rd, st));
+    SparseLevel lev[2];
+    int64_t soff = 0;
+    for (uint32_t i = 1; i < d; i++) {
+        const uint32_t t = p->t[i], ri = p->r[i - 1];
+        lev[i - 1] = SparseLevel{S_idx + soff, S_val + soff, (int)t, m + off_r(p, i), ri};
+        soff += m * t;
+    }
+    // Y_hat = Y' - tmp - sum_i S_{i+1} Q_i, then decode.
+    return unmask_decode(Z, ldz, m, od, l, m, lev, (int)d - 1, tmp, m, s_w, s_x, bias, Y, Yhat, ldy,
+                         st);
+}
+
+}  // extern "C"

@@ -1,0 +1,358 @@
+// Random Hadamard rotation R = H D fused with per-row quantisation and the
+// mask-add (Sec. 4 "Random Hadamard rotation"; Pi_Sec-Linear box, Init W
+// steps 1-2 and Online step 1; Approx-MatMul Online step 2).
+//
+// One row of n_pad = E * T fp32 values is held in registers by T threads
+// (E consecutive elements each).  The butterfly stages run in the order
+// h = 1, 2, ..., n_pad / 2 -- the same order as the plain radix-2 FWHT --
+// so every output is rounded exactly like the textbook transform:
+//   h <  E        inside a thread's registers,
+//   E <= h < 32E  across lanes with warp shuffles,
+//   h >= 32E      after one transpose through shared memory, again in
+//                 registers (each thread then holds E / WN elements of each of
+//                 the WN warp-sized segments).
+// HBM traffic per row: read n floats (+ n mask words), write n_pad words
+// (+ 4 bf16 digit planes when requested).
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "mosaic_internal.cuh"
+
+namespace mosaic {
+namespace {
+
+struct FwhtArgs {
+    const float *x;
+    int64_t ldx;
+    int64_t rows;
+    int64_t n;
+    int64_t n_pad;
+    const uint32_t *signs;
+    int rotate;
+    int mode;          // 0: write y (fp32); 1: encode
+    float inv_sqrt;    // fl32(1 / sqrt(n_pad))
+    float *y;
+    int32_t qmax;
+    const uint32_t *mask;
+    int64_t ldm;
+    uint32_t *out;
+    int64_t ldo;
+    float *scale;
+    uint16_t *planes;  // [4][rows][n_pad]
+    int vec_x;         // x rows 16-byte aligned
+};
+
+__device__ __forceinline__ int pad_idx(int i) { return i + (i >> 5); }
+
+// Signed base-2^8 digit i of a (b = a + 0x80808080; digit = byte_i(b) - 128)
+// as bf16 bits.  Digits in [-128, 127] are exact in bf16.
+__device__ __forceinline__ uint16_t digit_bf16(uint32_t a, int i) {
+    const uint32_t b = a + 0x80808080u;
+    const int d = (int)((b >> (8 * i)) & 0xffu) - 128;
+    return __bfloat16_as_ushort(__float2bfloat16_rn((float)d));
+}
+
+template <int CNT>
+__device__ __forceinline__ void store_f32(float *p, const float *v) {
+    if constexpr (CNT % 4 == 0) {
+#pragma unroll
+        for (int q = 0; q < CNT; q += 4) *reinterpret_cast<float4 *>(p + q) = make_float4(v[q], v[q + 1], v[q + 2], v[q + 3]);
+    } else if constexpr (CNT == 2) {
+        *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
+    } else {
+#pragma unroll
+        for (int q = 0; q < CNT; q++) p[q] = v[q];
+    }
+}
+
+template <int CNT>
+__device__ __forceinline__ void store_u32(uint32_t *p, const uint32_t *v) {
+    if constexpr (CNT % 4 == 0) {
+#pragma unroll
+        for (int q = 0; q < CNT; q += 4) *reinterpret_cast<uint4 *>(p + q) = make_uint4(v[q], v[q + 1], v[q + 2], v[q + 3]);
+    } else if constexpr (CNT == 2) {
+        *reinterpret_cast<uint2 *>(p) = make_uint2(v[0], v[1]);
+    } else {
+#pragma unroll
+        for (int q = 0; q < CNT; q++) p[q] = v[q];
+    }
+}
+
+template <int CNT>
+__device__ __forceinline__ void load_u32(const uint32_t *p, uint32_t *v) {
+    if constexpr (CNT % 4 == 0) {
+#pragma unroll
+        for (int q = 0; q < CNT; q += 4) {
+            uint4 t = *reinterpret_cast<const uint4 *>(p + q);
+            v[q] = t.x; v[q + 1] = t.y; v[q + 2] = t.z; v[q + 3] = t.w;
+        }
+    } else if constexpr (CNT == 2) {
+        uint2 t = *reinterpret_cast<const uint2 *>(p);
+        v[0] = t.x; v[1] = t.y;
+    } else {
+#pragma unroll
+        for (int q = 0; q < CNT; q++) v[q] = p[q];
+    }
+}
+
+template <int CNT>
+__device__ __forceinline__ void store_planes(uint16_t *p, int64_t plane_stride, const uint32_t *code) {
+#pragma unroll
+    for (int d = 0; d < 4; d++) {
+        uint16_t h[CNT];
+#pragma unroll
+        for (int q = 0; q < CNT; q++) h[q] = digit_bf16(code[q], d);
+        uint16_t *pd = p + d * plane_stride;
+        if constexpr (CNT % 8 == 0) {
+#pragma unroll
+            for (int q = 0; q < CNT; q += 8) {
+                uint4 t;
+                t.x = h[q] | ((uint32_t)h[q + 1] << 16);
+                t.y = h[q + 2] | ((uint32_t)h[q + 3] << 16);
+                t.z = h[q + 4] | ((uint32_t)h[q + 5] << 16);
+                t.w = h[q + 6] | ((uint32_t)h[q + 7] << 16);
+                *reinterpret_cast<uint4 *>(pd + q) = t;
+            }
+        } else if constexpr (CNT == 4) {
+            uint2 t;
+            t.x = h[0] | ((uint32_t)h[1] << 16);
+            t.y = h[2] | ((uint32_t)h[3] << 16);
+            *reinterpret_cast<uint2 *>(pd) = t;
+        } else if constexpr (CNT == 2) {
+            *reinterpret_cast<uint32_t *>(pd) = h[0] | ((uint32_t)h[1] << 16);
+        } else {
+#pragma unroll
+            for (int q = 0; q < CNT; q++) pd[q] = h[q];
+        }
+    }
+}
+
+template <int E, int T>
+struct Cfg {
+    static constexpr int N = E * T;
+    static constexpr int RPB = T >= 256 ? 1 : 256 / T;   // rows per block
+    static constexpr int WN = T / 32;                     // warps per row
+    static constexpr int CS = WN > 1 ? E / WN : E;        // run length per thread after phase 3
+    static constexpr int RUNS = E / CS;                   // runs per thread
+    static constexpr int SMEM_ROW = WN > 1 ? N + N / 32 : 0;
+    static constexpr size_t SMEM = (size_t)RPB * SMEM_ROW * sizeof(float);
+};
+
+template <int E, int T>
+__global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
+    using C = Cfg<E, T>;
+    constexpr int N = C::N, WN = C::WN, CS = C::CS, RUNS = C::RUNS;
+    static_assert(WN == 1 || E >= WN, "phase-3 layout needs E >= warps per row");
+    extern __shared__ float smem[];
+    __shared__ float red_max[C::RPB][WN];
+    __shared__ int red_ok[C::RPB][WN];
+
+    const int lt = threadIdx.x % T;
+    const int rb = threadIdx.x / T;
+    const int lane = threadIdx.x & 31;
+    const int64_t row = (int64_t)blockIdx.x * C::RPB + rb;
+    const bool active = row < a.rows;
+    const int base = lt * E;
+
+    float v[E];
+    if (active) {
+        const float *xr = a.x + row * a.ldx;
+        if (E % 4 == 0 && a.vec_x && base + E <= a.n) {
+#pragma unroll
+            for (int q = 0; q < E; q += 4) {
+                float4 t = *reinterpret_cast<const float4 *>(xr + base + q);
+                v[q] = t.x; v[q + 1] = t.y; v[q + 2] = t.z; v[q + 3] = t.w;
+            }
+        } else {
+#pragma unroll
+            for (int e = 0; e < E; e++) v[e] = (base + e < a.n) ? xr[base + e] : 0.0f;
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < E; e++) v[e] = 0.0f;
+    }
+
+    if (a.rotate) {
+        if (a.signs) {
+            const uint32_t w = a.signs[base >> 5] >> (base & 31);
+#pragma unroll
+            for (int e = 0; e < E; e++)
+                if ((w >> e) & 1u) v[e] = -v[e];
+        }
+        // Phase 1: h = 1 .. E/2 in registers.
+#pragma unroll
+        for (int h = 1; h < E; h <<= 1) {
+#pragma unroll
+            for (int i = 0; i < E; i += 2 * h) {
+#pragma unroll
+                for (int j = i; j < i + h; j++) {
+                    const float p = v[j], q = v[j + h];
+                    v[j] = __fadd_rn(p, q);
+                    v[j + h] = __fsub_rn(p, q);
+                }
+            }
+        }
+        // Phase 2: h = E .. 16E across lanes.
+#pragma unroll
+        for (int hl = 1; hl < 32; hl <<= 1) {
+            const bool upper = (lane & hl) != 0;
+#pragma unroll
+            for (int e = 0; e < E; e++) {
+                const float o = __shfl_xor_sync(0xffffffffu, v[e], hl);
+                v[e] = upper ? __fsub_rn(o, v[e]) : __fadd_rn(v[e], o);
+            }
+        }
+    }
+
+    // Phase 3: h = 32E .. N/2 after a transpose through shared memory.  The
+    // transpose runs whether or not the row is rotated, so that the output
+    // layout below is the same in both cases.
+    if constexpr (WN > 1) {
+        float *buf = smem + rb * C::SMEM_ROW;
+#pragma unroll
+        for (int e = 0; e < E; e++) buf[pad_idx(base + e)] = v[e];
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < WN; j++)
+#pragma unroll
+            for (int u = 0; u < CS; u++) v[j * CS + u] = buf[pad_idx(j * 32 * E + lt * CS + u)];
+        if (a.rotate) {
+#pragma unroll
+            for (int hj = 1; hj < WN; hj <<= 1) {
+#pragma unroll
+                for (int i = 0; i < WN; i += 2 * hj) {
+#pragma unroll
+                    for (int j = i; j < i + hj; j++) {
+#pragma unroll
+                        for (int u = 0; u < CS; u++) {
+                            const float p = v[j * CS + u], q = v[(j + hj) * CS + u];
+                            v[j * CS + u] = __fadd_rn(p, q);
+                            v[(j + hj) * CS + u] = __fsub_rn(p, q);
+                        }
+                    }
+                }
+            }
+        }
+    }
+    if (a.rotate) {
+#pragma unroll
+        for (int e = 0; e < E; e++) v[e] = __fmul_rn(v[e], a.inv_sqrt);
+    }
+
+    // Element index of v[run * CS + u].
+    auto elem = [&](int run) -> int {
+        if constexpr (WN > 1) return run * 32 * E + lt * CS;
+        else return base;
+    };
+    (void)elem;
+
+    if (a.mode == 0) {
+        if (active) {
+            float *yr = a.y + row * a.n_pad;
+#pragma unroll
+            for (int run = 0; run < RUNS; run++) store_f32<CS>(yr + elem(run), v + run * CS);
+        }
+        return;
+    }
+
+    // Encode: per-row absmax (and finiteness) reduction.
+    float mx = 0.0f;
+    int ok = 1;
+#pragma unroll
+    for (int e = 0; e < E; e++) {
+        ok &= isfinite(v[e]) ? 1 : 0;
+        mx = fmaxf(mx, fabsf(v[e]));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        ok &= __shfl_xor_sync(0xffffffffu, ok, o);
+    }
+    if constexpr (WN > 1) {
+        const int wr = lt >> 5;
+        if (lane == 0) { red_max[rb][wr] = mx; red_ok[rb][wr] = ok; }
+        __syncthreads();
+#pragma unroll
+        for (int w = 0; w < WN; w++) { mx = fmaxf(mx, red_max[rb][w]); ok &= red_ok[rb][w]; }
+    }
+    if (!active) return;
+    const float s = ok ? __fdiv_rn(mx, (float)a.qmax) : __int_as_float(0x7fc00000);
+    if (lt == 0) a.scale[row] = s;
+    const float q = (float)a.qmax;
+    uint32_t code[E];
+#pragma unroll
+    for (int e = 0; e < E; e++) {
+        int32_t c = 0;
+        if (ok && s != 0.0f) {
+            float f = rintf(__fdiv_rn(v[e], s));
+            f = fminf(fmaxf(f, -q), q);
+            c = (int32_t)f;
+        }
+        code[e] = (uint32_t)c;
+    }
+    if (a.mask) {
+        const uint32_t *mr = a.mask + row * a.ldm;
+#pragma unroll
+        for (int run = 0; run < RUNS; run++) {
+            uint32_t mk[CS];
+            load_u32<CS>(mr + elem(run), mk);
+#pragma unroll
+            for (int u = 0; u < CS; u++) code[run * CS + u] += mk[u];
+        }
+    }
+    uint32_t *orow = a.out + row * a.ldo;
+#pragma unroll
+    for (int run = 0; run < RUNS; run++) store_u32<CS>(orow + elem(run), code + run * CS);
+    if (a.planes) {
+        const int64_t ps = a.rows * a.n_pad;
+        uint16_t *prow = a.planes + row * a.n_pad;
+#pragma unroll
+        for (int run = 0; run < RUNS; run++) store_planes<CS>(prow + elem(run), ps, code + run * CS);
+    }
+}
+
+template <int E, int T>
+mosaic_status launch(const FwhtArgs &a, cudaStream_t st) {
+    using C = Cfg<E, T>;
+    static_assert(C::N >= 32, "");
+    if (C::SMEM > 48 * 1024) {
+        if (cudaFuncSetAttribute(fwht_kernel<E, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)C::SMEM) != cudaSuccess)
+            return MOSAIC_ERR_CUDA;
+    }
+    const int64_t blocks = (a.rows + C::RPB - 1) / C::RPB;
+    fwht_kernel<E, T><<<(unsigned)blocks, T * C::RPB, C::SMEM, st>>>(a);
+    return launch_status();
+}
+
+}  // namespace
+
+mosaic_status fwht_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, int64_t n_pad,
+                          const uint32_t *sign_words, int rotate, int mode, float *y, int32_t qmax,
+                          const uint32_t *mask, int64_t ldm, uint32_t *out, int64_t ldo, float *scale,
+                          uint16_t *planes, cudaStream_t st) {
+    if (rows == 0) return MOSAIC_OK;
+    FwhtArgs a;
+    a.x = x; a.ldx = ldx; a.rows = rows; a.n = n; a.n_pad = n_pad;
+    a.signs = sign_words; a.rotate = rotate; a.mode = mode;
+    a.inv_sqrt = (float)(1.0 / sqrt((double)n_pad));
+    a.y = y; a.qmax = qmax; a.mask = mask; a.ldm = ldm; a.out = out; a.ldo = ldo;
+    a.scale = scale; a.planes = planes;
+    a.vec_x = aligned16(x) && (ldx % 4 == 0);
+    switch (n_pad) {
+        case 32: return launch<1, 32>(a, st);
+        case 64: return launch<2, 32>(a, st);
+        case 128: return launch<4, 32>(a, st);
+        case 256: return launch<8, 32>(a, st);
+        case 512: return launch<16, 32>(a, st);
+        case 1024: return launch<16, 64>(a, st);
+        case 2048: return launch<16, 128>(a, st);
+        case 4096: return launch<16, 256>(a, st);
+        case 8192: return launch<32, 256>(a, st);
+        case 16384: return launch<32, 512>(a, st);
+        case 32768: return launch<32, 1024>(a, st);
+        default: return MOSAIC_ERR_SHAPE;
+    }
+}
+
+}  // namespace mosaic

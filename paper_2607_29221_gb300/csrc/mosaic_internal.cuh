@@ -1,0 +1,146 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/mosaic.h"
+
+namespace mosaic {
+
+constexpr int kSparseWindow = 65536;   // stream words reserved per sparse row
+constexpr int kMaxGaussBound = 96;     // B = ceil(12 sigma) for sigma <= 8
+
+// ChaCha quarter round and block (RFC 8439 Sec. 2.1-2.3).
+__device__ __forceinline__ uint32_t rotl(uint32_t v, int c) { return __funnelshift_l(v, v, c); }
+
+#define MOSAIC_QR(a, b, c, d)             \
+    a += b; d ^= a; d = rotl(d, 16);      \
+    c += d; b ^= c; b = rotl(b, 12);      \
+    a += b; d ^= a; d = rotl(d, 8);       \
+    c += d; b ^= c; b = rotl(b, 7);
+
+struct Key {
+    uint32_t k[8];
+};
+
+// Block `ctr` of stream (n0, n1, n2) -> 16 words in `o`.
+__device__ __forceinline__ void chacha_block(const Key &key, uint32_t ctr, uint32_t n0, uint32_t n1,
+                                             uint32_t n2, int rounds, uint32_t o[16]) {
+    uint32_t x0 = 0x61707865u, x1 = 0x3320646eu, x2 = 0x79622d32u, x3 = 0x6b206574u;
+    uint32_t x4 = key.k[0], x5 = key.k[1], x6 = key.k[2], x7 = key.k[3];
+    uint32_t x8 = key.k[4], x9 = key.k[5], x10 = key.k[6], x11 = key.k[7];
+    uint32_t x12 = ctr, x13 = n0, x14 = n1, x15 = n2;
+    for (int r = 0; r < rounds; r += 2) {
+        MOSAIC_QR(x0, x4, x8, x12);
+        MOSAIC_QR(x1, x5, x9, x13);
+        MOSAIC_QR(x2, x6, x10, x14);
+        MOSAIC_QR(x3, x7, x11, x15);
+        MOSAIC_QR(x0, x5, x10, x15);
+        MOSAIC_QR(x1, x6, x11, x12);
+        MOSAIC_QR(x2, x7, x8, x13);
+        MOSAIC_QR(x3, x4, x9, x14);
+    }
+    o[0] = x0 + 0x61707865u; o[1] = x1 + 0x3320646eu; o[2] = x2 + 0x79622d32u; o[3] = x3 + 0x6b206574u;
+    o[4] = x4 + key.k[0]; o[5] = x5 + key.k[1]; o[6] = x6 + key.k[2]; o[7] = x7 + key.k[3];
+    o[8] = x8 + key.k[4]; o[9] = x9 + key.k[5]; o[10] = x10 + key.k[6]; o[11] = x11 + key.k[7];
+    o[12] = x12 + ctr; o[13] = x13 + n0; o[14] = x14 + n1; o[15] = x15 + n2;
+}
+
+inline Key to_key(const mosaic_key *k) {
+    Key r;
+    for (int i = 0; i < 8; i++) r.k[i] = k->key[i];
+    return r;
+}
+
+inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
+
+inline mosaic_status launch_status() {
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
+}
+
+#define MOSAIC_TRY(expr)                        \
+    do {                                        \
+        mosaic_status _s = (expr);              \
+        if (_s != MOSAIC_OK) return _s;         \
+    } while (0)
+
+inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline bool is_pow2(int64_t v) { return v > 0 && (v & (v - 1)) == 0; }
+
+// ---- internal launchers (all enqueue on `st`, validate nothing beyond what they state) ----
+
+// Uniform words: out[i * ldo + j] = word (i * cols + j).
+mosaic_status prg_uniform(const Key &key, uint32_t tag, uint64_t sid, int rounds, int64_t rows,
+                          int64_t cols, uint32_t *out, int64_t ldo, cudaStream_t st);
+// Discrete Gaussian elements.
+mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int rounds, float sigma,
+                           int64_t count, uint32_t *out, cudaStream_t st);
+// Sparse rows.
+mosaic_status prg_sparse(const Key &key, uint32_t tag, uint64_t sid, int rounds, int64_t rows,
+                         uint32_t r, uint32_t t, uint32_t *idx, uint32_t *val, uint32_t *fail,
+                         cudaStream_t st);
+// Host-side Gaussian CDF table (long double), B = ceil(12 sigma); returns B.
+int gaussian_table_host(float sigma, unsigned long long *table /* 2*kMaxGaussBound+1 */);
+
+// FWHT / encode.
+mosaic_status fwht_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, int64_t n_pad,
+                          const uint32_t *sign_words, int rotate, int mode /*0 hadamard,1 encode*/,
+                          float *y, int32_t qmax, const uint32_t *mask, int64_t ldm, uint32_t *out,
+                          int64_t ldo, float *scale, uint16_t *planes, cudaStream_t st);
+
+// Generic strided ring GEMM on CUDA cores:
+// C[i*ldc + j] = (Cin ? Cin[i*ldcin + j] : 0) + sgn * sum_k A[i*sai + k*sak] * B[j*sbj + k*sbk]
+mosaic_status ring_gemm_imad(const uint32_t *A, int64_t sai, int64_t sak, const uint32_t *B,
+                             int64_t sbj, int64_t sbk, uint32_t *C, int64_t ldc,
+                             const uint32_t *Cin, int64_t ldcin, int sgn, int64_t M, int64_t N,
+                             int64_t K, cudaStream_t st);
+
+// Digit planes.
+mosaic_status digit_split(const uint32_t *a, int64_t lda, int64_t rows, int64_t cols,
+                          uint16_t *planes, int64_t ldp, int64_t plane_stride, cudaStream_t st);
+
+// Tensor-core ring GEMM from planes (NT, K-major planes); C = (Cin?) + sgn * A B^T.
+mosaic_status ring_gemm_tc_planes(const uint16_t *Ap, int64_t ldpa, int64_t a_plane,
+                                  const uint16_t *Bp, int64_t ldpb, int64_t b_plane, uint32_t *C,
+                                  int64_t ldc, const uint32_t *Cin, int64_t ldcin, int sgn,
+                                  int64_t M, int64_t N, int64_t K, cudaStream_t st);
+// Legacy mma.sync s8 ring GEMM from int8 digits packed in uint32 operands (NT).
+mosaic_status ring_gemm_mma_s8(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb,
+                               uint32_t *C, int64_t ldc, const uint32_t *Cin, int64_t ldcin,
+                               int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st);
+bool tc_available();
+bool mma_s8_available();
+
+// Sparse gathers.
+// out[row][col] = a[row][col] - b[row][col] (b nullable) + sgn * sum_lev sum_q val * src[g][off_lev + idx]
+// where (list entity, staged row g) = (row, col) if !list_is_col else (col, row).
+struct SparseLevel {
+    const uint32_t *idx;   // nlist x t
+    const uint32_t *val;
+    int t;
+    int64_t off;           // offset of this level's segment (columns of src, or rows of P)
+    uint32_t r;            // positions are < r; larger ones are skipped
+};
+mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, int64_t seg_len,
+                            int64_t g_count, int64_t nlist, bool list_is_col, const SparseLevel *lev,
+                            int nlev, const uint32_t *a, int64_t lda, const uint32_t *b, int64_t ldb,
+                            int sgn, uint32_t *out, int64_t ldo, cudaStream_t st);
+// Unmask epilogue: list = output column j; staged rows = tokens k of Z.
+mosaic_status unmask_decode(const uint32_t *Z, int64_t ldz, int64_t seg_off, int64_t seg_len,
+                            int64_t l, int64_t m, const SparseLevel *lev, int nlev,
+                            const uint32_t *tmp, int64_t ldt, const float *s_w, const float *s_x,
+                            const float *bias, float *Y, uint32_t *Yhat, int64_t ldy,
+                            cudaStream_t st);
+// out[j][c] = a[j][c] + sum_lev sum_q val[j][q] * P[(row_off_lev + idx[j][q]) * ldp + c]
+mosaic_status sparse_rowgather(const uint32_t *P, int64_t ldp, const SparseLevel *lev, int nlev,
+                               int64_t m, int64_t ncols, const uint32_t *a, int64_t lda,
+                               uint32_t *out, int64_t ldo, cudaStream_t st);
+// Elementwise and layout helpers.
+mosaic_status add_u32(const uint32_t *a, int64_t lda, const uint32_t *b, int64_t ldb, uint32_t *out,
+                      int64_t ldo, int64_t rows, int64_t cols, cudaStream_t st);
+mosaic_status transpose_u32(const uint32_t *a, int64_t lda, int64_t rows, int64_t cols, uint32_t *out,
+                            int64_t ldo, cudaStream_t st);
+
+}  // namespace mosaic

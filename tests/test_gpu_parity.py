@@ -1,0 +1,286 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle on the
+same seeded inputs: bit-exact for every ring, integer and sampled output and
+for the fp32 rotation (same stage order); decoded floats within
+1e-6 x (|Y_hat s_w s_x| + |b|) of the oracle's fp64 decode."""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2607_29221_gb300 import workloads as wl
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+KEY = wl.mask_key()
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2607_29221_gb300 import build
+    build.build()
+    from paper_2607_29221_gb300 import mosaic as M
+    M.lib()
+    yield
+
+
+def M_():
+    from paper_2607_29221_gb300 import mosaic as M
+    return M
+
+
+def dev(a):
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint32:
+        a = a.view(np.int32)
+    return torch.from_numpy(a).cuda()
+
+
+def host_u32(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy().view(np.uint32)
+
+
+def host_f32(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+def ckey():
+    return M_().make_key(KEY)
+
+
+# --------------------------------------------------------------------------
+# Samplers
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("rows,cols,ld,rounds", [(1, 1, 1, 20), (3, 17, 20, 20), (65, 652, 652, 20),
+                                                 (1024, 1536, 1536, 20), (7, 33, 40, 8),
+                                                 (9, 31, 31, 12)])
+def test_prg_uniform(rows, cols, ld, rounds):
+    M = M_()
+    tg, sid = O.tag(O.KIND_L), 0x123456789
+    out = torch.full((rows, ld), -1, dtype=torch.int32, device="cuda")
+    M.mosaic_prg_uniform(ckey(), tg, sid, rounds, rows, cols, out, ld)
+    got = host_u32(out)
+    assert np.array_equal(got[:, :cols], O.sample_uniform(KEY, tg, sid, rows, cols, rounds))
+    assert np.all(got[:, cols:] == 0xFFFFFFFF)
+
+
+@pytest.mark.parametrize("sigma", [0.5, 1.0, 2.0, 0.0, 8.0])
+@pytest.mark.parametrize("count", [1, 7, 12345, 1 << 20])
+def test_prg_gaussian(sigma, count):
+    M = M_()
+    out = torch.full((count + 3,), 7, dtype=torch.int32, device="cuda")
+    M.mosaic_prg_gaussian(ckey(), O.tag(O.KIND_EW), 42, 20, sigma, count, out)
+    got = host_u32(out)
+    assert np.array_equal(got[:count], O.sample_gaussian(KEY, O.tag(O.KIND_EW), 42, count, sigma))
+    assert np.all(got[count:] == 7)
+
+
+@pytest.mark.parametrize("rows,r,t", [(1, 4, 2), (100, 1536, 80), (2049, 1024, 80), (33, 652, 1),
+                                      (5, 64, 32)])
+def test_prg_sparse(rows, r, t):
+    M = M_()
+    idx = torch.zeros(rows, t, dtype=torch.int32, device="cuda")
+    val = torch.zeros(rows, t, dtype=torch.int32, device="cuda")
+    fail = torch.zeros(1, dtype=torch.int32, device="cuda")
+    M.mosaic_prg_sparse(ckey(), O.tag(O.KIND_T, 2), 9, 20, rows, r, t, idx, val, fail)
+    wi, wv = O.sample_sparse(KEY, O.tag(O.KIND_T, 2), 9, rows, r, t)
+    assert np.array_equal(host_u32(idx), wi)
+    assert np.array_equal(host_u32(val), wv)
+    assert host_u32(fail)[0] == 0
+
+
+# --------------------------------------------------------------------------
+# Rotation and encoding
+# --------------------------------------------------------------------------
+NPADS = [32, 64, 128, 256, 512, 1024, 2048, 4096, 8192, 16384, 32768]
+
+
+@pytest.mark.parametrize("n_pad", NPADS)
+def test_hadamard_bit_exact(n_pad):
+    M = M_()
+    rows = 5 if n_pad >= 8192 else 19
+    for n in sorted({n_pad, max(1, n_pad - 3), n_pad // 2 + 1}):
+        x = wl.activations(rows, n, seed=n)
+        words = O.sample_signs(KEY, 11, n_pad)
+        y = torch.empty(rows, n_pad, dtype=torch.float32, device="cuda")
+        M.mosaic_hadamard(dev(x), n, y, rows, n, n_pad, dev(words))
+        want = O.fwht_rows(x, n_pad, words)
+        assert np.array_equal(host_f32(y).view(np.uint32), want.view(np.uint32)), n
+    # D = I and a row stride larger than n
+    x = wl.activations(3, n_pad + 8, seed=5)
+    y = torch.empty(3, n_pad, dtype=torch.float32, device="cuda")
+    M.mosaic_hadamard(dev(x), n_pad + 8, y, 3, n_pad, n_pad, None)
+    assert np.array_equal(host_f32(y), O.fwht_rows(x[:, :n_pad], n_pad, None))
+
+
+@pytest.mark.parametrize("n_pad", [32, 256, 1024, 4096, 16384, 32768])
+def test_encode_bit_exact(n_pad):
+    M = M_()
+    rows = 6 if n_pad >= 16384 else 23
+    n = n_pad - 5 if n_pad > 64 else n_pad
+    x = wl.spike_activations(rows, n, seed=3)
+    x[1, :] = 0.0                  # zero row: scale 0, code 0
+    x[2, 7] = np.inf               # non-finite row: scale NaN, code 0
+    words = O.sample_signs(KEY, 12, n_pad)
+    mask = wl.uniform_u32(9, rows, n_pad)
+    qmax = O.qmax_for(n_pad)
+    for rotate in (1, 0):
+        out = torch.empty(rows, n_pad, dtype=torch.int32, device="cuda")
+        sc = torch.empty(rows, dtype=torch.float32, device="cuda")
+        planes = torch.empty(4, rows, n_pad, dtype=torch.int16, device="cuda")
+        M.mosaic_encode(dev(x), n, rows, n, n_pad, qmax, rotate, dev(words), dev(mask), n_pad, out,
+                        n_pad, sc, planes)
+        if rotate:
+            v = O.fwht_rows(x, n_pad, words)
+        else:
+            v = np.zeros((rows, n_pad), np.float32); v[:, :n] = x
+        code, scale = O.encode_rows(v, qmax)
+        got = host_u32(out)
+        assert np.array_equal(got, code + mask)
+        gs = host_f32(sc)
+        assert np.array_equal(np.isnan(gs), np.isnan(scale))
+        assert np.array_equal(gs[~np.isnan(gs)], scale[~np.isnan(scale)])
+        assert np.isnan(gs[2]) and gs[1] == 0
+        # planes are the signed digits of out, exactly representable in bf16
+        pl = host_f32(planes.view(torch.bfloat16).float()).astype(np.int64)
+        rebuilt = sum(pl[i] << (8 * i) for i in range(4)) % (1 << 32)
+        assert np.array_equal(rebuilt.astype(np.uint32), got)
+        assert pl.min() >= -128 and pl.max() <= 127
+
+
+def test_digit_split_identity():
+    M = M_()
+    a = wl.uniform_u32(4, 37, 64)
+    a[0, :8] = [0, 0x7F7F7F7F, 0x80808080, 0xFFFFFFFF, 1, 0x80000000, 0x7FFFFFFF, 0x01010101]
+    planes = torch.empty(4, 37, 64, dtype=torch.int16, device="cuda")
+    M.mosaic_digit_split(dev(a), 64, 37, 64, planes)
+    pl = host_f32(planes.view(torch.bfloat16).float()).astype(np.int64)
+    assert pl.min() >= -128 and pl.max() <= 127
+    rebuilt = sum(pl[i] << (8 * i) for i in range(4)) % (1 << 32)
+    assert np.array_equal(rebuilt.astype(np.uint32), a)
+    # 0x80808080 + 0x80808080 = 0x01010100 (mod 2^32) -> digits (0-128, 1-128, 1-128, 1-128)
+    assert list(pl[:, 0, 2]) == [-128, -127, -127, -127]
+
+
+# --------------------------------------------------------------------------
+# Ring product
+# --------------------------------------------------------------------------
+GEMM_SHAPES = [(1, 1, 1), (5, 3, 7), (130, 257, 33), (128, 128, 16), (300, 129, 1000), (64, 200, 0),
+               (257, 384, 652)]
+
+
+@pytest.mark.parametrize("Mm,N,K", GEMM_SHAPES)
+def test_ring_gemm_imad(Mm, N, K):
+    M = M_()
+    A = wl.uniform_u32(1, Mm, max(K, 1))[:, :K].copy()
+    B = wl.uniform_u32(2, N, max(K, 1))[:, :K].copy()
+    if K:
+        A[0, :] = 0xFFFFFFFF; B[0, :] = 0xFFFFFFFF
+    C = torch.full((Mm, N + 3), -1, dtype=torch.int32, device="cuda")
+    M.mosaic_ring_gemm(dev(A) if K else torch.zeros(Mm, 1, dtype=torch.int32, device="cuda"),
+                       max(K, 1), dev(B) if K else torch.zeros(N, 1, dtype=torch.int32, device="cuda"),
+                       max(K, 1), C, N + 3, Mm, N, K, M.GEMM_IMAD)
+    got = host_u32(C)
+    want = O.matmul(A, B.T.copy()) if K else np.zeros((Mm, N), np.uint32)
+    assert np.array_equal(got[:, :N], want)
+    assert np.all(got[:, N:] == 0xFFFFFFFF)
+
+
+# --------------------------------------------------------------------------
+# Masks, server, unmask
+# --------------------------------------------------------------------------
+def _params(d, r, t, sigma=0.5):
+    M = M_()
+    tt = [0] + list(t)
+    return (M.default_params(d=d, r=list(r) + [0] * (3 - len(r)), t=tt + [0] * (3 - len(tt)),
+                             sigma=sigma),
+            O.Params(d=d, r=tuple(r), t=tuple(t), sigma=sigma))
+
+
+def _run_layer(d, r, t, m, n, l, sigma=0.5, w_std=1.0, bias=True, variant=None):
+    from paper_2607_29221_gb300 import protocol as PR
+    M = M_()
+    gp, op = _params(d, r, t, sigma)
+    variant = M.GEMM_IMAD if variant is None else variant
+    proto = PR.Protocol(KEY, gp, variant=variant)
+    n_pad = PR.pad_width(n)
+    W = wl.weights(m, n, std=w_std)
+    X_tm = wl.activations(l, n)
+    b = wl.bias(m) if bias else None
+    ch = PR.Chains(proto, n_pad)
+    layer = PR.SecureLinear(proto, dev(W), 5, ch, bias=dev(b) if bias else None)
+    mp = layer.init_x(l, 77)
+    Xp, s_x, Xpl = layer.mask_input(dev(X_tm), mp)
+    Z = layer.server(Xp, Xpl)
+    Yhat = torch.empty(l, m, dtype=torch.int32, device="cuda")
+    Y = layer.unmask(Z, mp, s_x, Yhat=Yhat)
+    g = dict(P=host_u32(ch.P), C=host_u32(ch.C), CT=host_u32(ch.CT), Wp=host_u32(layer.Wp),
+             J=host_u32(layer.J), L=host_u32(layer.L), S_idx=host_u32(layer.S_idx),
+             S_val=host_u32(layer.S_val), s_w=host_f32(layer.s_w), signs=host_u32(layer.sign_words),
+             Ux=host_u32(mp.Ux), K=host_u32(mp.K), Xp=host_u32(Xp), s_x=host_f32(s_x),
+             Z=host_u32(Z), Yhat=host_u32(Yhat), Y=host_f32(Y))
+    ref = O.secure_linear(KEY, op, W, X_tm.T.copy(), matrix_id=5, pass_id=77, b=b)
+    ref["bias"] = b
+    return g, ref, op, m, l
+
+
+def _check_layer(g, ref, op, m, l):
+    P = np.vstack(ref["P"]); C = np.hstack(ref["C"])
+    assert np.array_equal(g["P"], P)
+    assert np.array_equal(g["C"], C)
+    assert np.array_equal(g["CT"], C.T)
+    ws, ps = ref["ws"], ref["ps"]
+    assert np.array_equal(g["signs"], ws.sign_words)
+    assert np.array_equal(g["s_w"], ws.s_w)
+    assert np.array_equal(g["L"], ws.L)
+    off = 0
+    for i in range(1, op.d):
+        t = op.t[i - 1]
+        assert np.array_equal(g["S_idx"][off:off + m * t].reshape(m, t), ws.S[i + 1][0])
+        assert np.array_equal(g["S_val"][off:off + m * t].reshape(m, t), ws.S[i + 1][1])
+        off += m * t
+    assert np.array_equal(g["Wp"][:m], ws.W_masked)
+    assert np.array_equal(g["Wp"][m:], P)
+    assert np.array_equal(g["J"], np.hstack(ws.J))
+    assert np.array_equal(g["Ux"], ps.U_x.T)
+    assert np.array_equal(g["K"], ps.K.T)
+    assert np.array_equal(g["Xp"], ref["X_masked"].T)
+    assert np.array_equal(g["s_x"], ref["s_x"])
+    Zref = np.hstack([ref["Y_masked"].T] + [q.T for q in ref["Q"]])
+    assert np.array_equal(g["Z"], Zref)
+    assert np.array_equal(g["Yhat"], ref["Y_hat"].T)
+    Yref = ref["Y"].T
+    mag = np.abs(ref["Y_hat"].T.view(np.int32).astype(np.float64) * ws.s_w[None, :].astype(np.float64)
+                 * ref["s_x"][:, None].astype(np.float64))
+    if ref["bias"] is not None:
+        mag = mag + np.abs(ref["bias"].astype(np.float64))[None, :]
+    assert np.all(np.abs(g["Y"].astype(np.float64) - Yref) <= 1e-6 * mag)
+
+
+@pytest.mark.parametrize("d,r,t", [(1, (96,), ()), (2, (96, 64), (6,)), (3, (96, 64, 40), (6, 5))])
+def test_layer_small_ranks(d, r, t):
+    g, ref, op, m, l = _run_layer(d, r, t, m=40, n=100, l=21)
+    _check_layer(g, ref, op, m, l)
+
+
+def test_layer_zero_noise_and_no_bias():
+    g, ref, op, m, l = _run_layer(3, (96, 64, 40), (6, 5), m=33, n=64, l=9, sigma=0.0, bias=False)
+    _check_layer(g, ref, op, m, l)
+    assert np.array_equal(ref["Y_hat"], ref["ws"].W_hat @ ref["X_hat"])
+
+
+def test_layer_single_64x256x128():
+    """The small workload (X 64x256, W 256->128, N(0,1)) with Example 3.1 parameters."""
+    g, ref, op, m, l = _run_layer(3, (1536, 1024, 652), (80, 80), m=128, n=256, l=64)
+    _check_layer(g, ref, op, m, l)
+
+
+@pytest.mark.slow
+def test_layer_attn_proj_7b_full():
+    """Attention projection at 7B shape (X 512x4096, W 4096x4096), full oracle."""
+    g, ref, op, m, l = _run_layer(3, (1536, 1024, 652), (80, 80), m=4096, n=4096, l=512,
+                                  w_std=0.02)
+    _check_layer(g, ref, op, m, l)
