@@ -280,6 +280,12 @@ mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const 
                             const float *s_x, const float *bias, float *Y, uint32_t *Yhat,
                             int64_t ldy, int variant, void *ws, size_t ws_bytes, void *stream);
 
+/* Synchronises `stream` and reports device-side failures of earlier calls:
+ * MOSAIC_ERR_TIMEOUT if a tensor-core product gave up a bounded wait (the
+ * device error word is cleared by this call), MOSAIC_ERR_CUDA if a CUDA error
+ * is pending, else MOSAIC_OK. */
+mosaic_status mosaic_device_status(void *stream);
+
 /* Workspace sizes. */
 typedef enum {
     MOSAIC_OP_RING_GEMM = 1,        /* M = rows of A, n_pad = rows of B (N), l = K */

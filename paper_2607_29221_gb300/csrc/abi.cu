@@ -270,6 +270,12 @@ mosaic_status mosaic_ring_gemm_planes(const uint16_t *A_planes, int64_t ldpa, in
                                1, M, N, K, as_stream(stream));
 }
 
+mosaic_status mosaic_device_status(void *stream) {
+    const mosaic_status s = device_status(as_stream(stream));
+    if (s != MOSAIC_OK) return s;
+    return cudaGetLastError() == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
+}
+
 size_t mosaic_workspace_bytes(int op, int64_t m, int64_t n_pad, int64_t l, const mosaic_params *p) {
     if (m < 0 || n_pad < 0 || l < 0) return 0;
     switch (op) {

@@ -111,6 +111,7 @@ mosaic_status ring_gemm_mma_s8(const uint32_t *A, int64_t lda, const uint32_t *B
                                uint32_t *C, int64_t ldc, const uint32_t *Cin, int64_t ldcin,
                                int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st);
 bool tc_available();
+mosaic_status device_status(cudaStream_t st);
 bool mma_s8_available();
 
 // Sparse gathers.

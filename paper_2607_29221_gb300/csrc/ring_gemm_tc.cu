@@ -1,21 +1,448 @@
-// Tensor-core ring product (placeholder until the tcgen05 kernel lands).
+// Ring product over Z_{2^32} on the 5th-generation tensor cores (tcgen05).
+//
+// Sec. 5.2 ("Emulation approach") emulates each 32-bit ring MAC with 8-bit
+// limb products on INT8 tensor cores.  The INT8 tensor path (tcgen05
+// kind::i8) does not exist on sm_103a, so this kernel re-designs the limb
+// products for kind::f16 with bf16 operands:
+//   * every operand a is split into SIGNED base-2^8 digits
+//     d_i = byte_i(a + 0x80808080) - 128 in [-128, 127], so that
+//     a = sum_i d_i 2^(8i) mod 2^32; each digit is an exact bf16 value;
+//   * a b mod 2^32 = sum_{i+j<=3} 2^(8(i+j)) d_i e_j: only the 10 digit pairs
+//     with i + j <= 3 survive mod 2^32, grouped into 4 shift groups
+//     s = i + j (1, 2, 3, 4 products);
+//   * each group accumulates in fp32 in tensor memory (TMEM); a product of
+//     two digits is at most 2^14 in magnitude, so a group that has summed at
+//     most 1024 products is still an exact integer (|sum| <= 2^24).  Every
+//     CHUNK * BK = 256 values of K (group 3 then holds 1024 products) the
+//     epilogue warps drain all four groups to int32 registers:
+//     acc += (int32)g_s << 8s, with 32-bit wraparound, which is exact mod 2^32.
+//
+// Pipeline (one 128 x BN output tile per CTA, 6 warps):
+//   warp 0      TMA producer: per stage one 3-D box {32 K, rows, 4 planes}
+//               for A and one for B (64-byte swizzle), mbarrier complete_tx
+//   warp 1      TMEM allocation (512 columns) and the single-thread MMA issuer
+//               (20 tcgen05.mma of 128 x BN x 16 per stage)
+//   warps 2..5  epilogue: tcgen05.ld 32x32b, fp32 -> int32, shift-add
+// Every wait is bounded (about 2 s of %globaltimer); on expiry the kernel
+// raises a device error word, stops issuing work, waits (bounded) for its
+// own copies and products in flight, frees TMEM and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "mosaic_internal.cuh"
 
 namespace mosaic {
 
-bool tc_available() { return false; }
+__device__ uint32_t g_tc_error = 0;
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 32;          // bf16 K elements per stage = one 64-byte swizzled row
+constexpr int STAGES = 3;
+constexpr int CHUNK = 8;        // stages between drains: 256 K
+constexpr uint32_t TMEM_COLS = 512;
+constexpr int THREADS = 192;
+constexpr unsigned long long kWaitNs = 2000000000ull;
+
+template <int BN>
+struct Cfg {
+    static constexpr int A_PLANE = BM * BK * 2;
+    static constexpr int B_PLANE = BN * BK * 2;
+    static constexpr int A_BYTES = 4 * A_PLANE;
+    static constexpr int B_BYTES = 4 * B_PLANE;
+    static constexpr int STAGE = A_BYTES + B_BYTES;
+    static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+    // kind::f16 instruction descriptor: D f32, A/B bf16, K-major, N >> 3, M >> 4.
+    static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
+                                      ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+    static_assert(4 * BN <= (int)TMEM_COLS, "four shift groups must fit in TMEM");
+    static_assert(BN % 32 == 0 && BN >= 32 && BN <= 128, "");
+};
+
+struct TcArgs {
+    uint32_t *C;
+    int64_t ldc;
+    const uint32_t *Cin;
+    int64_t ldcin;
+    int sgn;
+    int M, N, K;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ unsigned long long gtime() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait on phase `parity`; false on timeout or when another role aborted.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort_flag) {
+    if (mbar_try(bar, parity)) return true;
+    const unsigned long long t0 = gtime();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try(bar, parity)) return true;
+        if ((it & 255u) == 0) {
+            if (*abort_flag) return false;
+            if (gtime() - t0 > kWaitNs) return false;
+        }
+    }
+}
+__device__ __forceinline__ void raise_abort(volatile int *abort_flag) {
+    *abort_flag = 1;
+    atomicExch(&g_tc_error, 1u);
+}
+__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, uint64_t *bar, int c0,
+                                            int c1, int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// Shared-memory matrix descriptor: K-major, 64-byte swizzle; rows of 64 B,
+// 8-row core groups 512 B apart (stride byte offset); descriptor version 1.
+__device__ __forceinline__ uint64_t sdesc_sw64(uint32_t saddr) {
+    uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1 << 16;               // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(512 >> 4) << 32;      // stride byte offset
+    d |= (uint64_t)1 << 46;               // version
+    d |= (uint64_t)4 << 61;               // SWIZZLE_64B
+    return d;
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *v) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+          "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+          "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+          "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+template <int BN>
+__global__ void __launch_bounds__(THREADS, 1)
+    ring_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                        TcArgs a) {
+    using C = Cfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~static_cast<uintptr_t>(1023));
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * C::STAGE);
+    uint64_t *empty = full + STAGES;
+    uint64_t *acc_full = empty + STAGES;
+    uint64_t *acc_empty = acc_full + 1;
+    uint64_t *drain = acc_empty + 1;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+    const int nk = (a.K + BK - 1) / BK;
+    const int nchunks = (nk + CHUNK - 1) / CHUNK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(acc_full, 1);
+        mbar_init(acc_empty, 4);
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int issued = 0;
+            for (int ks = 0; ks < nk; ++ks) {
+                const int s = ks % STAGES;
+                if (ks >= STAGES && !mbar_wait(&empty[s], ((ks / STAGES) - 1) & 1, abort_flag)) {
+                    raise_abort(abort_flag);
+                    break;
+                }
+                uint8_t *st = smem + s * C::STAGE;
+                mbar_expect_tx(&full[s], C::STAGE);
+                tma_load_3d(st, &tmA, &full[s], ks * BK, m0, 0);
+                tma_load_3d(st + C::A_BYTES, &tmB, &full[s], ks * BK, n0, 0);
+                issued = ks + 1;
+            }
+            if (*abort_flag) {
+                // Let the copies this thread started land before the CTA exits.
+                const int lo = issued > STAGES ? issued - STAGES : 0;
+                for (int ks = lo; ks < issued; ++ks) {
+                    const unsigned long long t0 = gtime();
+                    while (!mbar_try(&full[ks % STAGES], (ks / STAGES) & 1) && gtime() - t0 < kWaitNs) {
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            bool issued_any = false;
+            for (int ks = 0; ks < nk; ++ks) {
+                const int s = ks % STAGES;
+                const int chunk = ks / CHUNK;
+                const bool first = (ks % CHUNK) == 0;
+                if (first && chunk > 0 && !mbar_wait(acc_empty, (chunk - 1) & 1, abort_flag)) {
+                    raise_abort(abort_flag);
+                    break;
+                }
+                if (!mbar_wait(&full[s], (ks / STAGES) & 1, abort_flag)) {
+                    raise_abort(abort_flag);
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a_base = smem_u32(smem + s * C::STAGE);
+                const uint32_t b_base = a_base + C::A_BYTES;
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk) {
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+#pragma unroll
+                        for (int i = 0; i <= g; ++i) {
+                            const int j = g - i;
+                            const uint64_t ad = sdesc_sw64(a_base + i * C::A_PLANE + kk * 32);
+                            const uint64_t bd = sdesc_sw64(b_base + j * C::B_PLANE + kk * 32);
+                            const uint32_t acc = (first && kk == 0 && i == 0) ? 0u : 1u;
+                            umma_bf16(tmem + g * BN, ad, bd, C::IDESC, acc);
+                        }
+                    }
+                }
+                issued_any = true;
+                umma_commit(&empty[s]);
+                if ((ks % CHUNK) == CHUNK - 1 || ks == nk - 1) umma_commit(acc_full);
+            }
+            if (*abort_flag && issued_any) {
+                // Products in flight still read shared memory and write TMEM.
+                umma_commit(drain);
+                const unsigned long long t0 = gtime();
+                while (!mbar_try(drain, 0) && gtime() - t0 < kWaitNs) {
+                }
+            }
+        }
+    } else {
+        // Epilogue: warp w reads TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31.
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+        uint32_t acc[BN];
+#pragma unroll
+        for (int c = 0; c < BN; ++c) acc[c] = 0u;
+        bool ok = true;
+        for (int ch = 0; ch < nchunks; ++ch) {
+            if (!mbar_wait(acc_full, ch & 1, abort_flag)) {
+                raise_abort(abort_flag);
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+#pragma unroll
+                for (int c0 = 0; c0 < BN; c0 += 32) {
+                    uint32_t v[32];
+                    tmem_ld32(lane_addr + g * BN + c0, v);
+#pragma unroll
+                    for (int c = 0; c < 32; ++c)
+                        acc[c0 + c] += ((uint32_t)__float2int_rn(__uint_as_float(v[c]))) << (8 * g);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(acc_empty);
+        }
+        const int gm = m0 + row;
+        if (ok && gm < a.M) {
+            uint32_t *crow = a.C + (int64_t)gm * a.ldc;
+            const uint32_t *cin = a.Cin ? a.Cin + (int64_t)gm * a.ldcin : nullptr;
+            const bool vec = (n0 + BN <= a.N) && ((a.ldc & 3) == 0) &&
+                             ((reinterpret_cast<uintptr_t>(crow) & 15u) == 0) &&
+                             (!cin || (((a.ldcin & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin) & 15u) == 0)));
+            if (vec) {
+#pragma unroll
+                for (int c = 0; c < BN; c += 4) {
+                    uint4 o;
+                    o.x = a.sgn >= 0 ? acc[c] : 0u - acc[c];
+                    o.y = a.sgn >= 0 ? acc[c + 1] : 0u - acc[c + 1];
+                    o.z = a.sgn >= 0 ? acc[c + 2] : 0u - acc[c + 2];
+                    o.w = a.sgn >= 0 ? acc[c + 3] : 0u - acc[c + 3];
+                    if (cin) {
+                        const uint4 i4 = *reinterpret_cast<const uint4 *>(cin + n0 + c);
+                        o.x += i4.x; o.y += i4.y; o.z += i4.z; o.w += i4.w;
+                    }
+                    *reinterpret_cast<uint4 *>(crow + n0 + c) = o;
+                }
+            } else {
+#pragma unroll
+                for (int c = 0; c < BN; ++c) {
+                    const int gn = n0 + c;
+                    if (gn < a.N) {
+                        uint32_t v = a.sgn >= 0 ? acc[c] : 0u - acc[c];
+                        if (cin) v += cin[gn];
+                        crow[gn] = v;
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS)
+                     : "memory");
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+// 3-D map over bf16 digit planes: {K, rows, 4 planes}, box {BK, box_rows, 4}.
+bool make_plane_map(CUtensorMap *map, const uint16_t *base, int64_t K, int64_t rows, int64_t ldp,
+                    int64_t plane_stride, int box_rows) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)K, (cuuint64_t)rows, 4};
+    cuuint64_t strides[2] = {(cuuint64_t)ldp * 2, (cuuint64_t)plane_stride * 2};
+    cuuint32_t box[3] = {(cuuint32_t)BK, (cuuint32_t)box_rows, 4};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<uint16_t *>(base), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN>
+mosaic_status launch_tc(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const uint16_t *Bp,
+                        int64_t ldpb, int64_t b_plane, uint32_t *Cm, int64_t ldc, const uint32_t *Cin,
+                        int64_t ldcin, int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st) {
+    using C = Cfg<BN>;
+    CUtensorMap ta, tb;
+    if (!make_plane_map(&ta, Ap, K, M, ldpa, a_plane, BM) || !make_plane_map(&tb, Bp, K, N, ldpb, b_plane, BN))
+        return MOSAIC_ERR_CUDA;
+    static unsigned long long attr_set = 0;   // one bit per device ordinal
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return MOSAIC_ERR_CUDA;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(attr_set & bit)) {
+        if (cudaFuncSetAttribute(ring_gemm_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 C::SMEM) != cudaSuccess)
+            return MOSAIC_ERR_CUDA;
+        attr_set |= bit;
+    }
+    TcArgs args{Cm, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)K};
+    dim3 grid((unsigned)((N + BN - 1) / BN), (unsigned)((M + BM - 1) / BM));
+    ring_gemm_tc_kernel<BN><<<grid, THREADS, C::SMEM, st>>>(ta, tb, args);
+    return launch_status();
+}
+
+}  // namespace
+
+bool tc_available() {
+    int dev = 0, major = 0, minor = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) return false;
+    return major == 10 && minor == 3 && encode_fn() != nullptr;
+}
+
 bool mma_s8_available() { return false; }
 
-mosaic_status ring_gemm_tc_planes(const uint16_t *, int64_t, int64_t, const uint16_t *, int64_t,
-                                  int64_t, uint32_t *, int64_t, const uint32_t *, int64_t, int,
-                                  int64_t, int64_t, int64_t, cudaStream_t) {
+mosaic_status ring_gemm_tc_planes(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const uint16_t *Bp,
+                                  int64_t ldpb, int64_t b_plane, uint32_t *Cm, int64_t ldc,
+                                  const uint32_t *Cin, int64_t ldcin, int sgn, int64_t M, int64_t N,
+                                  int64_t K, cudaStream_t st) {
+    if (M == 0 || N == 0) return MOSAIC_OK;
+    if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX || (M + BM - 1) / BM > 65535)
+        return MOSAIC_ERR_SHAPE;
+    return launch_tc<128>(Ap, ldpa, a_plane, Bp, ldpb, b_plane, Cm, ldc, Cin, ldcin, sgn, M, N, K, st);
+}
+
+mosaic_status ring_gemm_mma_s8(const uint32_t *, int64_t, const uint32_t *, int64_t, uint32_t *, int64_t,
+                               const uint32_t *, int64_t, int, int64_t, int64_t, int64_t, cudaStream_t) {
     return MOSAIC_ERR_UNSUPPORTED;
 }
 
-mosaic_status ring_gemm_mma_s8(const uint32_t *, int64_t, const uint32_t *, int64_t, uint32_t *,
-                               int64_t, const uint32_t *, int64_t, int, int64_t, int64_t, int64_t,
-                               cudaStream_t) {
-    return MOSAIC_ERR_UNSUPPORTED;
+mosaic_status device_status(cudaStream_t st) {
+    if (cudaStreamSynchronize(st) != cudaSuccess) return MOSAIC_ERR_CUDA;
+    uint32_t v = 0, zero = 0;
+    if (cudaMemcpyFromSymbol(&v, g_tc_error, sizeof v) != cudaSuccess) return MOSAIC_ERR_CUDA;
+    if (v) {
+        cudaMemcpyToSymbol(g_tc_error, &zero, sizeof zero);
+        return MOSAIC_ERR_TIMEOUT;
+    }
+    return MOSAIC_OK;
 }
 
 }  // namespace mosaic

@@ -72,6 +72,7 @@ _SIGS = {
     "mosaic_unmask": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64, _INT,
                        _P, _SZ, _P], _INT),
     "mosaic_workspace_bytes": ([_INT, _I64, _I64, _I64, _PP], _SZ),
+    "mosaic_device_status": ([_P], _INT),
 }
 
 EXPORTS = tuple(_SIGS)
@@ -156,6 +157,10 @@ def mosaic_gaussian_table(sigma: float):
 
 def mosaic_gemm_variant_available(variant: int) -> bool:
     return bool(lib().mosaic_gemm_variant_available(variant))
+
+
+def mosaic_device_status(stream=None):
+    _call("mosaic_device_status", _stream(stream))
 
 
 def mosaic_workspace_bytes(op: int, m: int, n_pad: int, l: int, params: mosaic_params) -> int:

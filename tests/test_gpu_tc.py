@@ -1,0 +1,121 @@
+"""Tensor-core ring product (tcgen05 kind::f16 on exact bf16 digit planes)
+against the oracle's naive Z_{2^32} triple loop: bit-exact on random,
+ragged and adversarial operands.  All digits -128 (a = 0x7F7F7F80) make every
+digit product +2^14, so shift group 3 reaches exactly 2^24 at the end of each
+256-wide K chunk: the edge of exact fp32 accumulation."""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2607_29221_gb300 import workloads as wl
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+ALL_M128 = 0x7F7F7F80      # every signed digit is -128
+ALL_P127 = 0x7F7F7F7F      # every signed digit is +127
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2607_29221_gb300 import build
+    build.build()
+    from paper_2607_29221_gb300 import mosaic as M
+    if not M.mosaic_gemm_variant_available(M.GEMM_TC):
+        pytest.skip("tensor-core variant not available on this device")
+    yield
+
+
+def _M():
+    from paper_2607_29221_gb300 import mosaic as M
+    return M
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).cuda()
+
+
+def host(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy().view(np.uint32)
+
+
+def planes_of(a_dev, rows, K, ldp):
+    M = _M()
+    p = torch.zeros(4, rows, ldp, dtype=torch.int16, device="cuda")
+    if rows and K:
+        src = torch.zeros(rows, ldp, dtype=torch.int32, device="cuda")
+        src[:, :K] = a_dev
+        M.mosaic_digit_split(src, ldp, rows, ldp, p)
+    return p
+
+
+def tc_gemm(A, B):
+    M = _M()
+    Mm, K = A.shape
+    N = B.shape[0]
+    ldp = max(8, (K + 7) // 8 * 8)
+    Ap = planes_of(dev(A), Mm, K, ldp)
+    Bp = planes_of(dev(B), N, K, ldp)
+    C = torch.full((Mm, N + 4), -1, dtype=torch.int32, device="cuda")
+    M.mosaic_ring_gemm_planes(Ap, ldp, Mm * ldp, Bp, ldp, N * ldp, C, N + 4, Mm, N, K, M.GEMM_TC)
+    M.mosaic_device_status()
+    got = host(C)
+    assert np.all(got[:, N:] == 0xFFFFFFFF)
+    return got[:, :N]
+
+
+def ref(A, B):
+    return O.matmul(A, B.T.copy())
+
+
+@pytest.mark.parametrize("Mm,N,K", [(128, 128, 32), (128, 128, 256), (130, 257, 33), (1, 1, 8),
+                                    (300, 129, 1000), (257, 384, 652), (64, 200, 7),
+                                    (512, 640, 4096), (129, 1000, 2049)])
+def test_tc_random(Mm, N, K):
+    A = wl.uniform_u32(11, Mm, K)
+    B = wl.uniform_u32(12, N, K)
+    assert np.array_equal(tc_gemm(A, B), ref(A, B))
+
+
+@pytest.mark.parametrize("K", [256, 512, 1024, 768 + 32])
+@pytest.mark.parametrize("va,vb", [(ALL_M128, ALL_M128), (ALL_P127, ALL_M128), (ALL_P127, ALL_P127)])
+def test_tc_adversarial_digits(K, va, vb):
+    A = np.full((128, K), va, np.uint32)
+    B = np.full((128, K), vb, np.uint32)
+    assert np.array_equal(tc_gemm(A, B), ref(A, B))
+
+
+def test_tc_mixed_magnitudes():
+    """Large partial sums followed by small products (rounding would drop the small ones)."""
+    K = 512
+    A = np.full((256, K), ALL_M128, np.uint32)
+    B = np.full((128, K), ALL_M128, np.uint32)
+    rng = np.random.Generator(np.random.PCG64(5))
+    A[:, 200:] = rng.integers(0, 2**32, (256, K - 200), dtype=np.uint64).astype(np.uint32)
+    B[::2, 255] = 0x80808081          # digit 0 = +1, others 0
+    A[::3, 255] = 0x80808081
+    assert np.array_equal(tc_gemm(A, B), ref(A, B))
+
+
+def test_tc_through_uint32_entry():
+    M = _M()
+    A = wl.uniform_u32(21, 200, 96)
+    B = wl.uniform_u32(22, 300, 96)
+    p = M.default_params()
+    ws = torch.empty(M.mosaic_workspace_bytes(M.OP_RING_GEMM, 200, 300, 96, p), dtype=torch.uint8,
+                     device="cuda")
+    C = torch.empty(200, 300, dtype=torch.int32, device="cuda")
+    M.mosaic_ring_gemm(dev(A), 96, dev(B), 96, C, 300, 200, 300, 96, M.GEMM_TC, ws)
+    M.mosaic_device_status()
+    assert np.array_equal(host(C), ref(A, B))
+
+
+def test_tc_protocol_layer_matches_oracle():
+    """The single 64x256x128 layer with the server product on tensor cores."""
+    import test_gpu_parity as T
+    g, r, op, m, l = T._run_layer(3, (1536, 1024, 652), (80, 80), m=128, n=256, l=64,
+                                  variant=_M().GEMM_TC)
+    T._check_layer(g, r, op, m, l)
