@@ -286,6 +286,32 @@ mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const 
  * is pending, else MOSAIC_OK. */
 mosaic_status mosaic_device_status(void *stream);
 
+/* mosaic_unmask for callers that cannot allocate device memory (the paper
+ * has no counterpart: this is a deployment convenience of this library).
+ * Same arguments and results as mosaic_unmask, without `ws`/`ws_bytes`: the
+ * l x m words of scratch come from a fixed 16 MiB array inside the library,
+ * so it suits code that may not call cudaMalloc -- e.g. a plugin whose host
+ * framework owns all device memory, or a serving loop with a fixed memory
+ * budget.
+ *  - Limit: l * m <= 2^22 (4,194,304); larger requests return
+ *    MOSAIC_ERR_WORKSPACE and enqueue nothing.
+ *  - Every GPU that loads the library holds the 16 MiB array until the
+ *    process exits.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - All calls share the one array: calls whose GPU work overlaps (e.g. on two
+ *    streams at once) race on it, so order them (same stream or events).
+ *    Nothing in the array needs to start at zero: each call writes every
+ *    scratch word before reading it.
+ *  - It allocates and frees nothing. */
+mosaic_status mosaic_unmask_noalloc(const mosaic_params *p, int64_t l, int64_t m,
+                                    const uint32_t *Z, int64_t ldz, const uint32_t *K_tm,
+                                    const uint32_t *L, const uint32_t *S_idx,
+                                    const uint32_t *S_val, const float *s_w, const float *s_x,
+                                    const float *bias, float *Y, uint32_t *Yhat, int64_t ldy,
+                                    int variant, void *stream);
+
 /* Workspace sizes. */
 typedef enum {
     MOSAIC_OP_RING_GEMM = 1,        /* M = rows of A, n_pad = rows of B (N), l = K */

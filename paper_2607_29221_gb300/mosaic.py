@@ -73,6 +73,8 @@ _SIGS = {
                        _P, _SZ, _P], _INT),
     "mosaic_workspace_bytes": ([_INT, _I64, _I64, _I64, _PP], _SZ),
     "mosaic_device_status": ([_P], _INT),
+    "mosaic_unmask_noalloc": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
+                               _INT, _P], _INT),
 }
 
 EXPORTS = tuple(_SIGS)
@@ -237,3 +239,13 @@ def mosaic_unmask(params, l, m, Z, ldz, K_tm, L, S_idx, S_val, s_w, s_x, bias, Y
     _call("mosaic_unmask", ctypes.byref(params), l, m, _ptr(Z), ldz, _ptr(K_tm), _ptr(L),
           _ptr(S_idx), _ptr(S_val), _ptr(s_w), _ptr(s_x), _ptr(bias), _ptr(Y), _ptr(Yhat), ldy,
           variant, _ptr(ws), 0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
+
+
+def mosaic_unmask_noalloc(params, l, m, Z, ldz, K_tm, L, S_idx, S_val, s_w, s_x, bias, Y, Yhat, ldy,
+                          variant, stream=None):
+    """mosaic_unmask without a workspace: for callers that cannot allocate
+    device memory, the scratch is a fixed 16 MiB array inside the library
+    (l * m <= 2^22).  Calls whose GPU work overlaps share that array and race."""
+    _call("mosaic_unmask_noalloc", ctypes.byref(params), l, m, _ptr(Z), ldz, _ptr(K_tm), _ptr(L),
+          _ptr(S_idx), _ptr(S_val), _ptr(s_w), _ptr(s_x), _ptr(bias), _ptr(Y), _ptr(Yhat), ldy,
+          variant, _stream(stream))
