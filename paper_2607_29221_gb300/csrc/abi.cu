@@ -60,12 +60,36 @@ int64_t off_r(const mosaic_params *p, uint32_t i) {
 uint32_t tag_of(uint32_t kind, uint32_t level) { return kind | (level << 8); }
 bool npad_ok(int64_t n_pad) { return is_pow2(n_pad) && n_pad >= 32 && n_pad <= 32768; }
 
-// ring product dispatch for the internal compositions (uint32 operands)
-mosaic_status gemm_u32(int variant, const uint32_t *A, int64_t sai, int64_t sak, const uint32_t *B,
-                       int64_t sbj, int64_t sbk, uint32_t *C, int64_t ldc, const uint32_t *Cin,
-                       int64_t ldcin, int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st) {
-    (void)variant;
-    return ring_gemm_imad(A, sai, sak, B, sbj, sbk, C, ldc, Cin, ldcin, sgn, M, N, K, st);
+// Bytes of digit planes a tensor-core product of an M x K by N x K pair needs.
+size_t ws_gemm(int64_t M, int64_t N, int64_t K) {
+    const int64_t Kp = (K + 7) / 8 * 8;
+    return up(8 * (size_t)(M * Kp)) + up(8 * (size_t)(N * Kp));
+}
+
+// Ring product for the internal compositions (uint32 operands):
+// C = (Cin ? Cin : 0) + sgn * A B^T with A(i, k) = A[i sai + k sak], B(j, k) = B[j sbj + k sbk].
+// The tensor-core variant needs K-major operands with 16-byte aligned rows and
+// room in `cv` for both operands' digit planes; otherwise the CUDA-core
+// product runs.  The planes are dead once the product is enqueued (all work
+// is ordered on `st`), so their workspace is handed back.
+mosaic_status gemm_u32(int variant, Carve &cv, const uint32_t *A, int64_t sai, int64_t sak,
+                       const uint32_t *B, int64_t sbj, int64_t sbk, uint32_t *C, int64_t ldc,
+                       const uint32_t *Cin, int64_t ldcin, int sgn, int64_t M, int64_t N, int64_t K,
+                       cudaStream_t st) {
+    const bool want_tc = variant == MOSAIC_GEMM_TC || (variant == MOSAIC_GEMM_AUTO && tc_available());
+    const bool tc_ok = want_tc && sak == 1 && sbk == 1 && sai % 4 == 0 && sbj % 4 == 0 &&
+                       aligned16(A) && aligned16(B) && K > 0 && cv.used + ws_gemm(M, N, K) <= cv.cap;
+    if (!tc_ok) return ring_gemm_imad(A, sai, sak, B, sbj, sbk, C, ldc, Cin, ldcin, sgn, M, N, K, st);
+    const int64_t Kp = (K + 7) / 8 * 8;
+    const size_t mark = cv.used;
+    uint16_t *Ap = cv.take<uint16_t>((size_t)(4 * M * Kp));
+    uint16_t *Bp = cv.take<uint16_t>((size_t)(4 * N * Kp));
+    MOSAIC_TRY(digit_split(A, sai, M, K, Ap, Kp, M * Kp, st));
+    MOSAIC_TRY(digit_split(B, sbj, N, K, Bp, Kp, N * Kp, st));
+    const mosaic_status s =
+        ring_gemm_tc_planes(Ap, Kp, M * Kp, Bp, Kp, N * Kp, C, ldc, Cin, ldcin, sgn, M, N, K, st);
+    cv.used = mark;
+    return s;
 }
 
 size_t ws_chains(int64_t n_pad, const mosaic_params *p) {
@@ -78,20 +102,30 @@ size_t ws_chains(int64_t n_pad, const mosaic_params *p) {
     }
     return s;
 }
-size_t ws_weight(int64_t m, int64_t n_pad, const mosaic_params *) {
+int64_t sum_r(const mosaic_params *p);
+// Minimum workspaces (CUDA-core products) and the extra room that lets the
+// products run on the tensor cores.
+size_t ws_weight_min(int64_t m, int64_t n_pad, const mosaic_params *) {
     return up(sizeof(uint32_t) * (size_t)(m * n_pad));
 }
-size_t ws_activation(int64_t l, int64_t n_pad, const mosaic_params *p) {
-    (void)n_pad;
+size_t ws_weight(int64_t m, int64_t n_pad, const mosaic_params *p) {
+    return ws_weight_min(m, n_pad, p) + ws_gemm(m, sum_r(p), n_pad);
+}
+size_t ws_activation_min(int64_t l, const mosaic_params *p) {
     size_t s = up(sizeof(uint32_t) * (size_t)(l * p->r[p->d - 1]));
     for (uint32_t i = 2; i <= p->d; i++) s += 2 * up(sizeof(uint32_t) * (size_t)(l * p->t[i - 1]));
     return s;
 }
-size_t ws_unmask(int64_t m, int64_t l, const mosaic_params *) {
+size_t ws_activation(int64_t m, int64_t n_pad, int64_t l, const mosaic_params *p) {
+    const int64_t rd = p->r[p->d - 1];
+    const size_t g = ws_gemm(l, n_pad > m ? n_pad : m, rd);
+    return ws_activation_min(l, p) + g;
+}
+size_t ws_unmask_min(int64_t m, int64_t l, const mosaic_params *) {
     return up(sizeof(uint32_t) * (size_t)(l * m));
 }
-size_t ws_gemm(int64_t M, int64_t N, int64_t K) {
-    return up(8 * (size_t)(M * K)) + up(8 * (size_t)(N * K));
+size_t ws_unmask(int64_t m, int64_t l, const mosaic_params *p) {
+    return ws_unmask_min(m, l, p) + ws_gemm(l, m, p->r[p->d - 1]);
 }
 
 }  // namespace
@@ -242,7 +276,6 @@ mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B
     if (!tc_available()) return MOSAIC_ERR_UNSUPPORTED;
     const int64_t Kp = (K + 7) / 8 * 8;
     if (!aligned16(A) || !aligned16(B) || lda % 4 || ldb % 4) return MOSAIC_ERR_ALIGN;
-    if (K % 8) return MOSAIC_ERR_SHAPE;
     Carve cv{static_cast<char *>(ws), ws_bytes, 0};
     uint16_t *Ap = cv.take<uint16_t>((size_t)(4 * M * Kp));
     uint16_t *Bp = cv.take<uint16_t>((size_t)(4 * N * Kp));
@@ -283,7 +316,7 @@ size_t mosaic_workspace_bytes(int op, int64_t m, int64_t n_pad, int64_t l, const
         case MOSAIC_OP_MASK_CHAINS: return check_params(p) == MOSAIC_OK ? ws_chains(n_pad, p) : 0;
         case MOSAIC_OP_MASK_WEIGHT: return check_params(p) == MOSAIC_OK ? ws_weight(m, n_pad, p) : 0;
         case MOSAIC_OP_MASK_ACTIVATION:
-            return check_params(p) == MOSAIC_OK ? ws_activation(l, n_pad, p) : 0;
+            return check_params(p) == MOSAIC_OK ? ws_activation(m, n_pad, l, p) : 0;
         case MOSAIC_OP_UNMASK: return check_params(p) == MOSAIC_OK ? ws_unmask(m, l, p) : 0;
     }
     return 0;
@@ -336,7 +369,7 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, 
     if (!W || !P || !CT || !sign_words || !s_w || !L || !Wp || !J) return MOSAIC_ERR_ARG;
     if (p->d > 1 && (!S_idx || !S_val)) return MOSAIC_ERR_ARG;
     if (!aligned16(Wp) || (Wp_planes && !aligned16(Wp_planes))) return MOSAIC_ERR_ALIGN;
-    if (ws_bytes < ws_weight(m, n_pad, p)) return MOSAIC_ERR_WORKSPACE;
+    if (ws_bytes < ws_weight_min(m, n_pad, p)) return MOSAIC_ERR_WORKSPACE;
     cudaStream_t st = as_stream(stream);
     const Key k = to_key(key);
     const int R = (int)p->rounds;
@@ -356,7 +389,7 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, 
     MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EW, 0), matrix_id, R, p->sigma, m * n_pad, WE, st));
     MOSAIC_TRY(add_u32(Wp, n_pad, WE, n_pad, WE, n_pad, m, n_pad, st));
     // J_i = (W_hat + E_w) C_i for all i at once: J = WE CT^T (m x Sr).
-    MOSAIC_TRY(gemm_u32(variant, WE, n_pad, 1, CT, n_pad, 1, J, Sr, nullptr, 0, 1, m, Sr, n_pad, st));
+    MOSAIC_TRY(gemm_u32(variant, cv, WE, n_pad, 1, CT, n_pad, 1, J, Sr, nullptr, 0, 1, m, Sr, n_pad, st));
     // L, S_{i+1}.
     MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_L, 0), matrix_id, R, m, rd, L, rd, st));
     SparseLevel lev[2];
@@ -369,7 +402,7 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, 
         soff += m * t;
     }
     // W' = (W_hat + E_w) + L P_d + sum_i S_{i+1} P_i.
-    MOSAIC_TRY(gemm_u32(variant, L, rd, 1, P + od * n_pad, 1, n_pad, Wp, n_pad, WE, n_pad, 1, m,
+    MOSAIC_TRY(gemm_u32(variant, cv, L, rd, 1, P + od * n_pad, 1, n_pad, Wp, n_pad, WE, n_pad, 1, m,
                         n_pad, rd, st));
     if (d > 1)
         MOSAIC_TRY(sparse_rowgather(P, n_pad, lev, (int)d - 1, m, n_pad, Wp, n_pad, Wp, n_pad, st));
@@ -392,7 +425,7 @@ mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *k
     if (!npad_ok(n_pad) || m < 1 || l < 0 || l >= ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
     if (l == 0) return MOSAIC_OK;
     if (!C || !J || !Ux_tm || !K_tm) return MOSAIC_ERR_ARG;
-    if (ws_bytes < ws_activation(l, n_pad, p)) return MOSAIC_ERR_WORKSPACE;
+    if (ws_bytes < ws_activation_min(l, p)) return MOSAIC_ERR_WORKSPACE;
     cudaStream_t st = as_stream(stream);
     const Key k = to_key(key);
     const int R = (int)p->rounds;
@@ -413,13 +446,13 @@ mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *k
     }
     // U_x^T = E_x^T + R^T C_d^T + sum_i T_{i+1}^T C_i^T.
     MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EX, 0), pass_id, R, p->sigma, l * n_pad, Ux_tm, st));
-    MOSAIC_TRY(gemm_u32(variant, Rt, rd, 1, C + od, Sr, 1, Ux_tm, n_pad, Ux_tm, n_pad, 1, l, n_pad,
+    MOSAIC_TRY(gemm_u32(variant, cv, Rt, rd, 1, C + od, Sr, 1, Ux_tm, n_pad, Ux_tm, n_pad, 1, l, n_pad,
                         rd, st));
     if (d > 1)
         MOSAIC_TRY(sparse_gather(C, Sr, 0, od, n_pad, l, false, lev, (int)d - 1, Ux_tm, n_pad,
                                  nullptr, 0, 1, Ux_tm, n_pad, st));
     // K^T = R^T J_d^T + sum_i T_{i+1}^T J_i^T.
-    MOSAIC_TRY(gemm_u32(variant, Rt, rd, 1, J + od, Sr, 1, K_tm, m, nullptr, 0, 1, l, m, rd, st));
+    MOSAIC_TRY(gemm_u32(variant, cv, Rt, rd, 1, J + od, Sr, 1, K_tm, m, nullptr, 0, 1, l, m, rd, st));
     if (d > 1)
         MOSAIC_TRY(sparse_gather(J, Sr, 0, od, m, l, false, lev, (int)d - 1, K_tm, m, nullptr, 0, 1,
                                  K_tm, m, st));
@@ -438,13 +471,13 @@ mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const 
     if (l == 0) return MOSAIC_OK;
     if (!Z || !K_tm || !L || !s_w || !s_x || !Y) return MOSAIC_ERR_ARG;
     if (d > 1 && (!S_idx || !S_val)) return MOSAIC_ERR_ARG;
-    if (ws_bytes < ws_unmask(m, l, p)) return MOSAIC_ERR_WORKSPACE;
+    if (ws_bytes < ws_unmask_min(m, l, p)) return MOSAIC_ERR_WORKSPACE;
     cudaStream_t st = as_stream(stream);
     Carve cv{static_cast<char *>(ws), ws_bytes, 0};
     uint32_t *tmp = cv.take<uint32_t>((size_t)(l * m));
     if (!tmp) return MOSAIC_ERR_WORKSPACE;
     // tmp = K + Q_d L^T  (token-major: Q_d^T is the column block [m + od, m + Sr) of Z).
-    MOSAIC_TRY(gemm_u32(variant, Z + m + od, ldz, 1, L, rd, 1, tmp, m, K_tm, m, 1, l, m, rd, st));
+    MOSAIC_TRY(gemm_u32(variant, cv, Z + m + od, ldz, 1, L, rd, 1, tmp, m, K_tm, m, 1, l, m, rd, st));
     SparseLevel lev[2];
     int64_t soff = 0;
     for (uint32_t i = 1; i < d; i++) {

@@ -70,35 +70,80 @@ __global__ void gaussian_kernel(Key key, uint32_t tag, uint32_t sid_lo, uint32_t
     }
 }
 
-// One thread per sparse row; the row's window starts at block row * 4096.
-__global__ void sparse_kernel(Key key, uint32_t tag, uint32_t sid_lo, uint32_t sid_hi, int rounds,
-                              int64_t rows, uint32_t r, int t, uint32_t *idx, uint32_t *val,
-                              uint32_t *fail) {
-    const int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+// One warp per sparse row; the row's window starts at block row * 4096.
+// Each round the 32 lanes compute 32 consecutive ChaCha blocks (512 words),
+// which are then consumed in stream order, 32 words at a time: a word's
+// position is accepted if it is not in the row's bitmap and no lower lane of
+// the batch drew the same position (warp match), which is exactly the
+// sequential "skip repeats" rule; after the t-th accepted position the
+// following words are values (zero words skipped).
+constexpr int kSparseWarps = 4;
+
+__global__ void __launch_bounds__(kSparseWarps * 32)
+    sparse_kernel(Key key, uint32_t tag, uint32_t sid_lo, uint32_t sid_hi, int rounds, int64_t rows,
+                  uint32_t r, int t, uint32_t *idx, uint32_t *val, uint32_t *fail, int bitmap_words) {
+    extern __shared__ uint32_t sm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t j = (int64_t)blockIdx.x * kSparseWarps + warp;
     if (j >= rows) return;
+    uint32_t *words = sm + warp * (512 + bitmap_words);
+    uint32_t *bits = words + 512;
+    for (int w = lane; w < bitmap_words; w += 32) bits[w] = 0u;
+    __syncwarp();
     uint32_t *ri = idx + j * t;
     uint32_t *rv = val + j * t;
+    const unsigned lt_mask = (1u << lane) - 1u;
     int got = 0, nv = 0;
     const uint32_t blk0 = (uint32_t)(j * (kSparseWindow / 16));
-    for (int bi = 0; bi < kSparseWindow / 16 && nv < t; bi++) {
-        uint32_t w[16];
-        chacha_block(key, blk0 + bi, tag, sid_lo, sid_hi, rounds, w);
+    for (int round = 0; round < kSparseWindow / 512 && nv < t; ++round) {
+        uint32_t w16[16];
+        chacha_block(key, blk0 + round * 32 + lane, tag, sid_lo, sid_hi, rounds, w16);
 #pragma unroll
-        for (int i = 0; i < 16; i++) {
+        for (int i = 0; i < 16; i++) words[lane * 16 + i] = w16[i];
+        __syncwarp();
+        for (int b = 0; b < 16 && nv < t; ++b) {
+            const uint32_t w = words[b * 32 + lane];
+            int val_start = 0;
             if (got < t) {
-                const uint32_t p = (uint32_t)(((unsigned long long)w[i] * r) >> 32);
-                bool seen = false;
-                for (int q = 0; q < got; q++) seen |= (ri[q] == p);
-                if (!seen) ri[got++] = p;
-            } else if (nv < t) {
-                if (w[i] != 0u) rv[nv++] = w[i];
+                const uint32_t p = (uint32_t)(((unsigned long long)w * r) >> 32);
+                const bool taken = (bits[p >> 5] >> (p & 31)) & 1u;
+                const unsigned same = __match_any_sync(0xffffffffu, p);
+                const bool first = (__ffs(same) - 1) == lane;
+                unsigned acc = __ballot_sync(0xffffffffu, !taken && first);
+                const int need = t - got;
+                val_start = 32;
+                if (__popc(acc) >= need) {
+                    unsigned m = acc;
+                    for (int k = 1; k < need; ++k) m &= m - 1u;
+                    const int last = __ffs(m) - 1;
+                    acc &= last == 31 ? 0xffffffffu : ((2u << last) - 1u);
+                    val_start = last + 1;
+                }
+                if ((acc >> lane) & 1u) {
+                    ri[got + __popc(acc & lt_mask)] = p;
+                    atomicOr(&bits[p >> 5], 1u << (p & 31));
+                }
+                got += __popc(acc);
+                __syncwarp();
+            }
+            if (got >= t && val_start < 32) {
+                unsigned accv = __ballot_sync(0xffffffffu, lane >= val_start && w != 0u);
+                const int needv = t - nv;
+                if (__popc(accv) > needv) {
+                    unsigned m = accv;
+                    for (int k = 0; k < needv; ++k) m &= m - 1u;
+                    accv &= ~m;
+                }
+                if ((accv >> lane) & 1u) rv[nv + __popc(accv & lt_mask)] = w;
+                nv += __popc(accv);
             }
         }
+        __syncwarp();
     }
     if (nv < t) {
-        for (int q = got; q < t; q++) ri[q] = 0;
-        for (int q = nv; q < t; q++) rv[q] = 0;
-        if (fail) atomicExch(fail, 1u);
+        for (int q = got + lane; q < t; q += 32) ri[q] = 0u;
+        for (int q = nv + lane; q < t; q += 32) rv[q] = 0u;
+        if (lane == 0 && fail) atomicExch(fail, 1u);
     }
 }
 
@@ -161,9 +206,15 @@ mosaic_status prg_sparse(const Key &key, uint32_t tag, uint64_t sid, int rounds,
                          uint32_t r, uint32_t t, uint32_t *idx, uint32_t *val, uint32_t *fail,
                          cudaStream_t st) {
     if (rows == 0) return MOSAIC_OK;
-    const int threads = 64;
-    sparse_kernel<<<(unsigned)((rows + threads - 1) / threads), threads, 0, st>>>(
-        key, tag, (uint32_t)sid, (uint32_t)(sid >> 32), rounds, rows, r, (int)t, idx, val, fail);
+    const int bitmap_words = (int)((r + 31) / 32);
+    const size_t smem = (size_t)kSparseWarps * (512 + bitmap_words) * sizeof(uint32_t);
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(sparse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+            cudaSuccess)
+        return MOSAIC_ERR_CUDA;
+    sparse_kernel<<<(unsigned)((rows + kSparseWarps - 1) / kSparseWarps), kSparseWarps * 32, smem, st>>>(
+        key, tag, (uint32_t)sid, (uint32_t)(sid >> 32), rounds, rows, r, (int)t, idx, val, fail,
+        bitmap_words);
     return launch_status();
 }
 

@@ -17,12 +17,13 @@
 //     epilogue warps drain all four groups to int32 registers:
 //     acc += (int32)g_s << 8s, with 32-bit wraparound, which is exact mod 2^32.
 //
-// Pipeline (one 128 x BN output tile per CTA, 6 warps):
+// Pipeline (128 x BN output tiles, 10 warps):
 //   warp 0      TMA producer: per stage one 3-D box {32 K, rows, 4 planes}
 //               for A and one for B (64-byte swizzle), mbarrier complete_tx
 //   warp 1      TMEM allocation (512 columns) and the single-thread MMA issuer
 //               (20 tcgen05.mma of 128 x BN x 16 per stage)
-//   warps 2..5  epilogue: tcgen05.ld 32x32b, fp32 -> int32, shift-add
+//   warps 2..9  epilogue: tcgen05.ld 32x32b, fp32 -> int32, shift-add (each lane
+//               quarter of TMEM twice, half of the columns each)
 // Every wait is bounded (about 2 s of %globaltimer); on expiry the kernel
 // raises a device error word, stops issuing work, waits (bounded) for its
 // own copies and products in flight, frees TMEM and returns.
@@ -42,7 +43,8 @@ constexpr int BK = 32;          // bf16 K elements per stage = one 64-byte swizz
 constexpr int STAGES = 3;
 constexpr int CHUNK = 8;        // stages between drains: 256 K
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int THREADS = 192;
+constexpr int THREADS = 320;   // warp 0 TMA, warp 1 MMA, warps 2..9 epilogue
+constexpr int EPI_WARPS = 8;
 constexpr unsigned long long kWaitNs = 2000000000ull;
 
 template <int BN>
@@ -63,10 +65,12 @@ struct Cfg {
 struct TcArgs {
     uint32_t *C;
     int64_t ldc;
-    const uint32_t *Cin;
+    const uint32_t *Cin;   // plain mode only (stream-K mode prepares C instead)
     int64_t ldcin;
     int sgn;
     int M, N, K;
+    int tiles_m, tiles_n;
+    int split;             // 0: one CTA per tile; 1: stream-K over (tile, chunk) units
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -183,9 +187,20 @@ __global__ void __launch_bounds__(THREADS, 1)
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
     const int nk = (a.K + BK - 1) / BK;
     const int nchunks = (nk + CHUNK - 1) / CHUNK;
+    // Work of this CTA: units [u_begin, u_end) of (output tile, 256-wide K
+    // chunk), numbered tile-major; tile t covers rows (t % tiles_m) * BM and
+    // columns (t / tiles_m) * BN, so CTAs running side by side share B tiles.
+    int64_t u_begin, u_end;
+    if (a.split) {
+        const int64_t U = (int64_t)a.tiles_m * a.tiles_n * nchunks;
+        u_begin = U * blockIdx.x / gridDim.x;
+        u_end = U * (blockIdx.x + 1) / gridDim.x;
+    } else {
+        u_begin = (int64_t)blockIdx.x * nchunks;
+        u_end = u_begin + nchunks;
+    }
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -193,7 +208,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_init(&empty[s], 1);
         }
         mbar_init(acc_full, 1);
-        mbar_init(acc_empty, 4);
+        mbar_init(acc_empty, EPI_WARPS);
         mbar_init(drain, 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -213,25 +228,29 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     if (warp == 0) {
         if (lane == 0) {
-            int issued = 0;
-            for (int ks = 0; ks < nk; ++ks) {
-                const int s = ks % STAGES;
-                if (ks >= STAGES && !mbar_wait(&empty[s], ((ks / STAGES) - 1) & 1, abort_flag)) {
-                    raise_abort(abort_flag);
-                    break;
+            int64_t slot = 0;
+            for (int64_t u = u_begin; u < u_end && !*abort_flag; ++u) {
+                const int64_t tile = u / nchunks;
+                const int c = (int)(u - tile * nchunks);
+                const int m0 = (int)(tile % a.tiles_m) * BM, n0 = (int)(tile / a.tiles_m) * BN;
+                const int ks1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
+                for (int ks = c * CHUNK; ks < ks1; ++ks, ++slot) {
+                    const int s = (int)(slot % STAGES);
+                    if (slot >= STAGES && !mbar_wait(&empty[s], (uint32_t)((slot / STAGES) - 1) & 1, abort_flag)) {
+                        raise_abort(abort_flag);
+                        break;
+                    }
+                    uint8_t *st = smem + s * C::STAGE;
+                    mbar_expect_tx(&full[s], C::STAGE);
+                    tma_load_3d(st, &tmA, &full[s], ks * BK, m0, 0);
+                    tma_load_3d(st + C::A_BYTES, &tmB, &full[s], ks * BK, n0, 0);
                 }
-                uint8_t *st = smem + s * C::STAGE;
-                mbar_expect_tx(&full[s], C::STAGE);
-                tma_load_3d(st, &tmA, &full[s], ks * BK, m0, 0);
-                tma_load_3d(st + C::A_BYTES, &tmB, &full[s], ks * BK, n0, 0);
-                issued = ks + 1;
             }
             if (*abort_flag) {
                 // Let the copies this thread started land before the CTA exits.
-                const int lo = issued > STAGES ? issued - STAGES : 0;
-                for (int ks = lo; ks < issued; ++ks) {
+                for (int64_t q = slot > STAGES ? slot - STAGES : 0; q < slot; ++q) {
                     const unsigned long long t0 = gtime();
-                    while (!mbar_try(&full[ks % STAGES], (ks / STAGES) & 1) && gtime() - t0 < kWaitNs) {
+                    while (!mbar_try(&full[q % STAGES], (uint32_t)(q / STAGES) & 1) && gtime() - t0 < kWaitNs) {
                     }
                 }
             }
@@ -239,38 +258,47 @@ __global__ void __launch_bounds__(THREADS, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             bool issued_any = false;
-            for (int ks = 0; ks < nk; ++ks) {
-                const int s = ks % STAGES;
-                const int chunk = ks / CHUNK;
-                const bool first = (ks % CHUNK) == 0;
-                if (first && chunk > 0 && !mbar_wait(acc_empty, (chunk - 1) & 1, abort_flag)) {
+            int64_t slot = 0, chunk_count = 0;
+            for (int64_t u = u_begin; u < u_end && !*abort_flag; ++u) {
+                const int64_t tile = u / nchunks;
+                const int c = (int)(u - tile * nchunks);
+                const int ks0 = c * CHUNK, ks1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
+                if (chunk_count > 0 && !mbar_wait(acc_empty, (uint32_t)(chunk_count - 1) & 1, abort_flag)) {
                     raise_abort(abort_flag);
                     break;
                 }
-                if (!mbar_wait(&full[s], (ks / STAGES) & 1, abort_flag)) {
-                    raise_abort(abort_flag);
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t a_base = smem_u32(smem + s * C::STAGE);
-                const uint32_t b_base = a_base + C::A_BYTES;
+                bool ok = true;
+                for (int ks = ks0; ks < ks1; ++ks, ++slot) {
+                    const int s = (int)(slot % STAGES);
+                    if (!mbar_wait(&full[s], (uint32_t)(slot / STAGES) & 1, abort_flag)) {
+                        raise_abort(abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a_base = smem_u32(smem + s * C::STAGE);
+                    const uint32_t b_base = a_base + C::A_BYTES;
+                    const bool first = ks == ks0;
 #pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk) {
+                    for (int kk = 0; kk < BK / 16; ++kk) {
 #pragma unroll
-                    for (int g = 0; g < 4; ++g) {
+                        for (int g = 0; g < 4; ++g) {
 #pragma unroll
-                        for (int i = 0; i <= g; ++i) {
-                            const int j = g - i;
-                            const uint64_t ad = sdesc_sw64(a_base + i * C::A_PLANE + kk * 32);
-                            const uint64_t bd = sdesc_sw64(b_base + j * C::B_PLANE + kk * 32);
-                            const uint32_t acc = (first && kk == 0 && i == 0) ? 0u : 1u;
-                            umma_bf16(tmem + g * BN, ad, bd, C::IDESC, acc);
+                            for (int i = 0; i <= g; ++i) {
+                                const int j = g - i;
+                                const uint64_t ad = sdesc_sw64(a_base + i * C::A_PLANE + kk * 32);
+                                const uint64_t bd = sdesc_sw64(b_base + j * C::B_PLANE + kk * 32);
+                                const uint32_t acc = (first && kk == 0 && i == 0) ? 0u : 1u;
+                                umma_bf16(tmem + g * BN, ad, bd, C::IDESC, acc);
+                            }
                         }
                     }
+                    issued_any = true;
+                    umma_commit(&empty[s]);
                 }
-                issued_any = true;
-                umma_commit(&empty[s]);
-                if ((ks % CHUNK) == CHUNK - 1 || ks == nk - 1) umma_commit(acc_full);
+                if (!ok) break;
+                umma_commit(acc_full);
+                ++chunk_count;
             }
             if (*abort_flag && issued_any) {
                 // Products in flight still read shared memory and write TMEM.
@@ -281,25 +309,27 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
         }
     } else {
-        // Epilogue: warp w reads TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31.
+        // Epilogue: warp w reads TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31 and
+        // columns [h HB, (h + 1) HB) of each group, h = (w - 2) / 4.
+        constexpr int HB = BN / 2;
         const int q = warp & 3;
+        const int h = (warp - 2) >> 2;
         const int row = q * 32 + lane;
-        const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-        uint32_t acc[BN];
+        const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16) + h * HB;
+        uint32_t acc[HB];
 #pragma unroll
-        for (int c = 0; c < BN; ++c) acc[c] = 0u;
-        bool ok = true;
-        for (int ch = 0; ch < nchunks; ++ch) {
-            if (!mbar_wait(acc_full, ch & 1, abort_flag)) {
+        for (int c = 0; c < HB; ++c) acc[c] = 0u;
+        int64_t chunk_count = 0;
+        for (int64_t u = u_begin; u < u_end; ++u) {
+            if (!mbar_wait(acc_full, (uint32_t)chunk_count & 1, abort_flag)) {
                 raise_abort(abort_flag);
-                ok = false;
                 break;
             }
             tc_fence_after();
 #pragma unroll
             for (int g = 0; g < 4; ++g) {
 #pragma unroll
-                for (int c0 = 0; c0 < BN; c0 += 32) {
+                for (int c0 = 0; c0 < HB; c0 += 32) {
                     uint32_t v[32];
                     tmem_ld32(lane_addr + g * BN + c0, v);
 #pragma unroll
@@ -310,39 +340,53 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(acc_empty);
-        }
-        const int gm = m0 + row;
-        if (ok && gm < a.M) {
-            uint32_t *crow = a.C + (int64_t)gm * a.ldc;
-            const uint32_t *cin = a.Cin ? a.Cin + (int64_t)gm * a.ldcin : nullptr;
-            const bool vec = (n0 + BN <= a.N) && ((a.ldc & 3) == 0) &&
-                             ((reinterpret_cast<uintptr_t>(crow) & 15u) == 0) &&
-                             (!cin || (((a.ldcin & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin) & 15u) == 0)));
-            if (vec) {
+            ++chunk_count;
+
+            const int64_t tile = u / nchunks;
+            const int c = (int)(u - tile * nchunks);
+            if (c != nchunks - 1 && u != u_end - 1) continue;
+            // End of this CTA's segment of the tile: write it out.
+            const bool whole = (u_begin <= tile * nchunks) && (c == nchunks - 1);
+            const int m0 = (int)(tile % a.tiles_m) * BM, n0 = (int)(tile / a.tiles_m) * BN + h * HB;
+            const int gm = m0 + row;
+            if (gm < a.M) {
+                uint32_t *crow = a.C + (int64_t)gm * a.ldc;
+                const uint32_t *cin = a.Cin ? a.Cin + (int64_t)gm * a.ldcin : nullptr;
+                if (a.sgn < 0) {
 #pragma unroll
-                for (int c = 0; c < BN; c += 4) {
-                    uint4 o;
-                    o.x = a.sgn >= 0 ? acc[c] : 0u - acc[c];
-                    o.y = a.sgn >= 0 ? acc[c + 1] : 0u - acc[c + 1];
-                    o.z = a.sgn >= 0 ? acc[c + 2] : 0u - acc[c + 2];
-                    o.w = a.sgn >= 0 ? acc[c + 3] : 0u - acc[c + 3];
-                    if (cin) {
-                        const uint4 i4 = *reinterpret_cast<const uint4 *>(cin + n0 + c);
-                        o.x += i4.x; o.y += i4.y; o.z += i4.z; o.w += i4.w;
-                    }
-                    *reinterpret_cast<uint4 *>(crow + n0 + c) = o;
+                    for (int cc = 0; cc < HB; ++cc) acc[cc] = 0u - acc[cc];
                 }
-            } else {
+                const bool vec = (n0 + HB <= a.N) && ((a.ldc & 3) == 0) &&
+                                 ((reinterpret_cast<uintptr_t>(crow) & 15u) == 0) &&
+                                 (!cin || (((a.ldcin & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin) & 15u) == 0)));
+                if (a.split && !whole) {
+                    // Other CTAs add into this tile too: exact and order-free in Z_{2^32}.
 #pragma unroll
-                for (int c = 0; c < BN; ++c) {
-                    const int gn = n0 + c;
-                    if (gn < a.N) {
-                        uint32_t v = a.sgn >= 0 ? acc[c] : 0u - acc[c];
-                        if (cin) v += cin[gn];
-                        crow[gn] = v;
+                    for (int cc = 0; cc < HB; ++cc)
+                        if (n0 + cc < a.N) atomicAdd(crow + n0 + cc, acc[cc]);
+                } else if (vec) {
+                    // Plain mode: C = Cin + acc.  Stream-K mode: C (prepared) += acc.
+                    const uint32_t *base = a.split ? crow : cin;
+#pragma unroll
+                    for (int cc = 0; cc < HB; cc += 4) {
+                        uint4 o = make_uint4(acc[cc], acc[cc + 1], acc[cc + 2], acc[cc + 3]);
+                        if (base) {
+                            const uint4 i4 = *reinterpret_cast<const uint4 *>(base + n0 + cc);
+                            o.x += i4.x; o.y += i4.y; o.z += i4.z; o.w += i4.w;
+                        }
+                        *reinterpret_cast<uint4 *>(crow + n0 + cc) = o;
+                    }
+                } else {
+                    const uint32_t *base = a.split ? crow : cin;
+#pragma unroll
+                    for (int cc = 0; cc < HB; ++cc) {
+                        const int gn = n0 + cc;
+                        if (gn < a.N) crow[gn] = acc[cc] + (base ? base[gn] : 0u);
                     }
                 }
             }
+#pragma unroll
+            for (int cc = 0; cc < HB; ++cc) acc[cc] = 0u;
         }
     }
     tc_fence_before();
@@ -401,9 +445,34 @@ mosaic_status launch_tc(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const
             return MOSAIC_ERR_CUDA;
         attr_set |= bit;
     }
-    TcArgs args{Cm, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)K};
-    dim3 grid((unsigned)((N + BN - 1) / BN), (unsigned)((M + BM - 1) / BM));
-    ring_gemm_tc_kernel<BN><<<grid, THREADS, C::SMEM, st>>>(ta, tb, args);
+    const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = (N + BN - 1) / BN, tiles = tiles_m * tiles_n;
+    const int64_t nk = (K + BK - 1) / BK, nchunks = (nk + CHUNK - 1) / CHUNK;
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+        return MOSAIC_ERR_CUDA;
+    // One CTA per tile unless the last wave would leave more than 10% of the
+    // SMs idle; then a persistent grid shares the (tile, chunk) units evenly.
+    // Short products (fewer than 8 chunks, K < 2048) keep one CTA per tile:
+    // there the preparation of C and the split-tile atomics cost more than
+    // the idle SMs.
+    const int64_t waves = (tiles + sms - 1) / sms;
+    const bool split = nchunks >= 8 && (double)tiles / (double)(waves * sms) < 0.9;
+    TcArgs args{Cm, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)K, (int)tiles_m, (int)tiles_n, split ? 1 : 0};
+    int64_t grid = tiles;
+    if (split) {
+        // Split tiles are summed into C with atomic adds, so C starts as Cin (or 0).
+        cudaError_t e = cudaSuccess;
+        if (!Cin)
+            e = cudaMemset2DAsync(Cm, (size_t)ldc * 4, 0, (size_t)N * 4, (size_t)M, st);
+        else if (Cin != Cm)
+            e = cudaMemcpy2DAsync(Cm, (size_t)ldc * 4, Cin, (size_t)ldcin * 4, (size_t)N * 4, (size_t)M,
+                                  cudaMemcpyDeviceToDevice, st);
+        if (e != cudaSuccess) return MOSAIC_ERR_CUDA;
+        args.Cin = nullptr;
+        grid = tiles * nchunks < sms ? tiles * nchunks : sms;
+    }
+    if (grid > 0x7fffffff) return MOSAIC_ERR_SHAPE;
+    ring_gemm_tc_kernel<BN><<<(unsigned)grid, THREADS, C::SMEM, st>>>(ta, tb, args);
     return launch_status();
 }
 
@@ -424,8 +493,15 @@ mosaic_status ring_gemm_tc_planes(const uint16_t *Ap, int64_t ldpa, int64_t a_pl
                                   const uint32_t *Cin, int64_t ldcin, int sgn, int64_t M, int64_t N,
                                   int64_t K, cudaStream_t st) {
     if (M == 0 || N == 0) return MOSAIC_OK;
-    if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX || (M + BM - 1) / BM > 65535)
-        return MOSAIC_ERR_SHAPE;
+    if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX) return MOSAIC_ERR_SHAPE;
+    if (K == 0) {
+        // Empty product: C = Cin (or 0).
+        cudaError_t e = !Cin ? cudaMemset2DAsync(Cm, (size_t)ldc * 4, 0, (size_t)N * 4, (size_t)M, st)
+                       : Cin == Cm ? cudaSuccess
+                                   : cudaMemcpy2DAsync(Cm, (size_t)ldc * 4, Cin, (size_t)ldcin * 4,
+                                                       (size_t)N * 4, (size_t)M, cudaMemcpyDeviceToDevice, st);
+        return e == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
+    }
     return launch_tc<128>(Ap, ldpa, a_plane, Bp, ldpb, b_plane, Cm, ldc, Cin, ldcin, sgn, M, N, K, st);
 }
 

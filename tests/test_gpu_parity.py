@@ -260,10 +260,26 @@ def _check_layer(g, ref, op, m, l):
     assert np.all(np.abs(g["Y"].astype(np.float64) - Yref) <= 1e-6 * mag)
 
 
+def _variants():
+    M = M_()
+    out = [M.GEMM_IMAD]
+    if M.mosaic_gemm_variant_available(M.GEMM_TC):
+        out.append(M.GEMM_TC)
+    return out
+
+
 @pytest.mark.parametrize("d,r,t", [(1, (96,), ()), (2, (96, 64), (6,)), (3, (96, 64, 40), (6, 5))])
 def test_layer_small_ranks(d, r, t):
-    g, ref, op, m, l = _run_layer(d, r, t, m=40, n=100, l=21)
-    _check_layer(g, ref, op, m, l)
+    for variant in _variants():
+        g, ref, op, m, l = _run_layer(d, r, t, m=40, n=100, l=21, variant=variant)
+        _check_layer(g, ref, op, m, l)
+
+
+def test_layer_ranks_not_multiple_of_eight():
+    """r_d = 37 and m, l ragged: every product has a ragged K tail."""
+    for variant in _variants():
+        g, ref, op, m, l = _run_layer(3, (100, 70, 37), (9, 7), m=131, n=300, l=67, variant=variant)
+        _check_layer(g, ref, op, m, l)
 
 
 def test_layer_zero_noise_and_no_bias():
@@ -282,5 +298,5 @@ def test_layer_single_64x256x128():
 def test_layer_attn_proj_7b_full():
     """Attention projection at 7B shape (X 512x4096, W 4096x4096), full oracle."""
     g, ref, op, m, l = _run_layer(3, (1536, 1024, 652), (80, 80), m=4096, n=4096, l=512,
-                                  w_std=0.02)
+                                  w_std=0.02, variant=_variants()[-1])
     _check_layer(g, ref, op, m, l)

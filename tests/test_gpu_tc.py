@@ -80,7 +80,7 @@ def test_tc_random(Mm, N, K):
     assert np.array_equal(tc_gemm(A, B), ref(A, B))
 
 
-@pytest.mark.parametrize("K", [256, 512, 1024, 768 + 32])
+@pytest.mark.parametrize("K", [256, 512, 1024, 768 + 32, 2048])
 @pytest.mark.parametrize("va,vb", [(ALL_M128, ALL_M128), (ALL_P127, ALL_M128), (ALL_P127, ALL_P127)])
 def test_tc_adversarial_digits(K, va, vb):
     A = np.full((128, K), va, np.uint32)
