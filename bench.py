@@ -49,6 +49,21 @@ def _peaks():
         return 6800.0, 1900.0, 1700.0, "fallback"
 
 
+def _traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu capture (profiles/traffic.json),
+    or None if the kernel's source changed since the capture."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f)[kernel]
+        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
+                return None
+        return float(rec["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -226,8 +241,9 @@ def run_mine(args, rank, world):
     ring_tops = 2 * ring_macs / (gemm_ms / 1e3) / 1e12
     if variant == M.GEMM_TC:
         achieved = 10 * 2 * ring_macs / (gemm_ms / 1e3) / 1e12      # bf16 digit-pair flops
+        traffic = _traffic("ring_gemm_tc") if args.workload == "attn_proj_7b_512x4096x4096" else None
         roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": bf16, "unit": "TFLOP/s",
-                "frac": round(achieved / bf16, 4), "traffic": None,
+                "frac": round(achieved / bf16, 4), "traffic": traffic,
                 "kernel": "ring_gemm_tc (10 bf16 digit-pair products per ring MAC)",
                 "peak_source": f"{peak_src} bf16 dense burst"}
     else:

@@ -46,6 +46,7 @@ struct GatherArgs {
     const float *s_w, *s_x, *bias;
     float *Y;
     int64_t ldy;
+    int trusted;   // positions known to be < r (drawn by this library)
 };
 
 // Staged rows plus the per-warp list rings.
@@ -60,7 +61,7 @@ constexpr size_t gather_smem(int tg, int64_t segp) {
 // warp serves 32 / TG list entities; the TG lanes of an entity share its
 // (position, value) loads (16-byte, prefetched 16 pairs at a time) and keep
 // four independent partial sums.
-template <int TG, bool LIST_IS_COL>
+template <int TG, bool LIST_IS_COL, bool CLAMP>
 __global__ void __launch_bounds__(GW * 32) gather_kernel(GatherArgs a) {
     constexpr int EPW = 32 / TG;
     extern __shared__ uint32_t sg[];
@@ -120,9 +121,12 @@ __global__ void __launch_bounds__(GW * 32) gather_kernel(GatherArgs a) {
         const int R = (t + 15) >> 4;
         const int steps = n_ent * R;
         uint32_t *ring = sg + ((int64_t)TG * a.segp + 3) / 4 * 4 + warp * (kRing * 32 * EPW);
+        // (ik, ir): entity iteration and round of the next step to issue.
+        int ik = 0, ir = 0;
         auto issue = [&](int s) {
+            const int k = ik, rr = ir;
+            if (++ir == R) { ir = 0; ++ik; }
             if (lane < 8 * EPW && s < steps) {
-                const int k = s / R, rr = s - k * R;
                 const int he = lane >> 3, part = lane & 7;
                 const int64_t e = e_begin + warp * EPW + he + (int64_t)k * stride;
                 const int q = rr * 16 + (part & 3) * 4;
@@ -147,10 +151,10 @@ __global__ void __launch_bounds__(GW * 32) gather_kernel(GatherArgs a) {
 #pragma unroll
             for (int u = 0; u < 4; u++) {
                 const uint4 I = slot[u], V = slot[4 + u];
-                s0 += V.x * row_g[min(I.x, rlast)];
-                s1 += V.y * row_g[min(I.y, rlast)];
-                s2 += V.z * row_g[min(I.z, rlast)];
-                s3 += V.w * row_g[min(I.w, rlast)];
+                s0 += V.x * row_g[CLAMP ? min(I.x, rlast) : I.x];
+                s1 += V.y * row_g[CLAMP ? min(I.y, rlast) : I.y];
+                s2 += V.z * row_g[CLAMP ? min(I.z, rlast) : I.z];
+                s3 += V.w * row_g[CLAMP ? min(I.w, rlast) : I.w];
             }
             __syncwarp();
             if (rr == R - 1) {
@@ -173,33 +177,33 @@ __global__ void __launch_bounds__(GW * 32) gather_kernel(GatherArgs a) {
     }
 }
 
-template <int TG, bool LIST_IS_COL>
+template <int TG, bool LIST_IS_COL, bool CLAMP>
 mosaic_status launch_gather(const GatherArgs &a, cudaStream_t st) {
     const size_t smem = gather_smem(TG, a.segp);
     if (smem > 48 * 1024 &&
-        cudaFuncSetAttribute(gather_kernel<TG, LIST_IS_COL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaFuncSetAttribute(gather_kernel<TG, LIST_IS_COL, CLAMP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem) != cudaSuccess)
         return MOSAIC_ERR_CUDA;
     dim3 grid((unsigned)((a.nlist + G_ENTS - 1) / G_ENTS), (unsigned)((a.g_count + TG - 1) / TG));
     if (grid.y > 65535) return MOSAIC_ERR_SHAPE;
-    gather_kernel<TG, LIST_IS_COL><<<grid, GW * 32, smem, st>>>(a);
+    gather_kernel<TG, LIST_IS_COL, CLAMP><<<grid, GW * 32, smem, st>>>(a);
     return launch_status();
 }
 
-template <bool LIST_IS_COL>
+template <bool LIST_IS_COL, bool CLAMP>
 mosaic_status dispatch_gather(GatherArgs a, cudaStream_t st) {
     a.segp = (int64_t)(a.r + 31) / 32 * 32 + 1;
     // The largest row tile with which two CTAs fit on an SM (one CTA stages
     // while the other gathers); else the largest that fits at all.
     const size_t two = 113 * 1024, one = 220 * 1024;
     for (size_t cap : {two, one}) {
-        if (gather_smem(32, a.segp) <= cap) return launch_gather<32, LIST_IS_COL>(a, st);
-        if (gather_smem(16, a.segp) <= cap) return launch_gather<16, LIST_IS_COL>(a, st);
-        if (gather_smem(8, a.segp) <= cap) return launch_gather<8, LIST_IS_COL>(a, st);
-        if (gather_smem(4, a.segp) <= cap) return launch_gather<4, LIST_IS_COL>(a, st);
+        if (gather_smem(32, a.segp) <= cap) return launch_gather<32, LIST_IS_COL, CLAMP>(a, st);
+        if (gather_smem(16, a.segp) <= cap) return launch_gather<16, LIST_IS_COL, CLAMP>(a, st);
+        if (gather_smem(8, a.segp) <= cap) return launch_gather<8, LIST_IS_COL, CLAMP>(a, st);
+        if (gather_smem(4, a.segp) <= cap) return launch_gather<4, LIST_IS_COL, CLAMP>(a, st);
     }
-    if (gather_smem(2, a.segp) <= one) return launch_gather<2, LIST_IS_COL>(a, st);
-    if (gather_smem(1, a.segp) <= one) return launch_gather<1, LIST_IS_COL>(a, st);
+    if (gather_smem(2, a.segp) <= one) return launch_gather<2, LIST_IS_COL, CLAMP>(a, st);
+    if (gather_smem(1, a.segp) <= one) return launch_gather<1, LIST_IS_COL, CLAMP>(a, st);
     return MOSAIC_ERR_SHAPE;
 }
 
@@ -224,7 +228,14 @@ mosaic_status gather_levels(GatherArgs base, bool list_is_col, const SparseLevel
         if (!last) {
             g.out = scratch_out; g.ldo = ld_scratch; g.decode = 0;
         }
-        MOSAIC_TRY(list_is_col ? dispatch_gather<true>(g, st) : dispatch_gather<false>(g, st));
+        // Lists drawn by this library's sampler are in range by construction;
+        // lists from callers are clamped per read.
+        mosaic_status rc;
+        if (base.trusted)
+            rc = list_is_col ? dispatch_gather<true, false>(g, st) : dispatch_gather<false, false>(g, st);
+        else
+            rc = list_is_col ? dispatch_gather<true, true>(g, st) : dispatch_gather<false, true>(g, st);
+        if (rc != MOSAIC_OK) return rc;
     }
     return MOSAIC_OK;
 }
@@ -327,6 +338,7 @@ mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, i
     GatherArgs g{};
     g.src = src; g.lds = lds; g.g_count = g_count; g.nlist = nlist;
     g.a = a; g.lda = lda; g.b = b; g.ldb = ldb; g.sgn = sgn; g.out = out; g.ldo = ldo;
+    g.trusted = 1;   // the T lists of Init X come from prg_sparse
     // Later levels accumulate in place in `out`.
     return gather_levels(g, list_is_col, lev, nlev, out, ldo, st);
 }
