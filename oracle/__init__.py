@@ -109,6 +109,9 @@ def _declare(L):
     L.orc_sample_gaussian.argtypes = [_P, _U32, _U64, _INT, _P, _INT, _I64, _P]
     L.orc_sample_sparse.argtypes = [_P, _U32, _U64, _INT, _I64, _U32, _INT, _P, _P]
     L.orc_sample_sparse.restype = _INT
+    L.orc_sample_gaussian_at.argtypes = [_P, _U32, _U64, _INT, _P, _INT, _I64, _I64, _P]
+    L.orc_sample_sparse_row.argtypes = [_P, _U32, _U64, _INT, _I64, _U32, _INT, _P, _P]
+    L.orc_sample_sparse_row.restype = _INT
     L.orc_fwht_rows.argtypes = [_P, _I64, _I64, _I64, _I64, _P, _P]
     L.orc_fwht_rows_f64.argtypes = [_P, _I64, _I64, _P, _P]
     L.orc_encode_rows.argtypes = [_P, _I64, _I64, ctypes.c_int32, _P, _P]
@@ -198,6 +201,29 @@ def sample_sparse(key, tg: int, stream_id: int, rows: int, r: int, t: int, round
     val = np.zeros((rows, t), np.uint32)
     st = lib().orc_sample_sparse(_ptr(k), tg, stream_id, rounds, rows, r, t, _ptr(idx), _ptr(val))
     if st != 0:
+        raise RuntimeError("sparse sampler exhausted a row window")
+    return idx, val
+
+
+def sample_gaussian_at(key, tg: int, stream_id: int, first: int, count: int, sigma: float,
+                       rounds: int = 20) -> np.ndarray:
+    """Elements [first, first + count) of the Gaussian stream of sample_gaussian."""
+    out = np.zeros(count, np.uint32)
+    if float(sigma) == 0.0 or count == 0:
+        return out
+    k = _c(key, np.uint32)
+    table = gaussian_table(sigma)
+    lib().orc_sample_gaussian_at(_ptr(k), tg, stream_id, rounds, _ptr(table), gaussian_bound(sigma),
+                                 first, count, _ptr(out))
+    return out
+
+
+def sample_sparse_row(key, tg: int, stream_id: int, row: int, r: int, t: int, rounds: int = 20):
+    """Row `row` of the sparse matrix of sample_sparse: (idx, val), each of length t."""
+    k = _c(key, np.uint32)
+    idx = np.zeros(t, np.uint32)
+    val = np.zeros(t, np.uint32)
+    if lib().orc_sample_sparse_row(_ptr(k), tg, stream_id, rounds, row, r, t, _ptr(idx), _ptr(val)) != 0:
         raise RuntimeError("sparse sampler exhausted a row window")
     return idx, val
 

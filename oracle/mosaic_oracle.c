@@ -111,6 +111,25 @@ void orc_sample_gaussian(const uint32_t key[8], uint32_t tag, uint64_t stream_id
     free(w);
 }
 
+/* Elements [first, first + count) of the same Gaussian stream (element e
+ * still reads words 2e and 2e + 1), for sampled checks of large matrices. */
+void orc_sample_gaussian_at(const uint32_t key[8], uint32_t tag, uint64_t stream_id, int rounds,
+                            const uint64_t *table, int bound, int64_t first, int64_t count,
+                            uint32_t *out)
+{
+    uint32_t *w = (uint32_t *)malloc(sizeof(uint32_t) * 2 * (size_t)(count > 0 ? count : 1));
+    orc_prg_words(key, tag, stream_id, rounds, 2 * (uint64_t)first, 2 * count, w);
+    for (int64_t e = 0; e < count; e++) {
+        uint64_t u = (uint64_t)w[2 * e] | ((uint64_t)w[2 * e + 1] << 32);
+        int32_t k = bound;
+        for (int j = 0; j <= 2 * bound; j++) {
+            if (u < table[j]) { k = j - bound; break; }
+        }
+        out[e] = (uint32_t)k;
+    }
+    free(w);
+}
+
 /* Sparse rows with exactly t nonzeros (LPN noise of Hamming weight t,
  * Example 3.1; S_i and T_i in the Sec. 3.2 box).  Row j draws from its own
  * window of 65536 stream words starting at word j * 65536: positions
@@ -143,6 +162,28 @@ int orc_sample_sparse(const uint32_t key[8], uint32_t tag, uint64_t stream_id, i
     }
     free(w);
     return status;
+}
+
+/* Row `row` alone of the sparse matrix above (same window, same rule). */
+int orc_sample_sparse_row(const uint32_t key[8], uint32_t tag, uint64_t stream_id, int rounds,
+                          int64_t row, uint32_t r, int t, uint32_t *idx, uint32_t *val)
+{
+    uint32_t *w = (uint32_t *)malloc(sizeof(uint32_t) * ORC_SPARSE_WINDOW);
+    orc_prg_words(key, tag, stream_id, rounds, (uint64_t)row * ORC_SPARSE_WINDOW, ORC_SPARSE_WINDOW, w);
+    int pos = 0, got = 0, nv = 0;
+    while (got < t && pos < ORC_SPARSE_WINDOW) {
+        uint32_t p = (uint32_t)(((uint64_t)w[pos++] * r) >> 32);
+        int seen = 0;
+        for (int q = 0; q < got; q++)
+            if (idx[q] == p) { seen = 1; break; }
+        if (!seen) idx[got++] = p;
+    }
+    while (nv < t && pos < ORC_SPARSE_WINDOW) {
+        uint32_t v = w[pos++];
+        if (v != 0) val[nv++] = v;
+    }
+    free(w);
+    return (got < t || nv < t) ? -1 : 0;
 }
 
 /* ---------------------------------------------------------------------- */
