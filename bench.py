@@ -1,26 +1,29 @@
 """Benchmark of the masked secure linear layer on GB300.
 
-One step = one pass of the whole per-call path of Pi_Sec-Linear over one
-batch of l tokens: Init X (PRG masks R, T_i, E_x and U_x, K), rotation +
-encode + mask-add of X, the server's ring product Z = X' [W'; P]^T over
-Z_{2^32}, and the unmask + decode.  Init W (public chains and the masked
-weights) is one-time and is timed apart (``init_w_s``).
+One step = one pass of the whole per-call path of Pi_Sec-Linear over one batch
+of tokens: Init X (PRG masks R, T_i, E_x and U_x, K), rotation + encode +
+mask-add of X, the server's ring product Z = X' [W'; P]^T over Z_{2^32}, and the
+unmask + decode.  Init W (public chains and the masked weights) is one-time and
+is timed apart (``init_w_s``).
 
-Default workload: the attention projection at 7B shape (X 512 x 4096,
-W 4096 x 4096, Example 3.1 parameters).  Inputs are seeded synthetic
-(activations ~ N(0,1), weights ~ N(0,0.02)).  L2 is flushed (256 MiB write)
-between timed steps.
+Workloads (``--workload``; seeded synthetic inputs, activations ~ N(0,1),
+weights ~ N(0,0.02), Example 3.1 parameters):
+  attn_proj_7b_512x4096x4096   (default) X 512 x 4096, W 4096 x 4096
+  ffn_7b_2048x4096x14336       up 4096 -> 14336 then down 14336 -> 4096, 2048 tokens
+  decoder_70b_prefill_2048     one 70B decoder layer: 4 masked linears + fp32
+                               RMSNorm / attention / SwiGLU / residuals, 2048 tokens
+  decode_70b_sweep             every linear of a 70B layer at 1..256 tokens
+L2 is flushed (256 MiB write) between timed steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
 
-Prints one JSON line (rank 0).  With N > 1 (torchrun), every rank runs an
+Prints one JSON line (rank 0).  With N > 1 (torchrun) every rank runs an
 independent replica on its own GPU (weak scaling, no data-path collective).
 """
 from __future__ import annotations
 
 import argparse
 import json
-import math
 import os
 import subprocess
 import sys
@@ -37,6 +40,7 @@ from paper_2607_29221_gb300 import workloads as wl  # noqa: E402
 
 METRIC = "masked ring-GEMM effective TOPS (Z_2^32) and masked-layer tokens/s; % of roofline"
 L2_FLUSH_BYTES = 256 << 20
+DEFAULT_WORKLOAD = "attn_proj_7b_512x4096x4096"
 
 
 def _peaks():
@@ -70,8 +74,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="mine", choices=["mine", "reference"])
-    ap.add_argument("--workload", default="attn_proj_7b_512x4096x4096")
-    ap.add_argument("--variant", default="auto", choices=["auto", "tc", "mma", "imad"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(wl.WORKLOADS))
+    ap.add_argument("--variant", default="auto", choices=["auto", "tc", "imad"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     return ap.parse_args()
@@ -135,8 +139,129 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------
+# workloads
+# ---------------------------------------------------------------------------
+class _Timed:
+    """CUDA events around the server products of the steps being timed."""
+
+    def __init__(self, stream):
+        self.stream = stream
+        self.active = False
+        self.pairs = []
+
+    def wrap(self, layer):
+        import torch
+        server = layer.server
+
+        def timed_server(*a, **k):
+            if not self.active:
+                return server(*a, **k)
+            e0 = torch.cuda.Event(enable_timing=True); e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(self.stream)
+            out = server(*a, **k)
+            e1.record(self.stream)
+            self.pairs.append((e0, e1))
+            return out
+        layer.server = timed_server
+
+
+class LinearChain:
+    """Secure linear calls in sequence, each call's decoded output feeding the
+    next (attention projection: one call; FFN: up then down)."""
+
+    def __init__(self, proto, dev, linears, l, rank, timed):
+        import torch
+        from paper_2607_29221_gb300 import protocol as PR
+        self.l, self.rank = l, rank
+        chains = {}
+        self.layers, self.bufs = [], []
+        for i, lin in enumerate(linears):
+            n_pad = PR.pad_width(lin.n)
+            if n_pad not in chains:
+                chains[n_pad] = PR.Chains(proto, n_pad)
+            W = torch.from_numpy(wl.weights(lin.m, lin.n, seed=wl.SEED_W + i, std=lin.w_std)).to(dev)
+            b = torch.from_numpy(wl.bias(lin.m, seed=wl.SEED_B + i)).to(dev)
+            layer = PR.SecureLinear(proto, W, 1 + i, chains[n_pad], bias=b)
+            timed.wrap(layer)
+            self.layers.append(layer)
+            Sr = proto.sum_r
+            self.bufs.append(dict(
+                Xp=torch.empty(l, n_pad, dtype=torch.int32, device=dev),
+                s_x=torch.empty(l, dtype=torch.float32, device=dev),
+                Xpl=torch.empty(4, l, n_pad, dtype=torch.int16, device=dev) if layer.use_planes else None,
+                Z=torch.empty(l, lin.m + Sr, dtype=torch.int32, device=dev),
+                Y=torch.empty(l, lin.m, dtype=torch.float32, device=dev)))
+        self.ring_macs = sum(l * (ly.m + proto.sum_r) * ly.n_pad for ly in self.layers)
+        self.n_in, self.m_out = linears[0].n, linears[-1].m
+
+    def step(self, x, i):
+        for c, (layer, bf) in enumerate(zip(self.layers, self.bufs)):
+            mp = layer.init_x(self.l, 1_000_000 * self.rank + 1000 * c + i)
+            layer.mask_input(x, mp, bf["Xp"], bf["s_x"], bf["Xpl"])
+            layer.server(bf["Xp"], bf["Xpl"], bf["Z"])
+            layer.unmask(bf["Z"], mp, bf["s_x"], bf["Y"])
+            x = bf["Y"]
+        return x
+
+
+class DecoderLayerRun:
+    """One 70B decoder layer: four masked linears and the fp32 glue."""
+
+    def __init__(self, proto, dev, l, rank, timed):
+        from paper_2607_29221_gb300 import decoder as D
+        s = D.LayerShape()
+        self.layer = D.SecureDecoderLayer(proto, D.LayerWeights(s, seed=11, device=dev))
+        for lin in self.layer.linears():
+            timed.wrap(lin)
+        self.ring_macs = sum(l * (lin.m + proto.sum_r) * lin.n_pad for lin in self.layer.linears())
+        self.n_in = self.m_out = s.hidden
+        self.l = l
+
+    def step(self, x, i):
+        return self.layer.forward(x)
+
+
+class LinearSet:
+    """Independent secure linear calls on the same tokens (decode sweep)."""
+
+    def __init__(self, chain_parts):
+        self.parts = chain_parts
+        self.ring_macs = sum(p.ring_macs for p in chain_parts)
+
+    def step(self, xs, i):
+        return [p.step(x, i) for p, x in zip(self.parts, xs)]
+
+
+# ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
+def _time_steps(torch, runner, make_input, steps, warmup, flush, stream, timed, world, counter=None):
+    for i in range(warmup):
+        runner.step(make_input(), i)
+    torch.cuda.synchronize()
+    _barrier(world)
+    torch.cuda.synchronize()
+    evs = []
+    timed.active = True
+    c0 = counter() if counter else 0
+    for i in range(steps):
+        flush.fill_(i & 0xFF)
+        x = make_input()
+        s0 = torch.cuda.Event(enable_timing=True); s1 = torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        runner.step(x, warmup + i)
+        s1.record(stream)
+        evs.append((s0, s1))
+    timed.active = False
+    launches = (counter() - c0) if counter else 0
+    torch.cuda.synchronize()
+    _barrier(world)
+    step_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    gemm_ms = float(np.sum([a.elapsed_time(b) for a, b in timed.pairs])) / steps if timed.pairs else 0.0
+    timed.pairs.clear()
+    return step_ms, gemm_ms, launches
+
+
 def run_mine(args, rank, world):
     import torch
     import __graft_entry__ as G
@@ -146,89 +271,55 @@ def run_mine(args, rank, world):
     G.build()
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
-    wk = wl.WORKLOADS[args.workload]
-    lin = wk.linears[0]
-    m, n, l = lin.m, lin.n, wk.l
-    n_pad = PR.pad_width(n)
-    variant = {"auto": M.GEMM_AUTO, "tc": M.GEMM_TC, "mma": M.GEMM_MMA_S8, "imad": M.GEMM_IMAD}[args.variant]
+    variant = {"auto": M.GEMM_AUTO, "tc": M.GEMM_TC, "imad": M.GEMM_IMAD}[args.variant]
     if variant == M.GEMM_AUTO:
         variant = M.GEMM_TC if M.mosaic_gemm_variant_available(M.GEMM_TC) else M.GEMM_IMAD
-    key = wl.mask_key()
-    proto = PR.Protocol(key, M.default_params(), variant=variant)
-    Sr = proto.sum_r
+    proto = PR.Protocol(wl.mask_key(), M.default_params(), variant=variant)
+    stream = torch.cuda.current_stream()
+    timed = _Timed(stream)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    wk = wl.WORKLOADS[args.workload]
 
-    W = torch.from_numpy(wl.weights(m, n, std=lin.w_std)).to(dev)
-    b = torch.from_numpy(wl.bias(m)).to(dev)
-    X_host = torch.from_numpy(wl.activations(l, n, seed=wl.SEED_X + rank)).pin_memory()
-    X = X_host.to(dev)
+    if args.workload == "decode_70b_sweep":
+        return run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed, flush, wk,
+                                variant)
 
     torch.cuda.synchronize()
     t0 = time.perf_counter()
-    chains = PR.Chains(proto, n_pad)
-    layer = PR.SecureLinear(proto, W, 1, chains, bias=b)
+    if args.workload == "decoder_70b_prefill_2048":
+        runner = DecoderLayerRun(proto, dev, wk.l, rank, timed)
+    else:
+        runner = LinearChain(proto, dev, list(wk.linears), wk.l, rank, timed)
     torch.cuda.synchronize()
     init_w_s = time.perf_counter() - t0
 
-    # persistent per-step buffers
-    Xp = torch.empty(l, n_pad, dtype=torch.int32, device=dev)
-    s_x = torch.empty(l, dtype=torch.float32, device=dev)
-    Xpl = torch.empty(4, l, n_pad, dtype=torch.int16, device=dev) if layer.use_planes else None
-    Z = torch.empty(l, m + Sr, dtype=torch.int32, device=dev)
-    Y = torch.empty(l, m, dtype=torch.float32, device=dev)
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
-    stream = torch.cuda.current_stream()
-
-    gemm_ev = []
-
-    def step(i, record=False):
-        mp = layer.init_x(l, 1000 * rank + i)
-        layer.mask_input(X, mp, Xp, s_x, Xpl)
-        if record:
-            e0 = torch.cuda.Event(enable_timing=True); e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-        layer.server(Xp, Xpl, Z)
-        if record:
-            e1.record(stream)
-            gemm_ev.append((e0, e1))
-        layer.unmask(Z, mp, s_x, Y)
-
-    for i in range(args.warmup):
-        step(i)
-    torch.cuda.synchronize()
+    l = wk.l
+    X_host = torch.from_numpy(wl.activations(l, runner.n_in, seed=wl.SEED_X + rank)).pin_memory()
+    X = X_host.to(dev)
 
     sampler = ClockSampler(_smi_index(dev.index))
     sampler.start()
     time.sleep(0.3)
-    _barrier(world)
-    torch.cuda.synchronize()
-    evs = []
-    for i in range(args.steps):
-        flush.fill_(i & 0xFF)
-        s0 = torch.cuda.Event(enable_timing=True); s1 = torch.cuda.Event(enable_timing=True)
-        s0.record(stream)
-        step(args.warmup + i, record=True)
-        s1.record(stream)
-        evs.append((s0, s1))
-    torch.cuda.synchronize()
-    _barrier(world)
-    step_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
-    gemm_ms = float(np.mean([a.elapsed_time(b) for a, b in gemm_ev]))
+    # our kernels launched inside the timed region, from the library's own counter
+    step_ms, gemm_ms, launches_timed = _time_steps(torch, runner, lambda: X, args.steps, args.warmup, flush,
+                                                   stream, timed, world, M.mosaic_kernel_launches)
 
     # end to end through the public API with host buffers
-    Y_host = torch.empty(l, m, dtype=torch.float32).pin_memory()
+    Y_host = torch.empty(l, runner.m_out, dtype=torch.float32).pin_memory()
     e2e = []
     for i in range(max(3, args.steps // 2)):
         flush.fill_(i & 0xFF)
         a = torch.cuda.Event(enable_timing=True); c = torch.cuda.Event(enable_timing=True)
         a.record(stream)
         X.copy_(X_host, non_blocking=True)
-        step(10_000 + i)
+        Y = runner.step(X, 10_000 + i)
         Y_host.copy_(Y, non_blocking=True)
         c.record(stream)
         e2e.append((a, c))
     torch.cuda.synchronize()
     e2e_ms = float(np.mean([a.elapsed_time(c) for a, c in e2e]))
     clocks = sampler.stop()
+    M.mosaic_device_status()
 
     step_ms_max = _max_over_ranks(step_ms, world, dev)
     e2e_ms_max = _max_over_ranks(e2e_ms, world, dev)
@@ -236,50 +327,109 @@ def run_mine(args, rank, world):
         return
 
     hbm, bf16, bf16_sus, peak_src = _peaks()
-    ring_macs = l * (m + Sr) * n_pad                       # server product Z = X' [W'; P]^T
     tokens_s = world * l / (step_ms_max / 1e3)
-    ring_tops = 2 * ring_macs / (gemm_ms / 1e3) / 1e12
-    if variant == M.GEMM_TC:
-        achieved = 10 * 2 * ring_macs / (gemm_ms / 1e3) / 1e12      # bf16 digit-pair flops
-        traffic = _traffic("ring_gemm_tc") if args.workload == "attn_proj_7b_512x4096x4096" else None
-        roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": bf16, "unit": "TFLOP/s",
-                "frac": round(achieved / bf16, 4), "traffic": traffic,
-                "kernel": "ring_gemm_tc (10 bf16 digit-pair products per ring MAC)",
-                "peak_source": f"{peak_src} bf16 dense burst"}
-    else:
-        imad_peak = 152 * 64 * 2 * 2.07e9 / 1e12               # ring-ops/s: 64 IMAD/clk/SM, 2 ops each
-        roof = {"bound": "alu", "achieved": round(ring_tops, 3), "peak": round(imad_peak, 2),
-                "unit": "TOPS", "frac": round(ring_tops / imad_peak, 4), "traffic": None,
-                "kernel": "ring_gemm_imad", "peak_source": "derived: 152 SMs x 64 IMAD/clk x 2070 MHz"}
-    launches_per_step = _launches_per_step(proto.d, layer.use_planes)
+    ring_tops = 2 * runner.ring_macs / (gemm_ms / 1e3) / 1e12
+    roof = _roofline(variant, M, runner.ring_macs, gemm_ms, bf16, peak_src,
+                     _traffic("ring_gemm_tc") if args.workload == DEFAULT_WORKLOAD else None)
+    cfg = {"workload": args.workload, "l": l,
+           "linears": [{"name": x.name, "m": x.m, "n": x.n} for x in wk.linears],
+           "params": "Example 3.1: d=3, r=1536/1024/652, t=80/80, sigma=0.5, b=16",
+           "gemm_variant": {M.GEMM_TC: "tc", M.GEMM_IMAD: "imad"}[variant],
+           "l2": "flushed between timed steps (256 MiB write)",
+           "parallelism": f"replicas x{world}"}
+    if args.workload == "decoder_70b_prefill_2048":
+        cfg["glue"] = "fp32 RMSNorm, causal GQA attention (64 q / 8 kv heads, d 128), SwiGLU, residuals"
     out = {
         "metric": METRIC, "value": round(tokens_s, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms_max, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
         "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights)",
-        "config": {"workload": args.workload, "l": l, "m": m, "n": n, "n_pad": n_pad,
-                   "params": "Example 3.1: d=3, r=1536/1024/652, t=80/80, sigma=0.5, b=16",
-                   "gemm_variant": {M.GEMM_TC: "tc", M.GEMM_IMAD: "imad", M.GEMM_MMA_S8: "mma_s8"}[variant],
-                   "l2": "flushed between timed steps (256 MiB write)",
-                   "parallelism": f"replicas x{world}"},
+        "config": cfg,
         "ring_tops": round(ring_tops, 2),
         "gemm_ms": round(gemm_ms, 4),
         "init_w_s": round(init_w_s, 3),
         "roofline": roof,
         "e2e": {"value": round(world * l / (e2e_ms_max / 1e3), 1), "unit": "tokens/s",
-                "h2d_bytes_per_step": l * n * 4, "d2h_bytes_per_step": l * m * 4},
-        "gpu_launches": launches_per_step * args.steps,
+                "h2d_bytes_per_step": l * runner.n_in * 4, "d2h_bytes_per_step": l * runner.m_out * 4},
+        "gpu_launches": int(launches_timed),
         "clocks": clocks,
     }
-    if world == 1 and not args.no_cpu_baseline:
+    if world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD:
         out["cpu_baseline"] = cpu_baseline(wk, args.cpu_budget_s)
     print(json.dumps(out), flush=True)
 
 
-def _launches_per_step(d: int, planes: bool) -> int:
-    # Init X: R, E_x, (d-1) sparse T, U_x product, K product, 2 sparse gathers (d > 1)
-    init_x = 4 + (d - 1) + (2 if d > 1 else 0)
-    return init_x + 1 + (1 if planes else 1) + 2      # encode, server product, unmask (2)
+def _roofline(variant, M, ring_macs, gemm_ms, bf16, peak_src, traffic):
+    ring_tops = 2 * ring_macs / (gemm_ms / 1e3) / 1e12
+    if variant == M.GEMM_TC:
+        achieved = 10 * 2 * ring_macs / (gemm_ms / 1e3) / 1e12      # bf16 digit-pair flops
+        return {"bound": "tensor", "achieved": round(achieved, 2), "peak": bf16, "unit": "TFLOP/s",
+                "frac": round(achieved / bf16, 4), "traffic": traffic,
+                "kernel": "ring_gemm_tc (10 bf16 digit-pair products per ring MAC)",
+                "peak_source": f"{peak_src} bf16 dense burst"}
+    imad_peak = 152 * 64 * 2 * 2.07e9 / 1e12               # ring-ops/s: 64 IMAD/clk/SM, 2 ops each
+    return {"bound": "alu", "achieved": round(ring_tops, 3), "peak": round(imad_peak, 2),
+            "unit": "TOPS", "frac": round(ring_tops / imad_peak, 4), "traffic": None,
+            "kernel": "ring_gemm_imad", "peak_source": "derived: 152 SMs x 64 IMAD/clk x 2070 MHz"}
+
+
+def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed, flush, wk, variant):
+    """Every linear of one 70B layer at 1..256 tokens against pre-masked weights."""
+    hbm, bf16, _, peak_src = _peaks()
+    t0 = time.perf_counter()
+    parts = {l: LinearSet([LinearChain(proto, dev, [lin], l, rank, timed) for lin in wk.linears])
+             for l in wk.decode_batches[:1]}
+    init_w_s = time.perf_counter() - t0
+    base = parts[wk.decode_batches[0]]
+    sweep = []
+    sampler = ClockSampler(_smi_index(dev.index))
+    sampler.start()
+    time.sleep(0.3)
+    for l in wk.decode_batches:
+        # the same pre-masked weights serve every batch size; only the per-call buffers differ
+        runs = []
+        for chain in base.parts:
+            c = LinearChain.__new__(LinearChain)
+            c.l, c.rank, c.layers = l, rank, chain.layers
+            c.bufs = [dict(
+                Xp=torch.empty(l, ly.n_pad, dtype=torch.int32, device=dev),
+                s_x=torch.empty(l, dtype=torch.float32, device=dev),
+                Xpl=torch.empty(4, l, ly.n_pad, dtype=torch.int16, device=dev) if ly.use_planes else None,
+                Z=torch.empty(l, ly.m + proto.sum_r, dtype=torch.int32, device=dev),
+                Y=torch.empty(l, ly.m, dtype=torch.float32, device=dev)) for ly in chain.layers]
+            c.ring_macs = sum(l * (ly.m + proto.sum_r) * ly.n_pad for ly in chain.layers)
+            runs.append(c)
+        runner = LinearSet(runs)
+        xs = [torch.from_numpy(wl.activations(l, ly.n, seed=wl.SEED_X + l)).to(dev)
+              for c in runs for ly in c.layers]
+        step_ms, gemm_ms, _ = _time_steps(torch, runner, lambda: xs, args.steps, args.warmup, flush, stream,
+                                          timed, world)
+        w_bytes = sum((ly.m + proto.sum_r) * ly.n_pad * 4 for c in runs for ly in c.layers)
+        plane_bytes = 2 * w_bytes
+        sweep.append({"l": l, "ms_per_step": round(step_ms, 4), "tokens_s": round(world * l / (step_ms / 1e3), 1),
+                      "gemm_ms": round(gemm_ms, 4), "ring_tops": round(2 * runner.ring_macs / (gemm_ms / 1e3) / 1e12, 2),
+                      "w_prime_bytes": w_bytes,
+                      "w_prime_gbs": round(w_bytes / (gemm_ms / 1e3) / 1e9, 1),
+                      "w_prime_hbm_frac": round(w_bytes / (gemm_ms / 1e3) / 1e9 / hbm, 4),
+                      "plane_gbs": round(plane_bytes / (gemm_ms / 1e3) / 1e9, 1)})
+    clocks = sampler.stop()
+    M.mosaic_device_status()
+    if rank != 0:
+        return
+    first = sweep[0]
+    out = {"metric": METRIC, "value": first["tokens_s"], "unit": "tokens/s", "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": first["ms_per_step"],
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+           "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights)",
+           "config": {"workload": args.workload, "batches": list(wk.decode_batches),
+                      "linears": [{"name": x.name, "m": x.m, "n": x.n} for x in wk.linears],
+                      "params": "Example 3.1", "l2": "flushed between timed steps (256 MiB write)"},
+           "init_w_s": round(init_w_s, 3), "sweep": sweep,
+           "roofline": {"bound": "hbm", "achieved": first["plane_gbs"], "peak": hbm, "unit": "GB/s",
+                        "frac": round(first["plane_gbs"] / hbm, 4), "traffic": None,
+                        "kernel": "ring_gemm_tc at 1 token (bf16 digit planes of W', 8 B per element)"},
+           "clocks": clocks}
+    print(json.dumps(out), flush=True)
 
 
 def _smi_index(dev_index: int) -> int:
@@ -353,7 +503,7 @@ def cpu_baseline(wk, budget_s, tokens=None):
 def run_reference(args, rank, world):
     if rank != 0:
         return
-    wk = wl.WORKLOADS[args.workload]
+    wk = wl.WORKLOADS[DEFAULT_WORKLOAD if args.workload not in (DEFAULT_WORKLOAD,) else args.workload]
     O, key, p, P, C, ws, init_s = _oracle_setup(wk)
     lin = wk.linears[0]
     l = min(wk.l, 64)               # bounded sample of the workload's tokens per step
@@ -372,7 +522,7 @@ def run_reference(args, rank, world):
            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": round(sec * 1e3, 3), "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "u32", "data": "synthetic",
-           "config": {"workload": args.workload, "l": wk.l, "m": lin.m, "n": lin.n,
+           "config": {"workload": wk.name, "l": wk.l, "m": lin.m, "n": lin.n,
                       "params": "Example 3.1"},
            "cpu_baseline": {"value": round(val, 2), "unit": "tokens/s", "cores": O.num_threads(),
                             "kind": "oracle",

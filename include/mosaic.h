@@ -78,6 +78,10 @@ typedef struct {
  * t = 80/80, sigma = 0.5, b = 16, 20 rounds, kappa = 32). */
 void mosaic_default_params(mosaic_params *p);
 
+/* Number of kernels this library has launched in this process (all devices,
+ * all threads; host-side counter, for benchmarking). */
+uint64_t mosaic_kernel_launches(void);
+
 /* Human-readable name of a status code (static string). */
 const char *mosaic_status_string(mosaic_status s);
 

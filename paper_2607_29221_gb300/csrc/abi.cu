@@ -5,9 +5,16 @@
 #include <math.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "mosaic_internal.cuh"
 
 using namespace mosaic;
+
+namespace mosaic {
+static std::atomic<unsigned long long> g_launches{0};
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+}  // namespace mosaic
 
 namespace {
 
@@ -131,6 +138,8 @@ size_t ws_unmask(int64_t m, int64_t l, const mosaic_params *p) {
 }  // namespace
 
 extern "C" {
+
+uint64_t mosaic_kernel_launches(void) { return mosaic::g_launches.load(std::memory_order_relaxed); }
 
 void mosaic_default_params(mosaic_params *p) {
     if (!p) return;

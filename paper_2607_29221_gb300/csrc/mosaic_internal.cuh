@@ -55,9 +55,14 @@ inline Key to_key(const mosaic_key *k) {
 
 inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
 
+// Counts every kernel this library launches (read by mosaic_kernel_launches).
+void count_launch();
+
 inline mosaic_status launch_status() {
     cudaError_t e = cudaGetLastError();
-    return e == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
+    if (e != cudaSuccess) return MOSAIC_ERR_CUDA;
+    count_launch();
+    return MOSAIC_OK;
 }
 
 #define MOSAIC_TRY(expr)                        \

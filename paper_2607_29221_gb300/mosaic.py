@@ -50,6 +50,7 @@ _PK = ctypes.POINTER(mosaic_key)
 
 _SIGS = {
     "mosaic_default_params": ([_PP], None),
+    "mosaic_kernel_launches": ([], ctypes.c_uint64),
     "mosaic_status_string": ([_INT], ctypes.c_char_p),
     "mosaic_qmax": ([_I64, _U32], ctypes.c_int32),
     "mosaic_gaussian_table": ([_F32, _P, _INT], _INT),
@@ -144,6 +145,10 @@ def _call(name, *args):
 
 
 # ---------------------------------------------------------------------------
+def mosaic_kernel_launches() -> int:
+    return int(lib().mosaic_kernel_launches())
+
+
 def mosaic_qmax(n_pad: int, qbits: int = 16) -> int:
     return int(lib().mosaic_qmax(n_pad, qbits))
 
