@@ -394,7 +394,8 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
             c.bufs = [dict(
                 Xp=torch.empty(l, ly.n_pad, dtype=torch.int32, device=dev),
                 s_x=torch.empty(l, dtype=torch.float32, device=dev),
-                Xpl=torch.empty(4, l, ly.n_pad, dtype=torch.int16, device=dev) if ly.use_planes else None,
+                Xpl=(torch.empty(4, l, ly.n_pad, dtype=torch.int16, device=dev)
+                     if ly.use_planes and l > M.SKINNY_MAX_M else None),
                 Z=torch.empty(l, ly.m + proto.sum_r, dtype=torch.int32, device=dev),
                 Y=torch.empty(l, ly.m, dtype=torch.float32, device=dev)) for ly in chain.layers]
             c.ring_macs = sum(l * (ly.m + proto.sum_r) * ly.n_pad for ly in chain.layers)
@@ -405,13 +406,17 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
         step_ms, gemm_ms, _ = _time_steps(torch, runner, lambda: xs, args.steps, args.warmup, flush, stream,
                                           timed, world)
         w_bytes = sum((ly.m + proto.sum_r) * ly.n_pad * 4 for c in runs for ly in c.layers)
-        plane_bytes = 2 * w_bytes
+        # up to SKINNY_MAX_M tokens the server streams uint32 W' (4 B an element),
+        # beyond that the tensor cores read its bf16 digit planes (8 B an element)
+        skinny = variant != M.GEMM_IMAD and l <= M.SKINNY_MAX_M
+        read_bytes = w_bytes if skinny or variant == M.GEMM_IMAD else 2 * w_bytes
         sweep.append({"l": l, "ms_per_step": round(step_ms, 4), "tokens_s": round(world * l / (step_ms / 1e3), 1),
                       "gemm_ms": round(gemm_ms, 4), "ring_tops": round(2 * runner.ring_macs / (gemm_ms / 1e3) / 1e12, 2),
-                      "w_prime_bytes": w_bytes,
-                      "w_prime_gbs": round(w_bytes / (gemm_ms / 1e3) / 1e9, 1),
-                      "w_prime_hbm_frac": round(w_bytes / (gemm_ms / 1e3) / 1e9 / hbm, 4),
-                      "plane_gbs": round(plane_bytes / (gemm_ms / 1e3) / 1e9, 1)})
+                      "server_kernel": "ring_gemm_skinny" if skinny else
+                                       ("ring_gemm_imad" if variant == M.GEMM_IMAD else "ring_gemm_tc"),
+                      "w_prime_bytes": w_bytes, "server_read_bytes": read_bytes,
+                      "server_read_gbs": round(read_bytes / (gemm_ms / 1e3) / 1e9, 1),
+                      "server_hbm_frac": round(read_bytes / (gemm_ms / 1e3) / 1e9 / hbm, 4)})
     clocks = sampler.stop()
     M.mosaic_device_status()
     if rank != 0:
@@ -425,9 +430,10 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
                       "linears": [{"name": x.name, "m": x.m, "n": x.n} for x in wk.linears],
                       "params": "Example 3.1", "l2": "flushed between timed steps (256 MiB write)"},
            "init_w_s": round(init_w_s, 3), "sweep": sweep,
-           "roofline": {"bound": "hbm", "achieved": first["plane_gbs"], "peak": hbm, "unit": "GB/s",
-                        "frac": round(first["plane_gbs"] / hbm, 4), "traffic": None,
-                        "kernel": "ring_gemm_tc at 1 token (bf16 digit planes of W', 8 B per element)"},
+           "roofline": {"bound": "hbm", "achieved": first["server_read_gbs"], "peak": hbm, "unit": "GB/s",
+                        "frac": first["server_hbm_frac"], "traffic": None, "peak_source": peak_src,
+                        "kernel": first["server_kernel"] + " at %d token(s): reads of the server operand"
+                                  % first["l"]},
            "clocks": clocks}
     print(json.dumps(out), flush=True)
 

@@ -84,6 +84,9 @@ mosaic_status gemm_u32(int variant, Carve &cv, const uint32_t *A, int64_t sai, i
                        const uint32_t *Cin, int64_t ldcin, int sgn, int64_t M, int64_t N, int64_t K,
                        cudaStream_t st) {
     const bool want_tc = variant == MOSAIC_GEMM_TC || (variant == MOSAIC_GEMM_AUTO && tc_available());
+    // A few tokens: stream B once at 4 bytes per element instead of its planes.
+    if (want_tc && sak == 1 && sbk == 1 && skinny_ok(A, sai, B, sbj, M, K))
+        return ring_gemm_skinny(A, sai, B, sbj, C, ldc, Cin, ldcin, sgn, M, N, K, st);
     const bool tc_ok = want_tc && sak == 1 && sbk == 1 && sai % 4 == 0 && sbj % 4 == 0 &&
                        aligned16(A) && aligned16(B) && K > 0 && cv.used + ws_gemm(M, N, K) <= cv.cap;
     if (!tc_ok) return ring_gemm_imad(A, sai, sak, B, sbj, sbk, C, ldc, Cin, ldcin, sgn, M, N, K, st);
@@ -277,12 +280,20 @@ mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B
     if (M == 0 || N == 0) return MOSAIC_OK;
     if (!A || !B || !C) return MOSAIC_ERR_ARG;
     cudaStream_t st = as_stream(stream);
-    if (variant == MOSAIC_GEMM_IMAD || (variant == MOSAIC_GEMM_AUTO && !tc_available()))
+    if (K == 0)   // empty sums: C = 0 whatever the variant
+        return cudaMemset2DAsync(C, (size_t)ldc * 4, 0, (size_t)N * 4, (size_t)M, st) == cudaSuccess
+                   ? MOSAIC_OK
+                   : MOSAIC_ERR_CUDA;
+    const bool tc_layout = aligned16(A) && aligned16(B) && lda % 4 == 0 && ldb % 4 == 0;
+    if (variant == MOSAIC_GEMM_IMAD || (variant == MOSAIC_GEMM_AUTO && (!tc_available() || !tc_layout)))
         return ring_gemm_imad(A, lda, 1, B, ldb, 1, C, ldc, nullptr, 0, 1, M, N, K, st);
     if (variant == MOSAIC_GEMM_MMA_S8)
         return ring_gemm_mma_s8(A, lda, B, ldb, C, ldc, nullptr, 0, 1, M, N, K, st);
-    // Tensor-core variant: split both operands into digit planes in ws.
     if (!tc_available()) return MOSAIC_ERR_UNSUPPORTED;
+    // A few tokens: the streaming kernel reads B once, no planes needed.
+    if (skinny_ok(A, lda, B, ldb, M, K))
+        return ring_gemm_skinny(A, lda, B, ldb, C, ldc, nullptr, 0, 1, M, N, K, st);
+    // Tensor-core variant: split both operands into digit planes in ws.
     const int64_t Kp = (K + 7) / 8 * 8;
     if (!aligned16(A) || !aligned16(B) || lda % 4 || ldb % 4) return MOSAIC_ERR_ALIGN;
     Carve cv{static_cast<char *>(ws), ws_bytes, 0};
@@ -314,7 +325,9 @@ mosaic_status mosaic_ring_gemm_planes(const uint16_t *A_planes, int64_t ldpa, in
 
 mosaic_status mosaic_device_status(void *stream) {
     const mosaic_status s = device_status(as_stream(stream));
+    const mosaic_status s2 = skinny_status();
     if (s != MOSAIC_OK) return s;
+    if (s2 != MOSAIC_OK) return s2;
     return cudaGetLastError() == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
 }
 

@@ -171,6 +171,23 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
 #pragma unroll
         for (int e = 0; e < E; e++) v[e] = 0.0f;
     }
+    // Element index of the run-th group of CS outputs this thread writes.
+    auto out_elem = [&](int run) -> int {
+        if constexpr (WN > 1) return run * 32 * E + lt * CS;
+        else return base;
+    };
+    // The mask words this thread adds at the end are loaded now, so that their
+    // latency overlaps the rotation (rows up to 16384 words: longer rows run
+    // 1024-thread blocks whose register budget has no room for them).
+    constexpr bool kPrefetch = N <= 16384;
+    uint32_t mk_pre[kPrefetch ? E : 1];
+    if constexpr (kPrefetch) {
+        if (a.mode == 1 && a.mask && active) {
+            const uint32_t *mr = a.mask + row * a.ldm;
+#pragma unroll
+            for (int run = 0; run < RUNS; run++) load_u32<CS>(mr + out_elem(run), mk_pre + run * CS);
+        }
+    }
 
     if (a.rotate) {
         if (a.signs) {
@@ -291,13 +308,18 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
         code[e] = (uint32_t)c;
     }
     if (a.mask) {
-        const uint32_t *mr = a.mask + row * a.ldm;
+        if constexpr (kPrefetch) {
 #pragma unroll
-        for (int run = 0; run < RUNS; run++) {
-            uint32_t mk[CS];
-            load_u32<CS>(mr + elem(run), mk);
+            for (int e = 0; e < E; e++) code[e] += mk_pre[e];
+        } else {
+            const uint32_t *mr = a.mask + row * a.ldm;
 #pragma unroll
-            for (int u = 0; u < CS; u++) code[run * CS + u] += mk[u];
+            for (int run = 0; run < RUNS; run++) {
+                uint32_t mk[CS];
+                load_u32<CS>(mr + elem(run), mk);
+#pragma unroll
+                for (int u = 0; u < CS; u++) code[run * CS + u] += mk[u];
+            }
         }
     }
     uint32_t *orow = a.out + row * a.ldo;

@@ -119,6 +119,18 @@ bool tc_available();
 mosaic_status device_status(cudaStream_t st);
 bool mma_s8_available();
 
+// Streaming ring GEMM for a few tokens (NT, uint32, K-contiguous):
+// C = (Cin?) + sgn * A B^T with 1 <= M <= kSkinnyMaxM, each element of B read
+// once through TMA.  skinny_ok() tells whether the operands qualify (16-byte
+// aligned bases, row strides multiples of 4 words, a Blackwell device).
+constexpr int64_t kSkinnyMaxM = 16;
+bool skinny_ok(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb, int64_t M, int64_t K);
+mosaic_status ring_gemm_skinny(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb,
+                               uint32_t *C, int64_t ldc, const uint32_t *Cin, int64_t ldcin, int sgn,
+                               int64_t M, int64_t N, int64_t K, cudaStream_t st);
+// Reads and clears the streaming kernel's timeout word (after a stream sync).
+mosaic_status skinny_status();
+
 // Sparse gathers.
 // out[row][col] = a[row][col] - b[row][col] (b nullable) + sgn * sum_lev sum_q val * src[g][off_lev + idx]
 // where (list entity, staged row g) = (row, col) if !list_is_col else (col, row).

@@ -21,6 +21,7 @@ STATUS = {0: "ok", 1: "invalid argument", 2: "invalid shape", 3: "misaligned", 4
           5: "CUDA error", 6: "workspace too small", 7: "device wait timed out"}
 
 GEMM_AUTO, GEMM_TC, GEMM_MMA_S8, GEMM_IMAD = 0, 1, 2, 3
+SKINNY_MAX_M = 16   # MOSAIC_SKINNY_MAX_M: token counts the streaming product serves
 OP_RING_GEMM, OP_MASK_CHAINS, OP_MASK_WEIGHT, OP_MASK_ACTIVATION, OP_UNMASK = 1, 2, 3, 4, 5
 TAG_M, TAG_N, TAG_L, TAG_S, TAG_EW, TAG_R, TAG_T, TAG_EX, TAG_SIGN = range(1, 10)
 
@@ -170,8 +171,9 @@ def mosaic_device_status(stream=None):
     _call("mosaic_device_status", _stream(stream))
 
 
-def mosaic_workspace_bytes(op: int, m: int, n_pad: int, l: int, params: mosaic_params) -> int:
-    return int(lib().mosaic_workspace_bytes(op, m, n_pad, l, ctypes.byref(params)))
+def mosaic_workspace_bytes(op: int, m: int, n_pad: int, l: int, params: mosaic_params = None) -> int:
+    return int(lib().mosaic_workspace_bytes(op, m, n_pad, l,
+                                            None if params is None else ctypes.byref(params)))
 
 
 def mosaic_prg_uniform(key, tag, stream_id, rounds, rows, cols, out, ldo=None, stream=None):

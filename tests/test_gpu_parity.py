@@ -282,6 +282,22 @@ def test_layer_ranks_not_multiple_of_eight():
         _check_layer(g, ref, op, m, l)
 
 
+@pytest.mark.parametrize("l", [1, 2, 5, 16, 17])
+def test_layer_few_tokens(l):
+    """Decode-size token counts: up to 16 tokens the server and the per-pass
+    client products stream their uint32 operands (aligned ranks here)."""
+    for variant in _variants():
+        g, ref, op, m, l = _run_layer(3, (96, 64, 40), (6, 5), m=200, n=256, l=l, variant=variant)
+        _check_layer(g, ref, op, m, l)
+
+
+def test_layer_one_token_example_params():
+    """One token through the 64x256x128 shape with Example 3.1 parameters."""
+    g, ref, op, m, l = _run_layer(3, (1536, 1024, 652), (80, 80), m=128, n=256, l=1,
+                                  variant=M_().GEMM_AUTO)
+    _check_layer(g, ref, op, m, l)
+
+
 def test_layer_zero_noise_and_no_bias():
     g, ref, op, m, l = _run_layer(3, (96, 64, 40), (6, 5), m=33, n=64, l=9, sigma=0.0, bias=False)
     _check_layer(g, ref, op, m, l)

@@ -119,3 +119,70 @@ def test_tc_protocol_layer_matches_oracle():
     g, r, op, m, l = T._run_layer(3, (1536, 1024, 652), (80, 80), m=128, n=256, l=64,
                                   variant=_M().GEMM_TC)
     T._check_layer(g, r, op, m, l)
+
+
+# --------------------------------------------------------------------------
+# Few tokens (M <= 16): the TC variant streams uint32 B through TMA instead of
+# splitting it into planes; same ring product, checked the same way.
+# --------------------------------------------------------------------------
+def ring_gemm_u32(A, B, pad_a=0, pad_b=0, variant=None):
+    M = _M()
+    variant = M.GEMM_TC if variant is None else variant
+    Mm, K = A.shape
+    N = B.shape[0]
+    lda = (K + 3) // 4 * 4 + pad_a
+    ldb = (K + 3) // 4 * 4 + pad_b
+    Ad = torch.zeros(Mm, lda, dtype=torch.int32, device="cuda")
+    Bd = torch.zeros(N, ldb, dtype=torch.int32, device="cuda")
+    Ad[:, :K] = dev(A)
+    Bd[:, :K] = dev(B)
+    C = torch.full((Mm, N + 4), -1, dtype=torch.int32, device="cuda")
+    nb = M.mosaic_workspace_bytes(M.OP_RING_GEMM, Mm, N, K)
+    ws = torch.empty(max(nb, 16), dtype=torch.uint8, device="cuda")
+    M.mosaic_ring_gemm(Ad, lda, Bd, ldb, C, N + 4, Mm, N, K, variant, ws)
+    M.mosaic_device_status()
+    got = host(C)
+    assert np.all(got[:, N:] == 0xFFFFFFFF)
+    return got[:, :N]
+
+
+@pytest.mark.parametrize("Mm", [1, 2, 3, 4, 5, 8, 9, 16])
+@pytest.mark.parametrize("N,K", [(1, 1), (61, 128), (59, 129), (300, 652), (1000, 4100), (121, 8192)])
+def test_few_tokens_random(Mm, N, K):
+    A = wl.uniform_u32(31 + Mm, Mm, K)
+    B = wl.uniform_u32(37, N, K)
+    assert np.array_equal(ring_gemm_u32(A, B), ref(A, B))
+
+
+@pytest.mark.parametrize("val", [0xFFFFFFFF, 0x80000000, ALL_M128, ALL_P127])
+def test_few_tokens_constant(val):
+    """Constant operands: every row of C is K * val^2 mod 2^32 exactly."""
+    Mm, N, K = 7, 190, 1000
+    A = np.full((Mm, K), val, dtype=np.uint32)
+    B = np.full((N, K), val, dtype=np.uint32)
+    want = np.uint32((K * val * val) % (1 << 32))
+    assert np.all(ring_gemm_u32(A, B) == want)
+
+
+def test_few_tokens_unaligned_rows():
+    """Row strides that are not multiples of 4 words: AUTO takes the CUDA-core
+    product, TC refuses them as misaligned."""
+    M = _M()
+    A = wl.uniform_u32(41, 3, 130)
+    B = wl.uniform_u32(42, 77, 130)
+    assert np.array_equal(ring_gemm_u32(A, B, pad_a=1, pad_b=3, variant=M.GEMM_AUTO), ref(A, B))
+    with pytest.raises(M.MosaicError, match="misaligned"):
+        ring_gemm_u32(A, B, pad_a=1, pad_b=3, variant=M.GEMM_TC)
+
+
+def test_few_tokens_edges():
+    """17 tokens leave the streaming kernel; K = 0 gives zeros."""
+    A = wl.uniform_u32(43, 17, 300)
+    B = wl.uniform_u32(44, 65, 300)
+    assert np.array_equal(ring_gemm_u32(A, B), ref(A, B))
+    M = _M()
+    C = torch.full((2, 8), -1, dtype=torch.int32, device="cuda")
+    Z = torch.zeros(2, 4, dtype=torch.int32, device="cuda")
+    M.mosaic_ring_gemm(Z, 4, Z, 4, C, 8, 2, 2, 0, M.GEMM_TC)
+    got = host(C)
+    assert np.all(got[:, :2] == 0) and np.all(got[:, 2:] == 0xFFFFFFFF)
