@@ -177,6 +177,261 @@ __global__ void __launch_bounds__(GW * 32) gather_kernel(GatherArgs a) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Persistent tiled gather (lists with t a multiple of 4 and 16-byte aligned,
+// segments of up to kPgMaxR words).
+//
+// A tile is 32 rows g of the level's segment, staged TRANSPOSED: the 32 rows'
+// words at position p form one 128-byte line (line p at byte 128 p), whose
+// eight 16-byte chunks are XOR-permuted by (p >> 2) & 7: rows 4c .. 4c+3 sit
+// in chunk c ^ ((p >> 2) & 7).  A warp serves four list entities at a time,
+// eight lanes each; lane i of an entity reads rows 4i .. 4i+3 at position p
+// with one 16-byte load, so the eight lanes of an entity read one whole line
+// (all 32 banks) and every 16-byte access phase is conflict-free.
+// Staging: a warp loads 4 rows x 32 positions (four 128-byte segments, one
+// 16-byte load a lane) and each of its four 4-byte stores hits 32 distinct
+// banks thanks to the permutation.
+// The (position, value) lists stream through a two-slot per-warp ring in
+// rounds of 16 pairs (cp.async, zero-filled past the end of a list).  Once a
+// round has landed, each lane rewrites two of its entity's positions into
+// line addresses with the permutation bits in place (clamping positions of
+// caller lists to r - 1), so that the gather loop needs one XOR per pair.
+// Work units are (tile, 64 entities), numbered tile-major and split evenly
+// over a persistent grid, so a CTA stages each of its one or two tiles once.
+// ---------------------------------------------------------------------------
+constexpr int kPgRows = 32;
+constexpr int kPgWarps = 16;
+constexpr int kPgEnts = 4 * kPgWarps;       // entities per unit
+constexpr int kPgSlot = 4 * 36;             // words per ring slot: 4 entities x (16 idx + 16 val + 4 pad)
+constexpr int kPgRing = 2;
+constexpr uint32_t kPgMaxR = 1632;
+
+size_t pgather_smem(uint32_t r) {   // + 128 bytes to align the stage to a line
+    return (size_t)((r + 31) / 32 * 32) * kPgRows * 4 + (size_t)kPgWarps * kPgRing * kPgSlot * 4 + 128;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(addr)
+                 : "memory");
+    return v;
+}
+__device__ __forceinline__ void sts32(uint32_t addr, uint32_t v) {
+    asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+constexpr int kPgStageBatch = 12;  // 16-byte loads a lane keeps in flight while staging
+
+template <bool LIST_IS_COL, bool CLAMP>
+__global__ void __launch_bounds__(kPgWarps * 32, 1)
+    pgather_kernel(GatherArgs a, int64_t units, int chunks, int vec_src) {
+    extern __shared__ __align__(16) uint32_t sm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int grp = lane >> 3, li = lane & 7;
+    const int r = (int)a.r, rp = (r + 31) / 32 * 32, t = a.t;
+    const uint32_t sm_base = ((uint32_t)__cvta_generic_to_shared(sm) + 127u) & ~127u;
+    const uint32_t ring_base = sm_base + 4u * (uint32_t)(rp * kPgRows + warp * (kPgRing * kPgSlot));
+    const int64_t u_begin = units * blockIdx.x / gridDim.x;
+    const int64_t u_end = units * (blockIdx.x + 1) / gridDim.x;
+    const int R = (t + 15) >> 4;
+    const int64_t steps = (u_end - u_begin) * R;
+    const uint32_t rlast = a.r - 1;
+    const uint32_t lane_chunk = 16u * (uint32_t)li;   // rows 4 li .. 4 li + 3 of a line, before permutation
+
+    // Prefetch cursor: the (round, entity chunk) of the next list round to copy.
+    int64_t i_step = 0;
+    int i_rr = 0, i_chunk = (int)(u_begin % chunks);
+    auto issue = [&]() {
+        if (i_step < steps) {
+            const int64_t e = (int64_t)i_chunk * kPgEnts + warp * 4 + grp;
+            const int part = li;   // 0..3: positions, 4..7: values
+            const int q = i_rr * 16 + (part & 3) * 4;
+            const bool ok = e < a.nlist && q < t;
+            const uint32_t *src = (part < 4 ? a.idx : a.val) + (ok ? e * t + q : 0);
+            const uint32_t dst = ring_base + 4u * (uint32_t)((int)(i_step & 1) * kPgSlot + grp * 36 +
+                                                             (part < 4 ? 0 : 16) + (part & 3) * 4);
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(ok ? 16 : 0)
+                         : "memory");
+            if (++i_rr == R) {
+                i_rr = 0;
+                if (++i_chunk == chunks) i_chunk = 0;
+            }
+        }
+        ++i_step;
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+
+    // Transposed, permuted copy of rows tile*32 .. +31 (zeros past the ends).
+    // Lane (gl, pq) of a warp loads words p .. p+3 (p = 32 b + 4 pq) of row
+    // 4 j + gl and stores word p+k in line p+k, chunk j ^ (((p+k) >> 2) & 7):
+    // for each k the 32 stores fall in 32 distinct banks.  Each lane keeps
+    // kPgStageBatch 16-byte loads in flight.
+    auto stage = [&](int64_t tile) {
+        const int64_t g0 = tile * kPgRows;
+        const int gl = lane >> 3, pq = lane & 7;
+        const int total = 8 * (rp / 32);
+        for (int it0 = warp; it0 < total; it0 += kPgWarps * kPgStageBatch) {
+            uint4 w[kPgStageBatch];
+#pragma unroll
+            for (int j = 0; j < kPgStageBatch; j++) {
+                const int it = it0 + j * kPgWarps;
+                const int g = (it & 7) * 4 + gl;
+                const int p = (it >> 3) * 32 + pq * 4;
+                w[j] = make_uint4(0u, 0u, 0u, 0u);
+                if (it < total && g0 + g < a.g_count && p < r) {
+                    const uint32_t *srow = a.src + (g0 + g) * a.lds + a.col0;
+                    if (vec_src && p + 4 <= r) {
+                        w[j] = __ldg(reinterpret_cast<const uint4 *>(srow + p));
+                    } else {
+                        w[j].x = srow[p];
+                        if (p + 1 < r) w[j].y = srow[p + 1];
+                        if (p + 2 < r) w[j].z = srow[p + 2];
+                        if (p + 3 < r) w[j].w = srow[p + 3];
+                    }
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < kPgStageBatch; j++) {
+                const int it = it0 + j * kPgWarps;
+                if (it < total) {
+                    const int g = (it & 7) * 4 + gl;
+                    const int p = (it >> 3) * 32 + pq * 4;
+                    const uint32_t v[4] = {w[j].x, w[j].y, w[j].z, w[j].w};
+#pragma unroll
+                    for (int k = 0; k < 4; k++) {
+                        const uint32_t pp = (uint32_t)(p + k);
+                        sts32(sm_base + (pp << 7) + ((((uint32_t)g >> 2) ^ (pp >> 2)) & 7u) * 16u +
+                                  4u * (uint32_t)(g & 3),
+                              v[k]);
+                    }
+                }
+            }
+        }
+    };
+
+    // The epilogue operands a - b of a unit's outputs are loaded when the unit
+    // starts, so that their latency hides behind the unit's rounds.
+    auto prefetch_ab = [&](int64_t tile, int64_t e, uint32_t (&ab)[4]) {
+#pragma unroll
+        for (int c = 0; c < 4; c++) {
+            const int64_t g = tile * kPgRows + li * 4 + c;
+            const int64_t row = LIST_IS_COL ? g : e;
+            const int64_t col = LIST_IS_COL ? e : g;
+            uint32_t v = 0u;
+            if (e < a.nlist && g < a.g_count) {
+                if (a.a) v += a.a[row * a.lda + col];
+                if (a.b) v -= a.b[row * a.ldb + col];
+            }
+            ab[c] = v;
+        }
+    };
+    auto finish = [&](int64_t tile, int64_t e, const uint32_t (&acc)[4], const uint32_t (&ab)[4]) {
+        if (e >= a.nlist) return;
+#pragma unroll
+        for (int c = 0; c < 4; c++) {
+            const int64_t g = tile * kPgRows + li * 4 + c;
+            if (g >= a.g_count) break;
+            const int64_t row = LIST_IS_COL ? g : e;
+            const int64_t col = LIST_IS_COL ? e : g;
+            const uint32_t res = (a.sgn >= 0 ? acc[c] : 0u - acc[c]) + ab[c];
+            if (a.out) a.out[row * a.ldo + col] = res;
+            if (a.decode) {
+                float y = __fmul_rn(__fmul_rn(__int2float_rn((int32_t)res), a.s_w[col]), a.s_x[row]);
+                if (a.bias) y = __fadd_rn(y, a.bias[col]);
+                a.Y[row * a.ldy + col] = y;
+            }
+        }
+    };
+
+    issue();
+    int64_t tile = u_begin / chunks;
+    int chunk = (int)(u_begin % chunks), rr = 0;
+    uint32_t acc[4] = {0u, 0u, 0u, 0u};
+    uint32_t ab[4] = {0u, 0u, 0u, 0u};
+    for (int64_t s = 0; s < steps; s++) {
+        if (rr == 0 && (s == 0 || chunk == 0)) {   // a new tile: the same step for every warp
+            __syncthreads();
+            stage(tile);
+            __syncthreads();
+        }
+        if (rr == 0) prefetch_ab(tile, (int64_t)chunk * kPgEnts + warp * 4 + grp, ab);
+        issue();
+        asm volatile("cp.async.wait_group 1;" ::: "memory");
+        __syncwarp();
+        const uint32_t slot = ring_base + 4u * (uint32_t)((int)(s & 1) * kPgSlot + grp * 36);
+        {
+            // Positions 2 li, 2 li + 1 of the round -> line address | permutation bits.
+            uint32_t p0, p1;
+            asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(p0), "=r"(p1) : "r"(slot + 8u * li) : "memory");
+            if (CLAMP) {
+                p0 = min(p0, rlast);
+                p1 = min(p1, rlast);
+            }
+            p0 = sm_base + (p0 << 7) + ((p0 << 2) & 0x70u);
+            p1 = sm_base + (p1 << 7) + ((p1 << 2) & 0x70u);
+            asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(slot + 8u * li), "r"(p0), "r"(p1) : "memory");
+        }
+        __syncwarp();
+#pragma unroll
+        for (int u4 = 0; u4 < 4; u4++) {
+            const uint4 I = lds128(slot + 16u * u4);
+            const uint4 V = lds128(slot + 64u + 16u * u4);
+            const uint32_t pi[4] = {I.x, I.y, I.z, I.w};
+            const uint32_t vi[4] = {V.x, V.y, V.z, V.w};
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                const uint4 x = lds128(pi[c] ^ lane_chunk);
+                acc[0] += vi[c] * x.x;
+                acc[1] += vi[c] * x.y;
+                acc[2] += vi[c] * x.z;
+                acc[3] += vi[c] * x.w;
+            }
+        }
+        __syncwarp();
+        if (++rr == R) {
+            finish(tile, (int64_t)chunk * kPgEnts + warp * 4 + grp, acc, ab);
+            acc[0] = acc[1] = acc[2] = acc[3] = 0u;
+            rr = 0;
+            if (++chunk == chunks) {
+                chunk = 0;
+                ++tile;
+            }
+        }
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
+template <bool LIST_IS_COL, bool CLAMP>
+mosaic_status launch_pgather(const GatherArgs &a, cudaStream_t st) {
+    const size_t smem = pgather_smem(a.r);
+    auto kern = pgather_kernel<LIST_IS_COL, CLAMP>;
+    static unsigned long long attr_set = 0;   // one bit per device ordinal
+    int dev = 0, sms = 0, per_sm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return MOSAIC_ERR_CUDA;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(attr_set & bit)) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) !=
+            cudaSuccess)
+            return MOSAIC_ERR_CUDA;
+        attr_set |= bit;
+    }
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kPgWarps * 32, smem) != cudaSuccess ||
+        per_sm < 1)
+        return MOSAIC_ERR_CUDA;
+    const int64_t tiles = (a.g_count + kPgRows - 1) / kPgRows;
+    const int64_t chunks = (a.nlist + kPgEnts - 1) / kPgEnts;
+    const int64_t units = tiles * chunks;
+    const int64_t slots = (int64_t)sms * per_sm;
+    const int64_t grid = units < slots ? units : slots;
+    if (chunks > 0x7fffffff) return MOSAIC_ERR_SHAPE;
+    const int vec_src = aligned16(a.src) && a.lds % 4 == 0 && a.col0 % 4 == 0;
+    kern<<<(unsigned)grid, kPgWarps * 32, smem, st>>>(a, units, (int)chunks, vec_src);
+    return launch_status();
+}
+
 template <int TG, bool LIST_IS_COL, bool CLAMP>
 mosaic_status launch_gather(const GatherArgs &a, cudaStream_t st) {
     const size_t smem = gather_smem(TG, a.segp);
@@ -192,6 +447,9 @@ mosaic_status launch_gather(const GatherArgs &a, cudaStream_t st) {
 
 template <bool LIST_IS_COL, bool CLAMP>
 mosaic_status dispatch_gather(GatherArgs a, cudaStream_t st) {
+    const bool lists_vec = a.t > 0 && (a.t & 3) == 0 &&
+                           ((reinterpret_cast<uintptr_t>(a.idx) | reinterpret_cast<uintptr_t>(a.val)) & 15u) == 0;
+    if (lists_vec && a.r >= 1 && a.r <= kPgMaxR) return launch_pgather<LIST_IS_COL, CLAMP>(a, st);
     a.segp = (int64_t)(a.r + 31) / 32 * 32 + 1;
     // The largest row tile with which two CTAs fit on an SM (one CTA stages
     // while the other gathers); else the largest that fits at all.

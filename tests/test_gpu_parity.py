@@ -298,6 +298,52 @@ def test_layer_one_token_example_params():
     _check_layer(g, ref, op, m, l)
 
 
+@pytest.mark.parametrize("r,t", [((98, 70, 37), (8, 4)), ((96, 64, 40), (16, 12)),
+                                 ((1536, 1024, 652), (80, 80))])
+def test_layer_tiled_gather_shapes(r, t):
+    """Hamming weights that are multiples of 4 take the tiled gather: ragged
+    row tiles (m = 131, l = 67), segments that are not multiples of 32 and a
+    segment offset that is not 16-byte aligned (r_1 = 98)."""
+    for variant in _variants():
+        g, ref, op, m, l = _run_layer(3, r, t, m=131, n=300, l=67, variant=variant)
+        _check_layer(g, ref, op, m, l)
+
+
+def test_unmask_clamps_out_of_range_positions():
+    """Caller-supplied S positions at or beyond r_i are read as r_i - 1 (no
+    read leaves the staged segment): the unmask with positions 2^32 - 1 gives
+    the same Y_hat as with positions r_i - 1."""
+    from paper_2607_29221_gb300 import protocol as PR
+    M = M_()
+    gp, op = _params(3, (96, 64, 40), (8, 4))
+    proto = PR.Protocol(KEY, gp, variant=M.GEMM_AUTO)
+    m, n, l = 70, 128, 40
+    ch = PR.Chains(proto, PR.pad_width(n))
+    layer = PR.SecureLinear(proto, dev(wl.weights(m, n, std=1.0)), 9, ch)
+    mp = layer.init_x(l, 3)
+    Xp, s_x, Xpl = layer.mask_input(dev(wl.activations(l, n)), mp)
+    Z = layer.server(Xp, Xpl)
+    rng = np.random.default_rng(5)
+    base = layer.S_idx.clone()
+    levels = ((96, 8), (64, 4))
+    hits = [torch.from_numpy(rng.random(m * ti) < 0.2).cuda() for _, ti in levels]
+    outs = []
+    for fill in ("huge", "last"):
+        idx = base.clone()
+        off = 0
+        for (ri, ti), hit in zip(levels, hits):
+            blk = idx[off:off + m * ti]
+            blk[hit] = -1 if fill == "huge" else ri - 1
+            off += m * ti
+        layer.S_idx = idx
+        Yhat = torch.empty(l, m, dtype=torch.int32, device="cuda")
+        layer.unmask(Z, mp, s_x, Yhat=Yhat)
+        M.mosaic_device_status()
+        outs.append(host_u32(Yhat))
+    layer.S_idx = base
+    assert np.array_equal(outs[0], outs[1])
+
+
 def test_layer_zero_noise_and_no_bias():
     g, ref, op, m, l = _run_layer(3, (96, 64, 40), (6, 5), m=33, n=64, l=9, sigma=0.0, bias=False)
     _check_layer(g, ref, op, m, l)
