@@ -67,6 +67,12 @@ typedef struct {
     float sigma;
     uint32_t qbits;
     uint32_t rounds;
+    /* 1: the activation mask nests like the weight mask (Sec. 3.2 box, Init X
+     * 1b-1c: U_x = C_d R + sum_i C_i T_{i+1} + E_x, K = J_d R + sum_i J_i T_{i+1}).
+     * 0: the paper's deployed variant (Sec. 5.2, "Protocol parameterization"):
+     * the recursive LPN part of the activation mask is omitted, U_x = C_1 R + E_x
+     * and K = J_1 R with R uniform r_1 x l; only J_1 is kept at Init W. */
+    uint32_t act_nested;
 } mosaic_params;
 
 /* 256-bit PRG key (8 little-endian words). */
@@ -75,7 +81,7 @@ typedef struct {
 } mosaic_key;
 
 /* Fills `p` with the Example 3.1 parameters (d = 3, r = 1536/1024/652,
- * t = 80/80, sigma = 0.5, b = 16, 20 rounds, kappa = 32). */
+ * t = 80/80, sigma = 0.5, b = 16, 20 rounds, kappa = 32, act_nested = 1). */
 void mosaic_default_params(mosaic_params *p);
 
 /* Number of kernels this library has launched in this process (all devices,
@@ -113,7 +119,8 @@ enum {
     MOSAIC_TAG_R = 6,     /* per-pass R         (stream_id: pass id)                            */
     MOSAIC_TAG_T = 7,     /* per-pass sparse T_i                                                */
     MOSAIC_TAG_EX = 8,    /* activation noise E_x                                               */
-    MOSAIC_TAG_SIGN = 9   /* rotation signs d   (stream_id: matrix id)                          */
+    MOSAIC_TAG_SIGN = 9,  /* rotation signs d   (stream_id: matrix id)                          */
+    MOSAIC_TAG_CHECK = 10 /* Freivalds check vectors a (stream_id: matrix id)                   */
 };
 
 /* out[i * ldo + j] = stream word i * cols + j: uniform elements of Z_{2^32}.
@@ -248,6 +255,8 @@ mosaic_status mosaic_mask_chains(const mosaic_params *p, const mosaic_key *key,
  *   Wp ((m + Sr) x n_pad)   rows [0, m):   W' = W_hat + L P_d + sum S_{i+1} P_i + E_w
  *                           rows [m, m+Sr): a copy of P (server-side operand)
  *   J (m x Sr)              columns [J_1 | ... | J_d], J_i = (W_hat + E_w) C_i
+ *                           (act_nested = 0: only J_1, columns [0, r_1), is
+ *                           written; the others are left untouched)
  * Wp_planes (nullable): bf16 digit planes of Wp ([4][m + Sr][n_pad]).
  * ws: mosaic_workspace_bytes(MOSAIC_OP_MASK_WEIGHT, m, n_pad, 0, p). */
 mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key,
@@ -262,7 +271,8 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key,
  * E_x^T (l x n_pad, stream (EX, pass_id)) and writes
  *   Ux_tm (l x n_pad) = (C_d R + sum_i C_i T_{i+1} + E_x)^T
  *   K_tm  (l x m)     = (J_d R + sum_i J_i T_{i+1})^T
- * from C (n_pad x Sr) and J (m x Sr).
+ * from C (n_pad x Sr) and J (m x Sr).  With act_nested = 0: R^T is l x r_1
+ * (same stream), no T is drawn, Ux_tm = (C_1 R + E_x)^T, K_tm = (J_1 R)^T.
  * ws: mosaic_workspace_bytes(MOSAIC_OP_MASK_ACTIVATION, m, n_pad, l, p). */
 mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *key,
                                      uint64_t pass_id, int64_t m, int64_t n_pad, int64_t l,
@@ -320,13 +330,47 @@ mosaic_status mosaic_unmask_noalloc(const mosaic_params *p, int64_t l, int64_t m
                                     const float *bias, float *Y, uint32_t *Yhat, int64_t ldy,
                                     int variant, void *stream);
 
+/* ------------------------------------------------------------------------ */
+/* Integrity check (Sec. 3.2 box, Init W step 4 and Online step 4; appendix  */
+/* "Computational integrity": Freivalds' check).                             */
+/* ------------------------------------------------------------------------ */
+/* The box draws a with n entries and checks Y^chk X = a^T Y'; the shapes only
+ * agree with a in Z_{2^32}^m and the masked input, so this library checks
+ *     a^T Y' == (a^T W') X'   over Z_{2^32}
+ * token by token, with k independent vectors a (an error e in Y' escapes one
+ * vector with probability 2^-(32 - v), v = the number of trailing zero bits
+ * of e, so k vectors bound it by 2^-k for the worst case e = 2^31).
+ *
+ * Setup (one-time per weight matrix): draws the k x m matrix a (row v = check
+ * vector v) from stream (CHECK, matrix_id) and writes Ychk = a W' (k x n_pad)
+ * from the masked weights W' (m x n_pad, leading dimension ldw; rows [0, m) of
+ * the Wp operand of mosaic_mask_weight).  1 <= k <= 16.  Device buffers. */
+mosaic_status mosaic_freivalds_setup(const mosaic_params *p, const mosaic_key *key,
+                                     uint64_t matrix_id, int k, const uint32_t *Wm, int64_t ldw,
+                                     int64_t m, int64_t n_pad, uint32_t *a, uint32_t *Ychk,
+                                     void *stream);
+
+/* Online check of one server answer: for every token j < l,
+ *     lhs_v = sum_{i<m} a[v][i] Z[j][i]          (Y' = the first m columns of Z)
+ *     rhs_v = sum_{c<n_pad} Ychk[v][c] Xp[j][c]  (X', leading dimension ldx)
+ * bad[j] = number of vectors v with lhs_v != rhs_v, and *n_bad is increased by
+ * the number of tokens with bad[j] != 0 (the caller zeroes it; read it after
+ * the stream has been synchronised; a nonzero count means: abort).
+ * ws: 2 k l words (mosaic_workspace_bytes(MOSAIC_OP_FREIVALDS_CHECK, k, 0, l, NULL)).
+ * All pointers are device pointers; the products stream Z and X' once. */
+mosaic_status mosaic_freivalds_check(int k, const uint32_t *a, const uint32_t *Ychk, int64_t m,
+                                     int64_t n_pad, int64_t l, const uint32_t *Z, int64_t ldz,
+                                     const uint32_t *Xp, int64_t ldx, uint32_t *bad,
+                                     uint32_t *n_bad, void *ws, size_t ws_bytes, void *stream);
+
 /* Workspace sizes. */
 typedef enum {
     MOSAIC_OP_RING_GEMM = 1,        /* M = rows of A, n_pad = rows of B (N), l = K */
     MOSAIC_OP_MASK_CHAINS = 2,
     MOSAIC_OP_MASK_WEIGHT = 3,
     MOSAIC_OP_MASK_ACTIVATION = 4,
-    MOSAIC_OP_UNMASK = 5
+    MOSAIC_OP_UNMASK = 5,
+    MOSAIC_OP_FREIVALDS_CHECK = 6   /* m = k vectors, l = tokens */
 } mosaic_op;
 
 /* Bytes of `ws` the op needs for the given sizes and variant-independent

@@ -20,6 +20,7 @@ order of the protocol boxes:
 * ``server``      -- Approx-MatMul Online step 3 (Y' = W'X', Q_i = P_i X')
 * ``unmask``      -- Approx-MatMul Online step 5
 * ``decode``      -- Pi_Sec-Linear Online step 3 (fp64)
+* ``freivalds_*`` -- Approx-MatMul Init W step 4 and Online step 4 (integrity check)
 
 Parity status: every function is pinned by ``tests/test_oracle_pins.py``
 except the PRG stream layout and the sampler details (which words feed which
@@ -46,7 +47,7 @@ _LIB_PATH = os.path.join(_BUILD, "libmosaic_oracle.so")
 # ---------------------------------------------------------------------------
 # Stream tags (this build's PRG layout: kind in the low byte, level i above it)
 # ---------------------------------------------------------------------------
-KIND_M, KIND_N, KIND_L, KIND_S, KIND_EW, KIND_R, KIND_T, KIND_EX, KIND_SIGN = range(1, 10)
+KIND_M, KIND_N, KIND_L, KIND_S, KIND_EW, KIND_R, KIND_T, KIND_EX, KIND_SIGN, KIND_CHECK = range(1, 11)
 
 
 def tag(kind: int, level: int = 0) -> int:
@@ -62,6 +63,7 @@ class Params:
     sigma: float = 0.5
     qbits: int = 16
     rounds: int = 20
+    act_nested: bool = True          # False: the paper's deployed LWE-only activation mask
 
     def ranks(self, n_pad: int) -> list:
         """[r_0 = n_pad, r_1, ..., r_d]"""
@@ -365,7 +367,9 @@ def init_w(key, p: Params, W: np.ndarray, matrix_id: int, P, C, n_pad: int) -> W
     U_w = U_w + E_w
     W_masked = W_hat + U_w
     WE = W_hat + E_w
-    J = [matmul(WE, C[i - 1]) for i in range(1, p.d + 1)]
+    # J_i = (W_hat + E_w) N_1 ... N_i (Init W step 3); without the nested
+    # activation mask only J_1 is needed (Sec. 5.2, "Protocol parameterization").
+    J = [matmul(WE, C[i - 1]) for i in range(1, (p.d if p.act_nested else 1) + 1)]
     return WeightState(W_masked, W_hat, s_w, d_words, L, S, E_w, J, n, n_pad, qmax)
 
 
@@ -382,8 +386,19 @@ class PassState:
 def init_x(key, p: Params, l: int, pass_id: int, C, J, n_pad: int) -> PassState:
     """Init X (Sec. 3.2 box, steps 1a-1c).  Layout: R^T is sampled as an
     l x r_d uniform matrix, column k of T_{i+1} is sparse row k, and E_x^T is
-    sampled as an l x n_pad Gaussian matrix."""
+    sampled as an l x n_pad Gaussian matrix.
+
+    Without the nested activation mask (Sec. 5.2, "Protocol
+    parameterization": the recursive LPN part is omitted for activations),
+    R is r_1 x l from the same stream, U_x = N_1 R + E_x and K = J_1 R."""
     r = p.ranks(n_pad)
+    if not p.act_nested:
+        R = sample_uniform(key, tag(KIND_R), pass_id, l, r[1], p.rounds).T.copy()
+        E_x = sample_gaussian(key, tag(KIND_EX), pass_id, l * n_pad, p.sigma,
+                              p.rounds).reshape(l, n_pad).T.copy()
+        U_x = matmul(C[0], R) + E_x
+        K = matmul(J[0], R)
+        return PassState(U_x, K, R, {}, E_x)
     R = sample_uniform(key, tag(KIND_R), pass_id, l, r[p.d], p.rounds).T.copy()
     T = {}
     for i in range(1, p.d):
@@ -423,6 +438,22 @@ def unmask(p: Params, ws: WeightState, ps: PassState, Y_masked: np.ndarray, Q) -
     for i in range(1, p.d):
         Y = Y - sparse_rows_matmul(ws.S[i + 1], Q[i - 1])
     return Y
+
+
+def freivalds_setup(key, p: Params, ws: WeightState, matrix_id: int, k: int):
+    """Init W step 4 with the check vectors in Z_{2^32}^m (rows of a, k x m,
+    from stream (CHECK, matrix_id)): returns (a, Y_chk = a W')."""
+    m = ws.W_masked.shape[0]
+    a = sample_uniform(key, tag(KIND_CHECK), matrix_id, k, m, p.rounds)
+    return a, matmul(a, ws.W_masked)
+
+
+def freivalds_check(a: np.ndarray, Y_chk: np.ndarray, Y_masked: np.ndarray, X_masked: np.ndarray):
+    """Online step 4 (appendix "Computational integrity"), per column j of Y':
+    the number of check vectors v with a_v^T Y'_j != Y_chk,v X'_j (mod 2^32)."""
+    lhs = matmul(a, Y_masked)
+    rhs = matmul(Y_chk, X_masked)
+    return np.sum(lhs != rhs, axis=0).astype(np.uint32)
 
 
 def decode(Y_hat: np.ndarray, s_w: np.ndarray, s_x: np.ndarray, b=None) -> np.ndarray:

@@ -50,8 +50,14 @@ mosaic_status check_params(const mosaic_params *p) {
     if (!(p->sigma >= 0.0f && p->sigma <= 8.0f)) return MOSAIC_ERR_ARG;
     if (p->qbits < 2 || p->qbits > 16) return MOSAIC_ERR_ARG;
     if (!rounds_ok(p->rounds)) return MOSAIC_ERR_ARG;
+    if (p->act_nested > 1) return MOSAIC_ERR_ARG;
     return MOSAIC_OK;
 }
+
+// Rank of the dense activation-mask factor R: r_d (nested) or r_1 (act_nested = 0).
+int64_t r_act(const mosaic_params *p) { return p->act_nested ? p->r[p->d - 1] : p->r[0]; }
+// Number of LPN levels in the activation mask.
+uint32_t act_levels(const mosaic_params *p) { return p->act_nested ? p->d - 1 : 0; }
 
 int64_t sum_r(const mosaic_params *p) {
     int64_t s = 0;
@@ -122,13 +128,12 @@ size_t ws_weight(int64_t m, int64_t n_pad, const mosaic_params *p) {
     return ws_weight_min(m, n_pad, p) + ws_gemm(m, sum_r(p), n_pad);
 }
 size_t ws_activation_min(int64_t l, const mosaic_params *p) {
-    size_t s = up(sizeof(uint32_t) * (size_t)(l * p->r[p->d - 1]));
-    for (uint32_t i = 2; i <= p->d; i++) s += 2 * up(sizeof(uint32_t) * (size_t)(l * p->t[i - 1]));
+    size_t s = up(sizeof(uint32_t) * (size_t)(l * r_act(p)));
+    for (uint32_t i = 2; i <= act_levels(p) + 1; i++) s += 2 * up(sizeof(uint32_t) * (size_t)(l * p->t[i - 1]));
     return s;
 }
 size_t ws_activation(int64_t m, int64_t n_pad, int64_t l, const mosaic_params *p) {
-    const int64_t rd = p->r[p->d - 1];
-    const size_t g = ws_gemm(l, n_pad > m ? n_pad : m, rd);
+    const size_t g = ws_gemm(l, n_pad > m ? n_pad : m, r_act(p));
     return ws_activation_min(l, p) + g;
 }
 size_t ws_unmask_min(int64_t m, int64_t l, const mosaic_params *) {
@@ -154,6 +159,7 @@ void mosaic_default_params(mosaic_params *p) {
     p->sigma = 0.5f;
     p->qbits = 16;
     p->rounds = 20;
+    p->act_nested = 1;
 }
 
 const char *mosaic_status_string(mosaic_status s) {
@@ -340,6 +346,7 @@ size_t mosaic_workspace_bytes(int op, int64_t m, int64_t n_pad, int64_t l, const
         case MOSAIC_OP_MASK_ACTIVATION:
             return check_params(p) == MOSAIC_OK ? ws_activation(m, n_pad, l, p) : 0;
         case MOSAIC_OP_UNMASK: return check_params(p) == MOSAIC_OK ? ws_unmask(m, l, p) : 0;
+        case MOSAIC_OP_FREIVALDS_CHECK: return 2 * up(sizeof(uint32_t) * (size_t)(m * l));
     }
     return 0;
 }
@@ -410,8 +417,10 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, 
     // E_w and W_hat + E_w.
     MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EW, 0), matrix_id, R, p->sigma, m * n_pad, WE, st));
     MOSAIC_TRY(add_u32(Wp, n_pad, WE, n_pad, WE, n_pad, m, n_pad, st));
-    // J_i = (W_hat + E_w) C_i for all i at once: J = WE CT^T (m x Sr).
-    MOSAIC_TRY(gemm_u32(variant, cv, WE, n_pad, 1, CT, n_pad, 1, J, Sr, nullptr, 0, 1, m, Sr, n_pad, st));
+    // J_i = (W_hat + E_w) C_i for all i at once: J = WE CT^T (m x Sr); with
+    // act_nested = 0 only J_1 (the first r_1 columns) is used and computed.
+    const int64_t nJ = p->act_nested ? Sr : (int64_t)p->r[0];
+    MOSAIC_TRY(gemm_u32(variant, cv, WE, n_pad, 1, CT, n_pad, 1, J, Sr, nullptr, 0, 1, m, nJ, n_pad, st));
     // L, S_{i+1}.
     MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_L, 0), matrix_id, R, m, rd, L, rd, st));
     SparseLevel lev[2];
@@ -451,8 +460,10 @@ mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *k
     cudaStream_t st = as_stream(stream);
     const Key k = to_key(key);
     const int R = (int)p->rounds;
-    const uint32_t d = p->d;
-    const int64_t Sr = sum_r(p), rd = p->r[d - 1], od = off_r(p, d);
+    // Nested (Init X 1b-1c): dense factor R at rank r_d against C_d, J_d plus
+    // d - 1 LPN levels.  act_nested = 0: R at rank r_1 against C_1, J_1 only.
+    const uint32_t d = act_levels(p) + 1;
+    const int64_t Sr = sum_r(p), rd = r_act(p), od = p->act_nested ? off_r(p, p->d) : 0;
     Carve cv{static_cast<char *>(ws), ws_bytes, 0};
     uint32_t *Rt = cv.take<uint32_t>((size_t)(l * rd));
     if (!Rt) return MOSAIC_ERR_WORKSPACE;
@@ -510,6 +521,34 @@ mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const 
     // Y_hat = Y' - tmp - sum_i S_{i+1} Q_i, then decode.
     return unmask_decode(Z, ldz, m, od, l, m, lev, (int)d - 1, tmp, m, s_w, s_x, bias, Y, Yhat, ldy,
                          st);
+}
+
+mosaic_status mosaic_freivalds_setup(const mosaic_params *p, const mosaic_key *key, uint64_t matrix_id,
+                                     int k, const uint32_t *Wm, int64_t ldw, int64_t m, int64_t n_pad,
+                                     uint32_t *a, uint32_t *Ychk, void *stream) {
+    MOSAIC_TRY(check_params(p));
+    if (!key) return MOSAIC_ERR_ARG;
+    if (k < 1 || k > 16) return MOSAIC_ERR_ARG;
+    if (!npad_ok(n_pad) || m < 1 || ldw < n_pad) return MOSAIC_ERR_SHAPE;
+    if (!Wm || !a || !Ychk) return MOSAIC_ERR_ARG;
+    cudaStream_t st = as_stream(stream);
+    MOSAIC_TRY(prg_uniform(to_key(key), tag_of(MOSAIC_TAG_CHECK, 0), matrix_id, (int)p->rounds, k, m, a, m, st));
+    return freivalds_colsum(a, k, Wm, ldw, m, n_pad, Ychk, st);
+}
+
+mosaic_status mosaic_freivalds_check(int k, const uint32_t *a, const uint32_t *Ychk, int64_t m,
+                                     int64_t n_pad, int64_t l, const uint32_t *Z, int64_t ldz,
+                                     const uint32_t *Xp, int64_t ldx, uint32_t *bad, uint32_t *n_bad,
+                                     void *ws, size_t ws_bytes, void *stream) {
+    if (k < 1 || k > 16) return MOSAIC_ERR_ARG;
+    if (m < 1 || n_pad < 1 || l < 0 || ldz < m || ldx < n_pad) return MOSAIC_ERR_SHAPE;
+    if (l == 0) return MOSAIC_OK;
+    if (!a || !Ychk || !Z || !Xp || !bad || !n_bad) return MOSAIC_ERR_ARG;
+    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    uint32_t *lhs = cv.take<uint32_t>((size_t)(k * l));
+    uint32_t *rhs = cv.take<uint32_t>((size_t)(k * l));
+    if (!lhs || !rhs) return MOSAIC_ERR_WORKSPACE;
+    return freivalds_check(k, a, Ychk, m, n_pad, l, Z, ldz, Xp, ldx, bad, n_bad, lhs, rhs, as_stream(stream));
 }
 
 }  // extern "C"

@@ -131,6 +131,14 @@ mosaic_status ring_gemm_skinny(const uint32_t *A, int64_t lda, const uint32_t *B
 // Reads and clears the streaming kernel's timeout word (after a stream sync).
 mosaic_status skinny_status();
 
+// Freivalds check: Y (k x ncols) = a (k x m) W (m x ncols, ldw), and the
+// per-token comparison a^T Y' vs Ychk X' (lhs, rhs: k x l scratch each).
+mosaic_status freivalds_colsum(const uint32_t *a, int k, const uint32_t *W, int64_t ldw, int64_t m,
+                               int64_t ncols, uint32_t *Y, cudaStream_t st);
+mosaic_status freivalds_check(int k, const uint32_t *a, const uint32_t *Ychk, int64_t m, int64_t n_pad,
+                              int64_t l, const uint32_t *Z, int64_t ldz, const uint32_t *Xp, int64_t ldx,
+                              uint32_t *bad, uint32_t *n_bad, uint32_t *lhs, uint32_t *rhs, cudaStream_t st);
+
 // Sparse gathers.
 // out[row][col] = a[row][col] - b[row][col] (b nullable) + sgn * sum_lev sum_q val * src[g][off_lev + idx]
 // where (list entity, staged row g) = (row, col) if !list_is_col else (col, row).

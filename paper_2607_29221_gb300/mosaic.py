@@ -23,7 +23,8 @@ STATUS = {0: "ok", 1: "invalid argument", 2: "invalid shape", 3: "misaligned", 4
 GEMM_AUTO, GEMM_TC, GEMM_MMA_S8, GEMM_IMAD = 0, 1, 2, 3
 SKINNY_MAX_M = 16   # MOSAIC_SKINNY_MAX_M: token counts the streaming product serves
 OP_RING_GEMM, OP_MASK_CHAINS, OP_MASK_WEIGHT, OP_MASK_ACTIVATION, OP_UNMASK = 1, 2, 3, 4, 5
-TAG_M, TAG_N, TAG_L, TAG_S, TAG_EW, TAG_R, TAG_T, TAG_EX, TAG_SIGN = range(1, 10)
+OP_FREIVALDS_CHECK = 6
+TAG_M, TAG_N, TAG_L, TAG_S, TAG_EW, TAG_R, TAG_T, TAG_EX, TAG_SIGN, TAG_CHECK = range(1, 11)
 
 
 class MosaicError(RuntimeError):
@@ -35,7 +36,7 @@ class MosaicError(RuntimeError):
 class mosaic_params(ctypes.Structure):
     _fields_ = [("kappa", ctypes.c_uint32), ("d", ctypes.c_uint32), ("r", ctypes.c_uint32 * 3),
                 ("t", ctypes.c_uint32 * 3), ("sigma", ctypes.c_float), ("qbits", ctypes.c_uint32),
-                ("rounds", ctypes.c_uint32)]
+                ("rounds", ctypes.c_uint32), ("act_nested", ctypes.c_uint32)]
 
 
 class mosaic_key(ctypes.Structure):
@@ -77,6 +78,9 @@ _SIGS = {
     "mosaic_device_status": ([_P], _INT),
     "mosaic_unmask_noalloc": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
                                _INT, _P], _INT),
+    "mosaic_freivalds_setup": ([_PP, _PK, _U64, _INT, _P, _I64, _I64, _I64, _P, _P, _P], _INT),
+    "mosaic_freivalds_check": ([_INT, _P, _P, _I64, _I64, _I64, _P, _I64, _P, _I64, _P, _P, _P, _SZ,
+                                _P], _INT),
 }
 
 EXPORTS = tuple(_SIGS)
@@ -256,3 +260,14 @@ def mosaic_unmask_noalloc(params, l, m, Z, ldz, K_tm, L, S_idx, S_val, s_w, s_x,
     _call("mosaic_unmask_noalloc", ctypes.byref(params), l, m, _ptr(Z), ldz, _ptr(K_tm), _ptr(L),
           _ptr(S_idx), _ptr(S_val), _ptr(s_w), _ptr(s_x), _ptr(bias), _ptr(Y), _ptr(Yhat), ldy,
           variant, _stream(stream))
+
+
+def mosaic_freivalds_setup(params, key, matrix_id, k, Wm, ldw, m, n_pad, a, Ychk, stream=None):
+    _call("mosaic_freivalds_setup", ctypes.byref(params), ctypes.byref(key), matrix_id, k, _ptr(Wm), ldw,
+          m, n_pad, _ptr(a), _ptr(Ychk), _stream(stream))
+
+
+def mosaic_freivalds_check(k, a, Ychk, m, n_pad, l, Z, ldz, Xp, ldx, bad, n_bad, ws, stream=None):
+    _call("mosaic_freivalds_check", k, _ptr(a), _ptr(Ychk), m, n_pad, l, _ptr(Z), ldz, _ptr(Xp), ldx,
+          _ptr(bad), _ptr(n_bad), _ptr(ws), 0 if ws is None else ws.numel() * ws.element_size(),
+          _stream(stream))

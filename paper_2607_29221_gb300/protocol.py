@@ -170,6 +170,30 @@ class SecureLinear:
                         self.s_w, s_x, self.bias, Y, Yhat, self.m, self.proto.variant, ws)
         return Y
 
+    # Integrity (Init W step 4, Online step 4) ---------------------------
+    def freivalds_setup(self, k: int = 4):
+        """Draws k check vectors a (k x m) and keeps Ychk = a W' (k x n_pad)."""
+        dev = self.proto.device
+        self.check_k = k
+        self.check_a = _u32(k, self.m, device=dev)
+        self.check_Y = _u32(k, self.n_pad, device=dev)
+        M.mosaic_freivalds_setup(self.proto.params, self.proto.key, self.matrix_id, k, self.Wp,
+                                 self.n_pad, self.m, self.n_pad, self.check_a, self.check_Y)
+
+    def freivalds_check(self, Z, Xp, bad=None, n_bad=None):
+        """Per-token check a^T Y' == Ychk X' on the device; returns (bad, n_bad)
+        device tensors (bad[j] = failing vectors of token j, n_bad = failing
+        tokens).  Read n_bad after a synchronise; nonzero means: abort."""
+        l = Z.shape[0]
+        dev = self.proto.device
+        bad = _u32(l, device=dev) if bad is None else bad
+        if n_bad is None:
+            n_bad = torch.zeros(1, dtype=torch.int32, device=dev)
+        ws = self.proto.workspace(M.mosaic_workspace_bytes(M.OP_FREIVALDS_CHECK, self.check_k, 0, l))
+        M.mosaic_freivalds_check(self.check_k, self.check_a, self.check_Y, self.m, self.n_pad, l, Z,
+                                 Z.stride(0), Xp, Xp.stride(0), bad, n_bad, ws)
+        return bad, n_bad
+
     def forward(self, X_tm: torch.Tensor, mp: PassMask, Yhat=None):
         Xp, s_x, Xplanes = self.mask_input(X_tm, mp)
         Z = self.server(Xp, Xplanes)

@@ -65,6 +65,18 @@ def spike_activations(l: int, n: int, seed: int = SEED_X, outlier: float = 100.0
     return a
 
 
+def outlier_weights(m: int, n: int, seed: int = SEED_W, std: float = 0.02, channels: int = 8,
+                    factor: float = 10.0) -> np.ndarray:
+    """N(0, std^2) weights whose few input channels (columns) are `factor`
+    times larger: the outlier-channel structure of trained LLM projections
+    that the rotation of Sec. 4 spreads out."""
+    w = weights(m, n, seed, std)
+    g = np.random.Generator(np.random.PCG64(seed + 2000))
+    ch = g.choice(n, size=channels, replace=False)
+    w[:, ch] *= np.float32(factor)
+    return w
+
+
 def uniform_u32(seed: int, rows: int, cols: int) -> np.ndarray:
     """Uniform ring elements for ring-only tests (not part of the protocol's PRG)."""
     g = np.random.Generator(np.random.PCG64(seed))
@@ -114,5 +126,22 @@ WORKLOADS = {
          Linear("gate_up", 57344, 8192), Linear("down", 8192, 28672)),
         decode_batches=(1, 8, 32, 128, 256),
         notes="decode sweep at 70B layer shape, pre-masked weights"),
+    "matvec_sweep": Workload(
+        "matvec_sweep", 1,
+        (Linear("n4096", 4096, 4096), Linear("n8192", 8192, 8192), Linear("n16384", 16384, 16384)),
+        notes="secure mat-vec n x n, one token (the paper's mat-vec figure; n = 36864 would "
+              "need a 65536-wide rotation, beyond this build's 32768)"),
+    "sigma_sweep_7b": Workload(
+        "sigma_sweep_7b", 128,
+        (Linear("attn", 4096, 4096), Linear("up", 14336, 4096), Linear("down", 4096, 14336)),
+        notes="single-layer relative l2 error vs sigma (the paper's single-layer error table), "
+              "N(0,0.02) weights with 8 outlier input channels (10x), N(0,1) activations with "
+              "4 outlier channels (20x)"),
+    "init_w_70b": Workload(
+        "init_w_70b", 0,
+        (Linear("qkv", 10240, 8192), Linear("o", 8192, 8192),
+         Linear("gate_up", 57344, 8192), Linear("down", 8192, 28672)),
+        notes="one-time Init W of a 70B layer's four matrices plus the public chains per "
+              "rotation width, extrapolated to 80 layers"),
 }
 

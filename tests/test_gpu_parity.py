@@ -192,18 +192,18 @@ def test_ring_gemm_imad(Mm, N, K):
 # --------------------------------------------------------------------------
 # Masks, server, unmask
 # --------------------------------------------------------------------------
-def _params(d, r, t, sigma=0.5):
+def _params(d, r, t, sigma=0.5, act_nested=True):
     M = M_()
     tt = [0] + list(t)
     return (M.default_params(d=d, r=list(r) + [0] * (3 - len(r)), t=tt + [0] * (3 - len(tt)),
-                             sigma=sigma),
-            O.Params(d=d, r=tuple(r), t=tuple(t), sigma=sigma))
+                             sigma=sigma, act_nested=int(act_nested)),
+            O.Params(d=d, r=tuple(r), t=tuple(t), sigma=sigma, act_nested=act_nested))
 
 
-def _run_layer(d, r, t, m, n, l, sigma=0.5, w_std=1.0, bias=True, variant=None):
+def _run_layer(d, r, t, m, n, l, sigma=0.5, w_std=1.0, bias=True, variant=None, act_nested=True):
     from paper_2607_29221_gb300 import protocol as PR
     M = M_()
-    gp, op = _params(d, r, t, sigma)
+    gp, op = _params(d, r, t, sigma, act_nested)
     variant = M.GEMM_IMAD if variant is None else variant
     proto = PR.Protocol(KEY, gp, variant=variant)
     n_pad = PR.pad_width(n)
@@ -244,7 +244,10 @@ def _check_layer(g, ref, op, m, l):
         off += m * t
     assert np.array_equal(g["Wp"][:m], ws.W_masked)
     assert np.array_equal(g["Wp"][m:], P)
-    assert np.array_equal(g["J"], np.hstack(ws.J))
+    if op.act_nested:
+        assert np.array_equal(g["J"], np.hstack(ws.J))
+    else:   # only J_1 is written
+        assert np.array_equal(g["J"][:, :op.r[0]], ws.J[0])
     assert np.array_equal(g["Ux"], ps.U_x.T)
     assert np.array_equal(g["K"], ps.K.T)
     assert np.array_equal(g["Xp"], ref["X_masked"].T)
@@ -342,6 +345,19 @@ def test_unmask_clamps_out_of_range_positions():
         outs.append(host_u32(Yhat))
     layer.S_idx = base
     assert np.array_equal(outs[0], outs[1])
+
+
+@pytest.mark.parametrize("d,r,t,l", [(3, (96, 64, 40), (6, 5), 21), (3, (96, 64, 40), (8, 4), 3),
+                                     (2, (100, 70), (9,), 67), (3, (1536, 1024, 652), (80, 80), 64)])
+def test_layer_lwe_only_activation_mask(d, r, t, l):
+    """act_nested = 0 (Sec. 5.2: the recursive LPN part of the activation mask
+    omitted, U_x = C_1 R + E_x, K = J_1 R at rank r_1): every ring output
+    bit-exact, on the tensor-core, streaming (l <= 16) and CUDA-core paths."""
+    for variant in _variants():
+        g, ref, op, m, l_ = _run_layer(d, r, t, m=131 if r[0] < 1000 else 128,
+                                       n=300 if r[0] < 1000 else 256, l=l, variant=variant,
+                                       act_nested=False)
+        _check_layer(g, ref, op, m, l_)
 
 
 def test_layer_zero_noise_and_no_bias():

@@ -5,6 +5,8 @@ brute-force ring arithmetic, and the algebraic identities of the protocol
 had-product-preserved, Thm 3.2, Table tab:lpn-tradeoff)."""
 import math
 
+import dataclasses
+
 import numpy as np
 import pytest
 
@@ -259,7 +261,7 @@ SMALL = O.Params(d=3, r=(96, 64, 40), t=(6, 5))
 
 def _run(p, m=24, n=48, l=10, sigma=None, x_zero=False, seed_off=0):
     if sigma is not None:
-        p = O.Params(d=p.d, r=p.r, t=p.t, sigma=sigma)
+        p = dataclasses.replace(p, sigma=sigma)
     W = wl.weights(m, n, seed=wl.SEED_W + seed_off, std=1.0)
     X = wl.activations(l, n, seed=wl.SEED_X + seed_off).T.copy()
     if x_zero:
@@ -267,19 +269,22 @@ def _run(p, m=24, n=48, l=10, sigma=None, x_zero=False, seed_off=0):
     return p, O.secure_linear(KEY, p, W, X, matrix_id=3 + seed_off, pass_id=17 + seed_off), W, X
 
 
+@pytest.mark.parametrize("act_nested", [True, False])
 @pytest.mark.parametrize("d", [1, 2, 3])
-def test_zero_noise_protocol_is_exact(d):
-    """sigma = 0: Y_hat = W_hat X_hat exactly (the INT16-rot-sigma=0 case, Sec. 4.3)."""
-    p = O.Params(d=d, r=SMALL.r, t=SMALL.t, sigma=0.0)
+def test_zero_noise_protocol_is_exact(d, act_nested):
+    """sigma = 0: Y_hat = W_hat X_hat exactly (the INT16-rot-sigma=0 case, Sec. 4.3),
+    with the nested activation mask and with the LWE-only one of Sec. 5.2."""
+    p = O.Params(d=d, r=SMALL.r[:d], t=SMALL.t[: d - 1], sigma=0.0, act_nested=act_nested)
     _, r, _, _ = _run(p)
     assert np.array_equal(r["Y_hat"], r["ws"].W_hat @ r["X_hat"])
 
 
+@pytest.mark.parametrize("act_nested", [True, False])
 @pytest.mark.parametrize("d", [1, 2, 3])
-def test_noise_identity(d):
+def test_noise_identity(d, act_nested):
     """Y_hat - W_hat X_hat = W_hat E_x + E_w X_hat + E_w E_x (mod 2^32), eq. approx-error
     and the Sec. 3.2 unmask derivation, with the E's re-read from the sampled state."""
-    p = O.Params(d=d, r=SMALL.r, t=SMALL.t, sigma=1.0)
+    p = O.Params(d=d, r=SMALL.r[:d], t=SMALL.t[: d - 1], sigma=1.0, act_nested=act_nested)
     _, r, _, _ = _run(p, seed_off=d)
     Wh, Xh, Ew, Ex = r["ws"].W_hat, r["X_hat"], r["ws"].E_w, r["ps"].E_x
     assert np.any(Ew) and np.any(Ex)
@@ -357,3 +362,59 @@ def test_oracle_layout_of_init_x():
     ps = O.init_x(KEY, p, 5, 2, C, ws.J, 64)
     assert np.array_equal(ps.R.T, O.sample_uniform(KEY, O.tag(O.KIND_R), 2, 5, 16))
     assert np.array_equal(ps.T[2][0], O.sample_sparse(KEY, O.tag(O.KIND_T, 2), 2, 5, 32, 3)[0])
+
+
+def test_lwe_only_activation_mask_structure():
+    """act_nested = False (Sec. 5.2, "Protocol parameterization"): only J_1 is
+    kept, no T is drawn and R has r_1 rows; the mask differs from the nested
+    one drawn from the same key (the identities above pin its arithmetic)."""
+    p = O.Params(d=3, r=(12, 8, 5), t=(3, 2), sigma=0.5, act_nested=False)
+    _, r, _, _ = _run(p, m=6, n=16, l=9)
+    ws, ps = r["ws"], r["ps"]
+    assert len(ws.J) == 1 and ps.T == {} and ps.R.shape == (12, 9)
+    _, rn, _, _ = _run(dataclasses.replace(p, act_nested=True), m=6, n=16, l=9)
+    assert len(rn["ws"].J) == 3 and rn["ps"].R.shape == (5, 9)
+    assert not np.array_equal(rn["ps"].U_x, ps.U_x)
+    assert np.array_equal(rn["ws"].J[0], ws.J[0])
+
+
+# --------------------------------------------------------------------------
+# Freivalds integrity check (Init W 4, Online 4; "Computational integrity")
+# --------------------------------------------------------------------------
+def test_freivalds_accepts_honest_and_flags_corruption():
+    """An honest Y' = W' X' passes for every vector (associativity of the ring
+    product); an odd error in one entry of column j is caught by every vector
+    with a_v[i] != 0 at that row (a_v[i] * e = 0 mod 2^32 needs a_v[i] = 0),
+    and an error 2^31 exactly by the vectors whose a_v[i] is odd."""
+    p = O.Params(d=3, r=SMALL.r, t=SMALL.t, sigma=0.5)
+    _, r, _, _ = _run(p, m=20, n=48, l=9)
+    ws = r["ws"]
+    a, Yc = O.freivalds_setup(KEY, p, ws, 3, 6)
+    assert a.shape == (6, 20) and Yc.shape == (6, 64)
+    assert np.array_equal(a, O.sample_uniform(KEY, O.tag(O.KIND_CHECK), 3, 6, 20))
+    Yp, Xp = r["Y_masked"], r["X_masked"]
+    assert not np.any(O.freivalds_check(a, Yc, Yp, Xp))
+    bad = Yp.copy()
+    bad[7, 4] = np.uint32((int(bad[7, 4]) + 12345) % 2**32)   # odd error at row 7, token 4
+    got = O.freivalds_check(a, Yc, bad, Xp)
+    assert got[4] == np.count_nonzero(a[:, 7]) and got[4] == 6
+    assert np.count_nonzero(got) == 1
+    bad = Yp.copy()
+    bad[2, 1] = np.uint32((int(bad[2, 1]) + 2**31) % 2**32)
+    got = O.freivalds_check(a, Yc, bad, Xp)
+    assert got[1] == int(np.sum(a[:, 2] & 1)) and np.count_nonzero(got) == (1 if got[1] else 0)
+
+
+def test_freivalds_check_vectors_on_a_bruteforce_case():
+    """Tiny case against Python integers: a^T (W' X') and (a^T W') X' mod 2^32."""
+    rng = np.random.default_rng(9)
+    W = rng.integers(0, 2**32, (3, 4), dtype=np.uint64).astype(np.uint32)
+    X = rng.integers(0, 2**32, (4, 2), dtype=np.uint64).astype(np.uint32)
+    a = rng.integers(0, 2**32, (2, 3), dtype=np.uint64).astype(np.uint32)
+    Y = O.matmul(W, X)
+    for v in range(2):
+        for j in range(2):
+            lhs = sum(int(a[v, i]) * sum(int(W[i, c]) * int(X[c, j]) for c in range(4)) for i in range(3))
+            assert (lhs % 2**32) == int(O.matmul(a, Y)[v, j])
+            rhs = sum(sum(int(a[v, i]) * int(W[i, c]) for i in range(3)) * int(X[c, j]) for c in range(4))
+            assert (rhs % 2**32) == int(O.matmul(O.matmul(a, W), X)[v, j])
