@@ -280,6 +280,27 @@ mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *k
                                      uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
                                      void *stream);
 
+/* Stationary operands of Init X as tensor-core digit planes, made once per
+ * weight matrix (after mosaic_mask_weight) so that no pass re-splits them:
+ * cj_planes = [4][n_pad + m][Kp] bf16 digits (Kp = r rounded up to a multiple
+ * of 8, r = r_d, or r_1 with act_nested = 0): rows [0, n_pad) the C-factor
+ * block (C_d, or C_1), rows [n_pad, n_pad + m) the J-factor block (J_d, or
+ * J_1).  Size: mosaic_workspace_bytes(MOSAIC_OP_ACTIVATION_PLANES, m, n_pad, 0, p).
+ * 16-byte aligned device buffer. */
+mosaic_status mosaic_prepare_activation(const mosaic_params *p, int64_t m, int64_t n_pad,
+                                        const uint32_t *C, const uint32_t *J, uint16_t *cj_planes,
+                                        void *stream);
+
+/* mosaic_mask_activation with the planes of mosaic_prepare_activation (same
+ * results; the two dense products R^T C^T and R^T J^T run as one tensor-core
+ * product against the cached planes when l > MOSAIC_SKINNY_MAX_M). */
+mosaic_status mosaic_mask_activation_planes(const mosaic_params *p, const mosaic_key *key,
+                                            uint64_t pass_id, int64_t m, int64_t n_pad, int64_t l,
+                                            const uint32_t *C, const uint32_t *J,
+                                            const uint16_t *cj_planes, uint32_t *Ux_tm,
+                                            uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
+                                            void *stream);
+
 /* ------------------------------------------------------------------------ */
 /* Unmask and decode (Approx-MatMul Online step 5; Pi_Sec-Linear Online      */
 /* step 3).                                                                  */
@@ -297,6 +318,20 @@ mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const 
                             const uint32_t *S_idx, const uint32_t *S_val, const float *s_w,
                             const float *s_x, const float *bias, float *Y, uint32_t *Yhat,
                             int64_t ldy, int variant, void *ws, size_t ws_bytes, void *stream);
+
+/* L (m x r_d) as tensor-core digit planes [4][m][Kp], Kp = r_d rounded up to a
+ * multiple of 8, made once per weight matrix.  Size:
+ * mosaic_workspace_bytes(MOSAIC_OP_UNMASK_PLANES, m, 0, 0, p); 16-byte aligned. */
+mosaic_status mosaic_prepare_unmask(const mosaic_params *p, int64_t m, const uint32_t *L,
+                                    uint16_t *L_planes, void *stream);
+
+/* mosaic_unmask with the planes of mosaic_prepare_unmask (same results). */
+mosaic_status mosaic_unmask_planes(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z,
+                                   int64_t ldz, const uint32_t *K_tm, const uint32_t *L,
+                                   const uint16_t *L_planes, const uint32_t *S_idx,
+                                   const uint32_t *S_val, const float *s_w, const float *s_x,
+                                   const float *bias, float *Y, uint32_t *Yhat, int64_t ldy,
+                                   int variant, void *ws, size_t ws_bytes, void *stream);
 
 /* Synchronises `stream` and reports device-side failures of earlier calls:
  * MOSAIC_ERR_TIMEOUT if a tensor-core product gave up a bounded wait (the
@@ -370,7 +405,9 @@ typedef enum {
     MOSAIC_OP_MASK_WEIGHT = 3,
     MOSAIC_OP_MASK_ACTIVATION = 4,
     MOSAIC_OP_UNMASK = 5,
-    MOSAIC_OP_FREIVALDS_CHECK = 6   /* m = k vectors, l = tokens */
+    MOSAIC_OP_FREIVALDS_CHECK = 6,  /* m = k vectors, l = tokens */
+    MOSAIC_OP_ACTIVATION_PLANES = 7,/* bytes of cj_planes for (m, n_pad)   */
+    MOSAIC_OP_UNMASK_PLANES = 8     /* bytes of L_planes for m              */
 } mosaic_op;
 
 /* Bytes of `ws` the op needs for the given sizes and variant-independent

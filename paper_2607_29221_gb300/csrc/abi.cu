@@ -132,9 +132,17 @@ size_t ws_activation_min(int64_t l, const mosaic_params *p) {
     for (uint32_t i = 2; i <= act_levels(p) + 1; i++) s += 2 * up(sizeof(uint32_t) * (size_t)(l * p->t[i - 1]));
     return s;
 }
+int64_t kpad8(int64_t k) { return (k + 7) / 8 * 8; }
 size_t ws_activation(int64_t m, int64_t n_pad, int64_t l, const mosaic_params *p) {
-    const size_t g = ws_gemm(l, n_pad > m ? n_pad : m, r_act(p));
+    // Room for the combined tensor-core product: planes of R^T and of [C; J].
+    const size_t g = ws_gemm(l, n_pad + m, r_act(p));
     return ws_activation_min(l, p) + g;
+}
+size_t activation_planes_bytes(int64_t m, int64_t n_pad, const mosaic_params *p) {
+    return 8 * (size_t)((n_pad + m) * kpad8(r_act(p)));
+}
+size_t unmask_planes_bytes(int64_t m, const mosaic_params *p) {
+    return 8 * (size_t)(m * kpad8(p->r[p->d - 1]));
 }
 size_t ws_unmask_min(int64_t m, int64_t l, const mosaic_params *) {
     return up(sizeof(uint32_t) * (size_t)(l * m));
@@ -347,6 +355,9 @@ size_t mosaic_workspace_bytes(int op, int64_t m, int64_t n_pad, int64_t l, const
             return check_params(p) == MOSAIC_OK ? ws_activation(m, n_pad, l, p) : 0;
         case MOSAIC_OP_UNMASK: return check_params(p) == MOSAIC_OK ? ws_unmask(m, l, p) : 0;
         case MOSAIC_OP_FREIVALDS_CHECK: return 2 * up(sizeof(uint32_t) * (size_t)(m * l));
+        case MOSAIC_OP_ACTIVATION_PLANES:
+            return check_params(p) == MOSAIC_OK ? activation_planes_bytes(m, n_pad, p) : 0;
+        case MOSAIC_OP_UNMASK_PLANES: return check_params(p) == MOSAIC_OK ? unmask_planes_bytes(m, p) : 0;
     }
     return 0;
 }
@@ -446,11 +457,17 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, 
     return MOSAIC_OK;
 }
 
-mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *key,
-                                     uint64_t pass_id, int64_t m, int64_t n_pad, int64_t l,
-                                     const uint32_t *C, const uint32_t *J, uint32_t *Ux_tm,
-                                     uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
-                                     void *stream) {
+}  // extern "C"
+
+namespace {
+
+// Init X; `cj` (nullable) holds the digit planes of [C-factor; J-factor] made
+// by mosaic_prepare_activation.
+mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key, uint64_t pass_id,
+                                   int64_t m, int64_t n_pad, int64_t l, const uint32_t *C,
+                                   const uint32_t *J, const uint16_t *cj, uint32_t *Ux_tm,
+                                   uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
+                                   void *stream) {
     MOSAIC_TRY(check_params(p));
     if (!key) return MOSAIC_ERR_ARG;
     if (!npad_ok(n_pad) || m < 1 || l < 0 || l >= ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
@@ -477,26 +494,93 @@ mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *k
         MOSAIC_TRY(prg_sparse(k, tag_of(MOSAIC_TAG_T, i + 1), pass_id, R, l, ri, t, ti, tv, nullptr, st));
         lev[i - 1] = SparseLevel{ti, tv, (int)t, off_r(p, i), ri};
     }
-    // U_x^T = E_x^T + R^T C_d^T + sum_i T_{i+1}^T C_i^T.
+    // U_x^T = E_x^T + R^T C_d^T + sum_i T_{i+1}^T C_i^T and
+    // K^T = R^T J_d^T + sum_i T_{i+1}^T J_i^T: the two dense products share
+    // R^T, so on the tensor cores they run as one product against the stacked
+    // [C_d; J_d] (planes cached by mosaic_prepare_activation, or split here).
     MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EX, 0), pass_id, R, p->sigma, l * n_pad, Ux_tm, st));
-    MOSAIC_TRY(gemm_u32(variant, cv, Rt, rd, 1, C + od, Sr, 1, Ux_tm, n_pad, Ux_tm, n_pad, 1, l, n_pad,
-                        rd, st));
+    const bool want_tc = variant == MOSAIC_GEMM_TC || (variant == MOSAIC_GEMM_AUTO && tc_available());
+    const int64_t Kp = kpad8(rd), bplane = (n_pad + m) * Kp;
+    const size_t need = up(8 * (size_t)(l * Kp)) + (cj ? 0 : up(8 * (size_t)bplane));
+    const bool skinny = skinny_ok(Rt, rd, C + od, Sr, l, rd) && skinny_ok(Rt, rd, J + od, Sr, l, rd);
+    const bool fused = want_tc && !skinny && n_pad % 128 == 0 && Sr % 4 == 0 && aligned16(C + od) &&
+                       aligned16(J + od) && cv.used + need <= cv.cap;
+    if (fused) {
+        const size_t mark = cv.used;
+        uint16_t *Rp = cv.take<uint16_t>((size_t)(4 * l * Kp));
+        MOSAIC_TRY(digit_split(Rt, rd, l, rd, Rp, Kp, l * Kp, st));
+        const uint16_t *B = cj;
+        if (!B) {
+            uint16_t *Bw = cv.take<uint16_t>((size_t)(4 * bplane));
+            MOSAIC_TRY(digit_split(C + od, Sr, n_pad, rd, Bw, Kp, bplane, st));
+            MOSAIC_TRY(digit_split(J + od, Sr, m, rd, Bw + n_pad * Kp, Kp, bplane, st));
+            B = Bw;
+        }
+        MOSAIC_TRY(ring_gemm_tc_planes2(Rp, Kp, l * Kp, B, Kp, bplane, Ux_tm, n_pad, Ux_tm, n_pad, n_pad,
+                                        K_tm, m, nullptr, 0, m, l, rd, st));
+        cv.used = mark;
+    } else {
+        MOSAIC_TRY(gemm_u32(variant, cv, Rt, rd, 1, C + od, Sr, 1, Ux_tm, n_pad, Ux_tm, n_pad, 1, l,
+                            n_pad, rd, st));
+        MOSAIC_TRY(gemm_u32(variant, cv, Rt, rd, 1, J + od, Sr, 1, K_tm, m, nullptr, 0, 1, l, m, rd, st));
+    }
     if (d > 1)
         MOSAIC_TRY(sparse_gather(C, Sr, 0, od, n_pad, l, false, lev, (int)d - 1, Ux_tm, n_pad,
                                  nullptr, 0, 1, Ux_tm, n_pad, st));
-    // K^T = R^T J_d^T + sum_i T_{i+1}^T J_i^T.
-    MOSAIC_TRY(gemm_u32(variant, cv, Rt, rd, 1, J + od, Sr, 1, K_tm, m, nullptr, 0, 1, l, m, rd, st));
     if (d > 1)
         MOSAIC_TRY(sparse_gather(J, Sr, 0, od, m, l, false, lev, (int)d - 1, K_tm, m, nullptr, 0, 1,
                                  K_tm, m, st));
     return MOSAIC_OK;
 }
 
-mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z,
-                            int64_t ldz, const uint32_t *K_tm, const uint32_t *L,
-                            const uint32_t *S_idx, const uint32_t *S_val, const float *s_w,
-                            const float *s_x, const float *bias, float *Y, uint32_t *Yhat,
-                            int64_t ldy, int variant, void *ws, size_t ws_bytes, void *stream) {
+}  // namespace
+
+extern "C" {
+
+mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *key,
+                                     uint64_t pass_id, int64_t m, int64_t n_pad, int64_t l,
+                                     const uint32_t *C, const uint32_t *J, uint32_t *Ux_tm,
+                                     uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
+                                     void *stream) {
+    return mask_activation_impl(p, key, pass_id, m, n_pad, l, C, J, nullptr, Ux_tm, K_tm, variant, ws,
+                                ws_bytes, stream);
+}
+
+mosaic_status mosaic_mask_activation_planes(const mosaic_params *p, const mosaic_key *key,
+                                            uint64_t pass_id, int64_t m, int64_t n_pad, int64_t l,
+                                            const uint32_t *C, const uint32_t *J,
+                                            const uint16_t *cj_planes, uint32_t *Ux_tm,
+                                            uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
+                                            void *stream) {
+    if (!cj_planes || !aligned16(cj_planes)) return MOSAIC_ERR_ARG;
+    return mask_activation_impl(p, key, pass_id, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm, variant, ws,
+                                ws_bytes, stream);
+}
+
+mosaic_status mosaic_prepare_activation(const mosaic_params *p, int64_t m, int64_t n_pad,
+                                        const uint32_t *C, const uint32_t *J, uint16_t *cj_planes,
+                                        void *stream) {
+    MOSAIC_TRY(check_params(p));
+    if (!npad_ok(n_pad) || m < 1) return MOSAIC_ERR_SHAPE;
+    if (!C || !J || !cj_planes) return MOSAIC_ERR_ARG;
+    if (!aligned16(cj_planes)) return MOSAIC_ERR_ALIGN;
+    const int64_t Sr = sum_r(p), rd = r_act(p), od = p->act_nested ? off_r(p, p->d) : 0;
+    const int64_t Kp = kpad8(rd), bplane = (n_pad + m) * Kp;
+    cudaStream_t st = as_stream(stream);
+    MOSAIC_TRY(digit_split(C + od, Sr, n_pad, rd, cj_planes, Kp, bplane, st));
+    return digit_split(J + od, Sr, m, rd, cj_planes + n_pad * Kp, Kp, bplane, st);
+}
+
+}  // extern "C"
+
+namespace {
+
+// Unmask + decode; `Lp` (nullable) holds L's digit planes from mosaic_prepare_unmask.
+mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z, int64_t ldz,
+                          const uint32_t *K_tm, const uint32_t *L, const uint16_t *Lp, const uint32_t *S_idx,
+                          const uint32_t *S_val, const float *s_w, const float *s_x, const float *bias,
+                          float *Y, uint32_t *Yhat, int64_t ldy, int variant, void *ws, size_t ws_bytes,
+                          void *stream) {
     MOSAIC_TRY(check_params(p));
     const uint32_t d = p->d;
     const int64_t Sr = sum_r(p), rd = p->r[d - 1], od = off_r(p, d);
@@ -510,7 +594,19 @@ mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const 
     uint32_t *tmp = cv.take<uint32_t>((size_t)(l * m));
     if (!tmp) return MOSAIC_ERR_WORKSPACE;
     // tmp = K + Q_d L^T  (token-major: Q_d^T is the column block [m + od, m + Sr) of Z).
-    MOSAIC_TRY(gemm_u32(variant, cv, Z + m + od, ldz, 1, L, rd, 1, tmp, m, K_tm, m, 1, l, m, rd, st));
+    const uint32_t *Qd = Z + m + od;
+    const bool want_tc = variant == MOSAIC_GEMM_TC || (variant == MOSAIC_GEMM_AUTO && tc_available());
+    const int64_t Kp = kpad8(rd);
+    if (Lp && want_tc && !skinny_ok(Qd, ldz, L, rd, l, rd) && ldz % 4 == 0 && aligned16(Qd) &&
+        cv.used + up(8 * (size_t)(l * Kp)) <= cv.cap) {
+        const size_t mark = cv.used;
+        uint16_t *Qp = cv.take<uint16_t>((size_t)(4 * l * Kp));
+        MOSAIC_TRY(digit_split(Qd, ldz, l, rd, Qp, Kp, l * Kp, st));
+        MOSAIC_TRY(ring_gemm_tc_planes(Qp, Kp, l * Kp, Lp, Kp, m * Kp, tmp, m, K_tm, m, 1, l, m, rd, st));
+        cv.used = mark;
+    } else {
+        MOSAIC_TRY(gemm_u32(variant, cv, Qd, ldz, 1, L, rd, 1, tmp, m, K_tm, m, 1, l, m, rd, st));
+    }
     SparseLevel lev[2];
     int64_t soff = 0;
     for (uint32_t i = 1; i < d; i++) {
@@ -521,6 +617,40 @@ mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const 
     // Y_hat = Y' - tmp - sum_i S_{i+1} Q_i, then decode.
     return unmask_decode(Z, ldz, m, od, l, m, lev, (int)d - 1, tmp, m, s_w, s_x, bias, Y, Yhat, ldy,
                          st);
+}
+
+}  // namespace
+
+extern "C" {
+
+mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z,
+                            int64_t ldz, const uint32_t *K_tm, const uint32_t *L,
+                            const uint32_t *S_idx, const uint32_t *S_val, const float *s_w,
+                            const float *s_x, const float *bias, float *Y, uint32_t *Yhat,
+                            int64_t ldy, int variant, void *ws, size_t ws_bytes, void *stream) {
+    return unmask_impl(p, l, m, Z, ldz, K_tm, L, nullptr, S_idx, S_val, s_w, s_x, bias, Y, Yhat, ldy, variant,
+                       ws, ws_bytes, stream);
+}
+
+mosaic_status mosaic_unmask_planes(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z,
+                                   int64_t ldz, const uint32_t *K_tm, const uint32_t *L,
+                                   const uint16_t *L_planes, const uint32_t *S_idx, const uint32_t *S_val,
+                                   const float *s_w, const float *s_x, const float *bias, float *Y,
+                                   uint32_t *Yhat, int64_t ldy, int variant, void *ws, size_t ws_bytes,
+                                   void *stream) {
+    if (!L_planes || !aligned16(L_planes)) return MOSAIC_ERR_ARG;
+    return unmask_impl(p, l, m, Z, ldz, K_tm, L, L_planes, S_idx, S_val, s_w, s_x, bias, Y, Yhat, ldy, variant,
+                       ws, ws_bytes, stream);
+}
+
+mosaic_status mosaic_prepare_unmask(const mosaic_params *p, int64_t m, const uint32_t *L, uint16_t *L_planes,
+                                    void *stream) {
+    MOSAIC_TRY(check_params(p));
+    if (m < 1) return MOSAIC_ERR_SHAPE;
+    if (!L || !L_planes) return MOSAIC_ERR_ARG;
+    if (!aligned16(L_planes)) return MOSAIC_ERR_ALIGN;
+    const int64_t rd = p->r[p->d - 1], Kp = kpad8(rd);
+    return digit_split(L, rd, m, rd, L_planes, Kp, m * Kp, as_stream(stream));
 }
 
 mosaic_status mosaic_freivalds_setup(const mosaic_params *p, const mosaic_key *key, uint64_t matrix_id,

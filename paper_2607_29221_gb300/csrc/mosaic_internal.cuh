@@ -111,6 +111,14 @@ mosaic_status ring_gemm_tc_planes(const uint16_t *Ap, int64_t ldpa, int64_t a_pl
                                   const uint16_t *Bp, int64_t ldpb, int64_t b_plane, uint32_t *C,
                                   int64_t ldc, const uint32_t *Cin, int64_t ldcin, int sgn,
                                   int64_t M, int64_t N, int64_t K, cudaStream_t st);
+// The same with two outputs side by side in B's rows: columns [0, N1) of the
+// product go to C1 (+ Cin1), columns [N1, N1 + N2) to C2 (+ Cin2); N1 is a
+// multiple of 128 and K > 0.
+mosaic_status ring_gemm_tc_planes2(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const uint16_t *Bp,
+                                   int64_t ldpb, int64_t b_plane, uint32_t *C1, int64_t ldc1,
+                                   const uint32_t *Cin1, int64_t ldcin1, int64_t N1, uint32_t *C2, int64_t ldc2,
+                                   const uint32_t *Cin2, int64_t ldcin2, int64_t N2, int64_t M, int64_t K,
+                                   cudaStream_t st);
 // Legacy mma.sync s8 ring GEMM from int8 digits packed in uint32 operands (NT).
 mosaic_status ring_gemm_mma_s8(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb,
                                uint32_t *C, int64_t ldc, const uint32_t *Cin, int64_t ldcin,

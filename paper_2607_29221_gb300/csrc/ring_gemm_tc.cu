@@ -21,7 +21,7 @@
 //   warp 0      TMA producer: per stage one 3-D box {32 K, rows, 4 planes}
 //               for A and one for B (64-byte swizzle), mbarrier complete_tx
 //   warp 1      TMEM allocation (512 columns) and the single-thread MMA issuer
-//               (20 tcgen05.mma of 128 x BN x 16 per stage)
+//               (12 tcgen05.mma per stage: 8 of 128 x 2BN x 16, 4 of 128 x BN x 16)
 //   warps 2..9  epilogue: tcgen05.ld 32x32b, fp32 -> int32, shift-add (each lane
 //               quarter of TMEM twice, half of the columns each)
 // Every wait is bounded (about 2 s of %globaltimer); on expiry the kernel
@@ -55,9 +55,13 @@ struct Cfg {
     static constexpr int B_BYTES = 4 * B_PLANE;
     static constexpr int STAGE = A_BYTES + B_BYTES;
     static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
-    // kind::f16 instruction descriptor: D f32, A/B bf16, K-major, N >> 3, M >> 4.
+    // kind::f16 instruction descriptors: D f32, A/B bf16, K-major, N >> 3, M >> 4;
+    // IDESC2 has N = 2 BN (two consecutive B digit planes as one operand).
     static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
                                       ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+    static constexpr uint32_t IDESC2 = (1u << 4) | (1u << 7) | (1u << 10) |
+                                       ((uint32_t)((2 * BN) >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+    static_assert(2 * BN <= 256, "paired B planes must fit one MMA");
     static_assert(4 * BN <= (int)TMEM_COLS, "four shift groups must fit in TMEM");
     static_assert(BN % 32 == 0 && BN >= 32 && BN <= 128, "");
 };
@@ -71,6 +75,14 @@ struct TcArgs {
     int M, N, K;
     int tiles_m, tiles_n;
     int split;             // 0: one CTA per tile; 1: stream-K over (tile, chunk) units
+    int dp_tiles;          // split mode: tiles [0, dp_tiles) run whole, one per CTA
+    // Columns [N1, N) go to a second output: C2[i][j - N1] (= Cin2 + ...).
+    // N1 is a multiple of BN, so no tile straddles the two; N1 = N: one output.
+    int N1;
+    uint32_t *C2;
+    int64_t ldc2;
+    const uint32_t *Cin2;
+    int64_t ldcin2;
 };
 
 __device__ __forceinline__ void raise_abort(volatile int *abort_flag) {
@@ -140,18 +152,30 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nk = (a.K + BK - 1) / BK;
     const int nchunks = (nk + CHUNK - 1) / CHUNK;
-    // Work of this CTA: units [u_begin, u_end) of (output tile, 256-wide K
-    // chunk), numbered tile-major; tile t covers rows (t % tiles_m) * BM and
-    // columns (t / tiles_m) * BN, so CTAs running side by side share B tiles.
-    int64_t u_begin, u_end;
+    // Work of this CTA: units of (output tile, 256-wide K chunk), numbered
+    // tile-major; tile t covers rows (t % tiles_m) * BM and columns
+    // (t / tiles_m) * BN, so CTAs running side by side share B tiles.
+    // Segment 0: whole tiles blockIdx.x + w * gridDim.x for every whole wave w
+    // (dp_tiles = waves * gridDim.x; CTAs in step read the same B tiles at the
+    // same K); segment 1: this CTA's even share of the remaining tiles' units
+    // (stream-K).  Without split, segment 0 is the CTA's one tile.
+    int64_t n0 = 0, s1b = 0, n1 = 0;
     if (a.split) {
-        const int64_t U = (int64_t)a.tiles_m * a.tiles_n * nchunks;
-        u_begin = U * blockIdx.x / gridDim.x;
-        u_end = U * (blockIdx.x + 1) / gridDim.x;
+        const int64_t dp_units = (int64_t)a.dp_tiles * nchunks;
+        n0 = (int64_t)(a.dp_tiles / (int)gridDim.x) * nchunks;
+        const int64_t U = (int64_t)a.tiles_m * a.tiles_n * nchunks - dp_units;
+        s1b = dp_units + U * blockIdx.x / gridDim.x;
+        n1 = dp_units + U * (blockIdx.x + 1) / gridDim.x - s1b;
     } else {
-        u_begin = (int64_t)blockIdx.x * nchunks;
-        u_end = u_begin + nchunks;
+        n0 = nchunks;
     }
+    const int64_t n_units = n0 + n1;
+    // Unit of this CTA's k-th step.
+    auto unit_at = [&](int64_t k) -> int64_t {
+        if (k >= n0) return s1b + (k - n0);
+        const int64_t w = k / nchunks;
+        return ((int64_t)blockIdx.x + w * (int64_t)gridDim.x) * nchunks + (k - w * nchunks);
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -179,7 +203,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 0) {
         if (lane == 0) {
             int64_t slot = 0;
-            for (int64_t u = u_begin; u < u_end && !*abort_flag; ++u) {
+            for (int64_t k = 0; k < n_units && !*abort_flag; ++k) {
+                const int64_t u = unit_at(k);
                 const int64_t tile = u / nchunks;
                 const int c = (int)(u - tile * nchunks);
                 const int m0 = (int)(tile % a.tiles_m) * BM, n0 = (int)(tile / a.tiles_m) * BN;
@@ -209,7 +234,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (lane == 0) {
             bool issued_any = false;
             int64_t slot = 0, chunk_count = 0;
-            for (int64_t u = u_begin; u < u_end && !*abort_flag; ++u) {
+            for (int64_t k = 0; k < n_units && !*abort_flag; ++k) {
+                const int64_t u = unit_at(k);
                 const int64_t tile = u / nchunks;
                 const int c = (int)(u - tile * nchunks);
                 const int ks0 = c * CHUNK, ks1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
@@ -229,19 +255,26 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const uint32_t a_base = smem_u32(smem + s * C::STAGE);
                     const uint32_t b_base = a_base + C::A_BYTES;
                     const bool first = ks == ks0;
+                    // The 10 digit products d_i e_j (i + j <= 3) as 6 MMAs: B planes
+                    // j and j + 1 are adjacent in shared memory and the shift
+                    // groups i + j and i + j + 1 adjacent in TMEM, so one N = 2 BN
+                    // product covers both.  A plane 0 goes first: its two paired
+                    // products start all four groups of a chunk.
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
-#pragma unroll
-                        for (int g = 0; g < 4; ++g) {
-#pragma unroll
-                            for (int i = 0; i <= g; ++i) {
-                                const int j = g - i;
-                                const uint64_t ad = sdesc_sw64(a_base + i * C::A_PLANE + kk * 32);
-                                const uint64_t bd = sdesc_sw64(b_base + j * C::B_PLANE + kk * 32);
-                                const uint32_t acc = (first && kk == 0 && i == 0) ? 0u : 1u;
-                                umma_bf16(tmem + g * BN, ad, bd, C::IDESC, acc);
-                            }
-                        }
+                        const uint32_t z = (first && kk == 0) ? 0u : 1u;
+                        const uint64_t a0 = sdesc_sw64(a_base + 0 * C::A_PLANE + kk * 32);
+                        const uint64_t a1 = sdesc_sw64(a_base + 1 * C::A_PLANE + kk * 32);
+                        const uint64_t a2 = sdesc_sw64(a_base + 2 * C::A_PLANE + kk * 32);
+                        const uint64_t a3 = sdesc_sw64(a_base + 3 * C::A_PLANE + kk * 32);
+                        const uint64_t b0 = sdesc_sw64(b_base + 0 * C::B_PLANE + kk * 32);
+                        const uint64_t b2 = sdesc_sw64(b_base + 2 * C::B_PLANE + kk * 32);
+                        umma_bf16(tmem + 0 * BN, a0, b0, C::IDESC2, z);    // d0 e0, d0 e1
+                        umma_bf16(tmem + 2 * BN, a0, b2, C::IDESC2, z);    // d0 e2, d0 e3
+                        umma_bf16(tmem + 1 * BN, a1, b0, C::IDESC2, 1u);   // d1 e0, d1 e1
+                        umma_bf16(tmem + 3 * BN, a1, b2, C::IDESC, 1u);    // d1 e2
+                        umma_bf16(tmem + 2 * BN, a2, b0, C::IDESC2, 1u);   // d2 e0, d2 e1
+                        umma_bf16(tmem + 3 * BN, a3, b0, C::IDESC, 1u);    // d3 e0
                     }
                     issued_any = true;
                     umma_commit(&empty[s]);
@@ -270,7 +303,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int c = 0; c < HB; ++c) acc[c] = 0u;
         int64_t chunk_count = 0;
-        for (int64_t u = u_begin; u < u_end; ++u) {
+        for (int64_t k = 0; k < n_units; ++k) {
+            const int64_t u = unit_at(k);
             if (!mbar_wait(acc_full, (uint32_t)chunk_count & 1, abort_flag)) {
                 raise_abort(abort_flag);
                 break;
@@ -294,26 +328,33 @@ __global__ void __launch_bounds__(THREADS, 1)
 
             const int64_t tile = u / nchunks;
             const int c = (int)(u - tile * nchunks);
-            if (c != nchunks - 1 && u != u_end - 1) continue;
+            if (c != nchunks - 1 && k != n0 - 1 && k != n_units - 1) continue;
             // End of this CTA's segment of the tile: write it out.
-            const bool whole = (u_begin <= tile * nchunks) && (c == nchunks - 1);
-            const int m0 = (int)(tile % a.tiles_m) * BM, n0 = (int)(tile / a.tiles_m) * BN + h * HB;
+            const bool whole = k < n0 || ((s1b <= tile * nchunks) && (c == nchunks - 1));
+            const int m0 = (int)(tile % a.tiles_m) * BM;
+            const int tn0 = (int)(tile / a.tiles_m) * BN;
+            const bool second = tn0 >= a.N1;
+            const int n0 = tn0 - (second ? a.N1 : 0) + h * HB;
+            const int nout = second ? a.N - a.N1 : a.N1;
             const int gm = m0 + row;
             if (gm < a.M) {
-                uint32_t *crow = a.C + (int64_t)gm * a.ldc;
-                const uint32_t *cin = a.Cin ? a.Cin + (int64_t)gm * a.ldcin : nullptr;
+                uint32_t *crow = second ? a.C2 + (int64_t)gm * a.ldc2 : a.C + (int64_t)gm * a.ldc;
+                const uint32_t *cin0 = second ? a.Cin2 : a.Cin;
+                const uint32_t *cin = cin0 ? cin0 + (int64_t)gm * (second ? a.ldcin2 : a.ldcin) : nullptr;
+                const int64_t ldc_o = second ? a.ldc2 : a.ldc;
+                const int64_t ldcin_o = second ? a.ldcin2 : a.ldcin;
                 if (a.sgn < 0) {
 #pragma unroll
                     for (int cc = 0; cc < HB; ++cc) acc[cc] = 0u - acc[cc];
                 }
-                const bool vec = (n0 + HB <= a.N) && ((a.ldc & 3) == 0) &&
+                const bool vec = (n0 + HB <= nout) && ((ldc_o & 3) == 0) &&
                                  ((reinterpret_cast<uintptr_t>(crow) & 15u) == 0) &&
-                                 (!cin || (((a.ldcin & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin) & 15u) == 0)));
+                                 (!cin || (((ldcin_o & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin) & 15u) == 0)));
                 if (a.split && !whole) {
                     // Other CTAs add into this tile too: exact and order-free in Z_{2^32}.
 #pragma unroll
                     for (int cc = 0; cc < HB; ++cc)
-                        if (n0 + cc < a.N) atomicAdd(crow + n0 + cc, acc[cc]);
+                        if (n0 + cc < nout) atomicAdd(crow + n0 + cc, acc[cc]);
                 } else if (vec) {
                     // Plain mode: C = Cin + acc.  Stream-K mode: C (prepared) += acc.
                     const uint32_t *base = a.split ? crow : cin;
@@ -331,7 +372,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
                     for (int cc = 0; cc < HB; ++cc) {
                         const int gn = n0 + cc;
-                        if (gn < a.N) crow[gn] = acc[cc] + (base ? base[gn] : 0u);
+                        if (gn < nout) crow[gn] = acc[cc] + (base ? base[gn] : 0u);
                     }
                 }
             }
@@ -362,10 +403,34 @@ bool make_plane_map(CUtensorMap *map, const uint16_t *base, int64_t K, int64_t r
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// C (and C2 for columns >= N1) = Cin + sgn * A B^T from digit planes.
+struct TcOut {
+    uint32_t *C;
+    int64_t ldc;
+    const uint32_t *Cin;
+    int64_t ldcin;
+    int64_t cols;
+};
+
+// Prepares a stream-K output: its tiles are summed with atomic adds, so it
+// starts as Cin (or 0).
+cudaError_t prepare_split(const TcOut &o, int64_t M, cudaStream_t st) {
+    if (o.cols == 0) return cudaSuccess;
+    if (!o.Cin) return cudaMemset2DAsync(o.C, (size_t)o.ldc * 4, 0, (size_t)o.cols * 4, (size_t)M, st);
+    if (o.Cin != o.C)
+        return cudaMemcpy2DAsync(o.C, (size_t)o.ldc * 4, o.Cin, (size_t)o.ldcin * 4, (size_t)o.cols * 4,
+                                 (size_t)M, cudaMemcpyDeviceToDevice, st);
+    return cudaSuccess;
+}
+
 template <int BN>
 mosaic_status launch_tc(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const uint16_t *Bp,
-                        int64_t ldpb, int64_t b_plane, uint32_t *Cm, int64_t ldc, const uint32_t *Cin,
-                        int64_t ldcin, int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st) {
+                        int64_t ldpb, int64_t b_plane, const TcOut &o1, const TcOut &o2, int sgn,
+                        int64_t M, int64_t K, cudaStream_t st) {
+    const int64_t N = o1.cols + o2.cols;
+    uint32_t *Cm = o1.C;
+    const uint32_t *Cin = o1.Cin;
+    const int64_t ldc = o1.ldc, ldcin = o1.ldcin;
     using C = Cfg<BN>;
     CUtensorMap ta, tb;
     if (!make_plane_map(&ta, Ap, K, M, ldpa, a_plane, BM) || !make_plane_map(&tb, Bp, K, N, ldpb, b_plane, BN))
@@ -392,19 +457,16 @@ mosaic_status launch_tc(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const
     // the idle SMs.
     const int64_t waves = (tiles + sms - 1) / sms;
     const bool split = nchunks >= 8 && (double)tiles / (double)(waves * sms) < 0.9;
-    TcArgs args{Cm, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)K, (int)tiles_m, (int)tiles_n, split ? 1 : 0};
+    TcArgs args{Cm, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)K, (int)tiles_m, (int)tiles_n, split ? 1 : 0,
+                0, (int)o1.cols, o2.C, o2.ldc, o2.Cin, o2.ldcin};
     int64_t grid = tiles;
     if (split) {
-        // Split tiles are summed into C with atomic adds, so C starts as Cin (or 0).
-        cudaError_t e = cudaSuccess;
-        if (!Cin)
-            e = cudaMemset2DAsync(Cm, (size_t)ldc * 4, 0, (size_t)N * 4, (size_t)M, st);
-        else if (Cin != Cm)
-            e = cudaMemcpy2DAsync(Cm, (size_t)ldc * 4, Cin, (size_t)ldcin * 4, (size_t)N * 4, (size_t)M,
-                                  cudaMemcpyDeviceToDevice, st);
-        if (e != cudaSuccess) return MOSAIC_ERR_CUDA;
+        if (prepare_split(o1, M, st) != cudaSuccess || prepare_split(o2, M, st) != cudaSuccess)
+            return MOSAIC_ERR_CUDA;
         args.Cin = nullptr;
+        args.Cin2 = nullptr;
         grid = tiles * nchunks < sms ? tiles * nchunks : sms;
+        args.dp_tiles = (int)((tiles / grid) * grid);   // whole waves run as whole tiles
     }
     if (grid > 0x7fffffff) return MOSAIC_ERR_SHAPE;
     ring_gemm_tc_kernel<BN><<<(unsigned)grid, THREADS, C::SMEM, st>>>(ta, tb, args);
@@ -437,7 +499,20 @@ mosaic_status ring_gemm_tc_planes(const uint16_t *Ap, int64_t ldpa, int64_t a_pl
                                                        (size_t)N * 4, (size_t)M, cudaMemcpyDeviceToDevice, st);
         return e == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
     }
-    return launch_tc<128>(Ap, ldpa, a_plane, Bp, ldpb, b_plane, Cm, ldc, Cin, ldcin, sgn, M, N, K, st);
+    const TcOut o1{Cm, ldc, Cin, ldcin, N}, none{nullptr, 0, nullptr, 0, 0};
+    return launch_tc<128>(Ap, ldpa, a_plane, Bp, ldpb, b_plane, o1, none, sgn, M, K, st);
+}
+
+mosaic_status ring_gemm_tc_planes2(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const uint16_t *Bp,
+                                   int64_t ldpb, int64_t b_plane, uint32_t *C1, int64_t ldc1,
+                                   const uint32_t *Cin1, int64_t ldcin1, int64_t N1, uint32_t *C2, int64_t ldc2,
+                                   const uint32_t *Cin2, int64_t ldcin2, int64_t N2, int64_t M, int64_t K,
+                                   cudaStream_t st) {
+    if (M == 0 || N1 + N2 == 0) return MOSAIC_OK;
+    if (M > (int64_t)INT32_MAX || N1 + N2 > (int64_t)INT32_MAX || N1 % 128 != 0 || K == 0)
+        return MOSAIC_ERR_SHAPE;
+    const TcOut o1{C1, ldc1, Cin1, ldcin1, N1}, o2{C2, ldc2, Cin2, ldcin2, N2};
+    return launch_tc<128>(Ap, ldpa, a_plane, Bp, ldpb, b_plane, o1, o2, 1, M, K, st);
 }
 
 mosaic_status ring_gemm_mma_s8(const uint32_t *, int64_t, const uint32_t *, int64_t, uint32_t *, int64_t,

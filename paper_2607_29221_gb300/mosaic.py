@@ -23,7 +23,7 @@ STATUS = {0: "ok", 1: "invalid argument", 2: "invalid shape", 3: "misaligned", 4
 GEMM_AUTO, GEMM_TC, GEMM_MMA_S8, GEMM_IMAD = 0, 1, 2, 3
 SKINNY_MAX_M = 16   # MOSAIC_SKINNY_MAX_M: token counts the streaming product serves
 OP_RING_GEMM, OP_MASK_CHAINS, OP_MASK_WEIGHT, OP_MASK_ACTIVATION, OP_UNMASK = 1, 2, 3, 4, 5
-OP_FREIVALDS_CHECK = 6
+OP_FREIVALDS_CHECK, OP_ACTIVATION_PLANES, OP_UNMASK_PLANES = 6, 7, 8
 TAG_M, TAG_N, TAG_L, TAG_S, TAG_EW, TAG_R, TAG_T, TAG_EX, TAG_SIGN, TAG_CHECK = range(1, 11)
 
 
@@ -78,6 +78,12 @@ _SIGS = {
     "mosaic_device_status": ([_P], _INT),
     "mosaic_unmask_noalloc": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
                                _INT, _P], _INT),
+    "mosaic_prepare_activation": ([_PP, _I64, _I64, _P, _P, _P, _P], _INT),
+    "mosaic_mask_activation_planes": ([_PP, _PK, _U64, _I64, _I64, _I64, _P, _P, _P, _P, _P, _INT, _P,
+                                       _SZ, _P], _INT),
+    "mosaic_prepare_unmask": ([_PP, _I64, _P, _P, _P], _INT),
+    "mosaic_unmask_planes": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
+                              _INT, _P, _SZ, _P], _INT),
     "mosaic_freivalds_setup": ([_PP, _PK, _U64, _INT, _P, _I64, _I64, _I64, _P, _P, _P], _INT),
     "mosaic_freivalds_check": ([_INT, _P, _P, _I64, _I64, _I64, _P, _I64, _P, _I64, _P, _P, _P, _SZ,
                                 _P], _INT),
@@ -271,3 +277,26 @@ def mosaic_freivalds_check(k, a, Ychk, m, n_pad, l, Z, ldz, Xp, ldx, bad, n_bad,
     _call("mosaic_freivalds_check", k, _ptr(a), _ptr(Ychk), m, n_pad, l, _ptr(Z), ldz, _ptr(Xp), ldx,
           _ptr(bad), _ptr(n_bad), _ptr(ws), 0 if ws is None else ws.numel() * ws.element_size(),
           _stream(stream))
+
+
+def mosaic_prepare_activation(params, m, n_pad, C, J, cj_planes, stream=None):
+    _call("mosaic_prepare_activation", ctypes.byref(params), m, n_pad, _ptr(C), _ptr(J), _ptr(cj_planes),
+          _stream(stream))
+
+
+def mosaic_mask_activation_planes(params, key, pass_id, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm, variant,
+                                  ws, stream=None):
+    _call("mosaic_mask_activation_planes", ctypes.byref(params), ctypes.byref(key), pass_id, m, n_pad, l,
+          _ptr(C), _ptr(J), _ptr(cj_planes), _ptr(Ux_tm), _ptr(K_tm), variant, _ptr(ws),
+          0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
+
+
+def mosaic_prepare_unmask(params, m, L, L_planes, stream=None):
+    _call("mosaic_prepare_unmask", ctypes.byref(params), m, _ptr(L), _ptr(L_planes), _stream(stream))
+
+
+def mosaic_unmask_planes(params, l, m, Z, ldz, K_tm, L, L_planes, S_idx, S_val, s_w, s_x, bias, Y, Yhat,
+                         ldy, variant, ws, stream=None):
+    _call("mosaic_unmask_planes", ctypes.byref(params), l, m, _ptr(Z), ldz, _ptr(K_tm), _ptr(L),
+          _ptr(L_planes), _ptr(S_idx), _ptr(S_val), _ptr(s_w), _ptr(s_x), _ptr(bias), _ptr(Y), _ptr(Yhat),
+          ldy, variant, _ptr(ws), 0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))

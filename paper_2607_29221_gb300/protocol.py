@@ -118,6 +118,15 @@ class SecureLinear:
         M.mosaic_mask_weight(p, proto.key, matrix_id, W, W.stride(0), m, self.n, n_pad, chains.P,
                              chains.CT, self.sign_words, self.s_w, self.L, self.S_idx, self.S_val,
                              self.Wp, self.Wp_planes, self.J, proto.variant, ws)
+        # Stationary tensor-core operands of every pass: [C; J] and L as digit planes.
+        self.cj_planes = self.L_planes = None
+        if self.use_planes:
+            self.cj_planes = torch.empty(M.mosaic_workspace_bytes(M.OP_ACTIVATION_PLANES, m, n_pad, 0, p) // 2,
+                                         dtype=torch.int16, device=dev)
+            M.mosaic_prepare_activation(p, m, n_pad, chains.C, self.J, self.cj_planes)
+            self.L_planes = torch.empty(M.mosaic_workspace_bytes(M.OP_UNMASK_PLANES, m, 0, 0, p) // 2,
+                                        dtype=torch.int16, device=dev)
+            M.mosaic_prepare_unmask(p, m, self.L, self.L_planes)
 
     # Init X ---------------------------------------------------------------
     def init_x(self, l: int, pass_id: int) -> PassMask:
@@ -126,8 +135,12 @@ class SecureLinear:
         K = _u32(l, self.m, device=dev)
         ws = self.proto.workspace(
             M.mosaic_workspace_bytes(M.OP_MASK_ACTIVATION, self.m, self.n_pad, l, p))
-        M.mosaic_mask_activation(p, self.proto.key, pass_id, self.m, self.n_pad, l,
-                                 self.chains.C, self.J, Ux, K, self.proto.variant, ws)
+        if self.cj_planes is not None:
+            M.mosaic_mask_activation_planes(p, self.proto.key, pass_id, self.m, self.n_pad, l, self.chains.C,
+                                            self.J, self.cj_planes, Ux, K, self.proto.variant, ws)
+        else:
+            M.mosaic_mask_activation(p, self.proto.key, pass_id, self.m, self.n_pad, l,
+                                     self.chains.C, self.J, Ux, K, self.proto.variant, ws)
         return PassMask(pass_id, l, Ux, K)
 
     # Online ---------------------------------------------------------------
@@ -166,8 +179,12 @@ class SecureLinear:
         p = self.proto.params
         Y = torch.empty(l, self.m, dtype=torch.float32, device=self.proto.device) if Y is None else Y
         ws = self.proto.workspace(M.mosaic_workspace_bytes(M.OP_UNMASK, self.m, 0, l, p))
-        M.mosaic_unmask(p, l, self.m, Z, Z.stride(0), mp.K, self.L, self.S_idx, self.S_val,
-                        self.s_w, s_x, self.bias, Y, Yhat, self.m, self.proto.variant, ws)
+        if self.L_planes is not None:
+            M.mosaic_unmask_planes(p, l, self.m, Z, Z.stride(0), mp.K, self.L, self.L_planes, self.S_idx,
+                                   self.S_val, self.s_w, s_x, self.bias, Y, Yhat, self.m, self.proto.variant, ws)
+        else:
+            M.mosaic_unmask(p, l, self.m, Z, Z.stride(0), mp.K, self.L, self.S_idx, self.S_val,
+                            self.s_w, s_x, self.bias, Y, Yhat, self.m, self.proto.variant, ws)
         return Y
 
     # Integrity (Init W step 4, Online step 4) ---------------------------

@@ -360,6 +360,35 @@ def test_layer_lwe_only_activation_mask(d, r, t, l):
         _check_layer(g, ref, op, m, l_)
 
 
+@pytest.mark.parametrize("l", [5, 64, 300])
+def test_cached_planes_match_uncached(l):
+    """mosaic_mask_activation_planes / mosaic_unmask_planes (stationary operands
+    split once) give exactly what the plain entry points give."""
+    from paper_2607_29221_gb300 import protocol as PR
+    M = M_()
+    if not M.mosaic_gemm_variant_available(M.GEMM_TC):
+        pytest.skip("tensor-core variant not available")
+    gp, _ = _params(3, (1536, 1024, 652), (80, 80))
+    proto = PR.Protocol(KEY, gp, variant=M.GEMM_TC)
+    m, n = 384, 1000
+    ch = PR.Chains(proto, PR.pad_width(n))
+    layer = PR.SecureLinear(proto, dev(wl.weights(m, n, std=1.0)), 4, ch, bias=dev(wl.bias(m)))
+    assert layer.cj_planes is not None
+    outs = []
+    for cached in (True, False):
+        if not cached:
+            layer.cj_planes = layer.L_planes = None
+        mp = layer.init_x(l, 9)
+        Xp, s_x, Xpl = layer.mask_input(dev(wl.activations(l, n)), mp)
+        Z = layer.server(Xp, Xpl)
+        Yhat = torch.empty(l, m, dtype=torch.int32, device="cuda")
+        Y = layer.unmask(Z, mp, s_x, Yhat=Yhat)
+        M.mosaic_device_status()
+        outs.append((host_u32(mp.Ux), host_u32(mp.K), host_u32(Yhat), host_f32(Y)))
+    for a, b in zip(*outs):
+        assert np.array_equal(a, b)
+
+
 def test_layer_zero_noise_and_no_bias():
     g, ref, op, m, l = _run_layer(3, (96, 64, 40), (6, 5), m=33, n=64, l=9, sigma=0.0, bias=False)
     _check_layer(g, ref, op, m, l)

@@ -186,3 +186,13 @@ def test_few_tokens_edges():
     M.mosaic_ring_gemm(Z, 4, Z, 4, C, 8, 2, 2, 0, M.GEMM_TC)
     got = host(C)
     assert np.all(got[:, :2] == 0) and np.all(got[:, 2:] == 0xFFFFFFFF)
+
+
+@pytest.mark.parametrize("N", [5000, 9984])
+def test_tc_whole_waves_then_stream_k(N):
+    """160 (312) tiles on 152 SMs with 8 K chunks: the first one (two) waves of
+    tiles run whole, one tile per CTA per wave, and the last 8 tiles' chunks
+    are shared by all CTAs."""
+    A = wl.uniform_u32(51, 512, 2048)
+    B = wl.uniform_u32(52, N, 2048)
+    assert np.array_equal(tc_gemm(A, B), ref(A, B))
