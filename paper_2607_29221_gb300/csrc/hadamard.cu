@@ -45,11 +45,17 @@ struct FwhtArgs {
 __device__ __forceinline__ int pad_idx(int i) { return i + (i >> 5); }
 
 // Signed base-2^8 digit i of a (b = a + 0x80808080; digit = byte_i(b) - 128)
-// as bf16 bits.  Digits in [-128, 127] are exact in bf16.
-__device__ __forceinline__ uint16_t digit_bf16(uint32_t a, int i) {
-    const uint32_t b = a + 0x80808080u;
-    const int d = (int)((b >> (8 * i)) & 0xffu) - 128;
-    return __bfloat16_as_ushort(__float2bfloat16_rn((float)d));
+// as an fp32 value, exactly: the byte is placed in the low mantissa bits of
+// 2^23 (the float 2^23 + byte) and 2^23 + 128 is subtracted.  A digit in
+// [-128, 127] has at most 8 significant bits, so its fp32 bits shifted right
+// by 16 are its exact bf16 bits.
+__device__ __forceinline__ uint32_t digit_f32_bits(uint32_t b, int i) {
+    const uint32_t f = __byte_perm(b, 0x4B000000u, 0x7650u | (uint32_t)i);
+    return __float_as_uint(__fadd_rn(__uint_as_float(f), -8388736.0f));
+}
+// bf16 bits of digit i of two ring elements, packed (first in the low half).
+__device__ __forceinline__ uint32_t digit_pair_bf16(uint32_t b0, uint32_t b1, int i) {
+    return __byte_perm(digit_f32_bits(b0, i), digit_f32_bits(b1, i), 0x7632u);
 }
 
 template <int CNT>
@@ -97,32 +103,30 @@ __device__ __forceinline__ void load_u32(const uint32_t *p, uint32_t *v) {
 
 template <int CNT>
 __device__ __forceinline__ void store_planes(uint16_t *p, int64_t plane_stride, const uint32_t *code) {
+    if constexpr (CNT == 1) {
+        const uint32_t b = code[0] + 0x80808080u;
 #pragma unroll
-    for (int d = 0; d < 4; d++) {
-        uint16_t h[CNT];
+        for (int d = 0; d < 4; d++) p[d * plane_stride] = (uint16_t)(digit_f32_bits(b, d) >> 16);
+    } else {
+        static_assert(CNT % 2 == 0, "digit planes are stored two elements at a time");
+        uint32_t b[CNT];
 #pragma unroll
-        for (int q = 0; q < CNT; q++) h[q] = digit_bf16(code[q], d);
-        uint16_t *pd = p + d * plane_stride;
-        if constexpr (CNT % 8 == 0) {
+        for (int q = 0; q < CNT; q++) b[q] = code[q] + 0x80808080u;
 #pragma unroll
-            for (int q = 0; q < CNT; q += 8) {
-                uint4 t;
-                t.x = h[q] | ((uint32_t)h[q + 1] << 16);
-                t.y = h[q + 2] | ((uint32_t)h[q + 3] << 16);
-                t.z = h[q + 4] | ((uint32_t)h[q + 5] << 16);
-                t.w = h[q + 6] | ((uint32_t)h[q + 7] << 16);
-                *reinterpret_cast<uint4 *>(pd + q) = t;
+        for (int d = 0; d < 4; d++) {
+            uint32_t w[CNT / 2];
+#pragma unroll
+            for (int q = 0; q < CNT / 2; q++) w[q] = digit_pair_bf16(b[2 * q], b[2 * q + 1], d);
+            uint16_t *pd = p + d * plane_stride;
+            if constexpr (CNT % 8 == 0) {
+#pragma unroll
+                for (int q = 0; q < CNT / 2; q += 4)
+                    *reinterpret_cast<uint4 *>(pd + 2 * q) = make_uint4(w[q], w[q + 1], w[q + 2], w[q + 3]);
+            } else if constexpr (CNT == 4) {
+                *reinterpret_cast<uint2 *>(pd) = make_uint2(w[0], w[1]);
+            } else {
+                *reinterpret_cast<uint32_t *>(pd) = w[0];
             }
-        } else if constexpr (CNT == 4) {
-            uint2 t;
-            t.x = h[0] | ((uint32_t)h[1] << 16);
-            t.y = h[2] | ((uint32_t)h[3] << 16);
-            *reinterpret_cast<uint2 *>(pd) = t;
-        } else if constexpr (CNT == 2) {
-            *reinterpret_cast<uint32_t *>(pd) = h[0] | ((uint32_t)h[1] << 16);
-        } else {
-#pragma unroll
-            for (int q = 0; q < CNT; q++) pd[q] = h[q];
         }
     }
 }
@@ -210,13 +214,16 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
             }
         }
         // Phase 2: h = E .. 16E across lanes.
+        // The lower lane of a pair keeps v + o, the upper o - v: one fused
+        // multiply-add by +-1 (the product is exact, so the single rounding is
+        // that of the plain sum or difference).
 #pragma unroll
         for (int hl = 1; hl < 32; hl <<= 1) {
-            const bool upper = (lane & hl) != 0;
+            const float sgn = (lane & hl) ? -1.0f : 1.0f;
 #pragma unroll
             for (int e = 0; e < E; e++) {
                 const float o = __shfl_xor_sync(0xffffffffu, v[e], hl);
-                v[e] = upper ? __fsub_rn(o, v[e]) : __fadd_rn(v[e], o);
+                v[e] = __fmaf_rn(v[e], sgn, o);
             }
         }
     }
@@ -295,17 +302,17 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
     if (!active) return;
     const float s = ok ? __fdiv_rn(mx, (float)a.qmax) : __int_as_float(0x7fc00000);
     if (lt == 0) a.scale[row] = s;
-    const float q = (float)a.qmax;
+    // code = clamp(rint(v / s), -qmax, qmax).  |v / s| <= qmax (1 + 2^-23)
+    // < 2^22, where adding 1.5 * 2^23 rounds to the nearest integer (ties to
+    // even) in the low mantissa bits, so the integer is read from the bits.
+    const bool quant = ok && s != 0.0f;
     uint32_t code[E];
 #pragma unroll
     for (int e = 0; e < E; e++) {
-        int32_t c = 0;
-        if (ok && s != 0.0f) {
-            float f = rintf(__fdiv_rn(v[e], s));
-            f = fminf(fmaxf(f, -q), q);
-            c = (int32_t)f;
-        }
-        code[e] = (uint32_t)c;
+        const float t = __fadd_rn(__fdiv_rn(v[e], s), 12582912.0f);
+        int32_t c = __float_as_int(t) - 0x4B400000;
+        c = min(max(c, -a.qmax), a.qmax);
+        code[e] = quant ? (uint32_t)c : 0u;
     }
     if (a.mask) {
         if constexpr (kPrefetch) {

@@ -137,6 +137,11 @@ WORKLOADS = {
         notes="single-layer relative l2 error vs sigma (the paper's single-layer error table), "
               "N(0,0.02) weights with 8 outlier input channels (10x), N(0,1) activations with "
               "4 outlier channels (20x)"),
+    "kernels_hbm": Workload(
+        "kernels_hbm", 2048,
+        (Linear("n4096", 4096, 4096), Linear("n16384", 4096, 16384), Linear("n32768", 1024, 32768)),
+        notes="memory-bound client kernels alone (rotation, encode + mask-add (+ digit planes), "
+              "E_x sampling) on token batches of l x n_pad, L2 flushed between launches"),
     "init_w_70b": Workload(
         "init_w_70b", 0,
         (Linear("qkv", 10240, 8192), Linear("o", 8192, 8192),
