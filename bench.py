@@ -221,20 +221,6 @@ class DecoderLayerRun:
         return self.layer.forward(x)
 
 
-class LinearSet:
-    """Independent secure linear calls on the same tokens (decode sweep)."""
-
-    def __init__(self, chain_parts):
-        self.parts = chain_parts
-        self.ring_macs = sum(p.ring_macs for p in chain_parts)
-
-    def step(self, xs, i):
-        return [p.step(x, i) for p, x in zip(self.parts, xs)]
-
-
-# ---------------------------------------------------------------------------
-# our arm
-# ---------------------------------------------------------------------------
 def _time_steps(torch, runner, make_input, steps, warmup, flush, stream, timed, world, counter=None):
     for i in range(warmup):
         runner.step(make_input(), i)
@@ -382,43 +368,81 @@ def _roofline(variant, M, ring_macs, gemm_ms, bf16, peak_src, traffic):
 
 
 def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed, flush, wk, variant):
-    """Every linear of one 70B layer at 1..256 tokens against pre-masked weights."""
+    """Every linear of one 70B layer at 1..256 tokens per step against
+    pre-masked weights.  Init X does not depend on the input, so the masks of
+    all the timed steps' tokens are drawn by one Init X call per linear before
+    the steps (timed apart and charged to the steps pro rata); each step runs
+    the online part: encode + mask-add, server product, unmask + decode."""
     hbm, bf16, _, peak_src = _peaks()
     t0 = time.perf_counter()
-    parts = {l: LinearSet([LinearChain(proto, dev, [lin], l, rank, timed) for lin in wk.linears])
-             for l in wk.decode_batches[:1]}
+    layers = [LinearChain(proto, dev, [lin], 1, rank, timed).layers[0] for lin in wk.linears]
     init_w_s = time.perf_counter() - t0
-    base = parts[wk.decode_batches[0]]
     sweep = []
     sampler = ClockSampler(_smi_index(dev.index))
     sampler.start()
     time.sleep(0.3)
+    nsteps = args.warmup + args.steps
     for l in wk.decode_batches:
-        # the same pre-masked weights serve every batch size; only the per-call buffers differ
-        runs = []
-        for chain in base.parts:
-            c = LinearChain.__new__(LinearChain)
-            c.l, c.rank, c.layers = l, rank, chain.layers
-            c.bufs = [dict(
-                Xp=torch.empty(l, ly.n_pad, dtype=torch.int32, device=dev),
-                s_x=torch.empty(l, dtype=torch.float32, device=dev),
-                Xpl=(torch.empty(4, l, ly.n_pad, dtype=torch.int16, device=dev)
-                     if ly.use_planes and l > M.SKINNY_MAX_M else None),
-                Z=torch.empty(l, ly.m + proto.sum_r, dtype=torch.int32, device=dev),
-                Y=torch.empty(l, ly.m, dtype=torch.float32, device=dev)) for ly in chain.layers]
-            c.ring_macs = sum(l * (ly.m + proto.sum_r) * ly.n_pad for ly in chain.layers)
-            runs.append(c)
-        runner = LinearSet(runs)
-        xs = [torch.from_numpy(wl.activations(l, ly.n, seed=wl.SEED_X + l)).to(dev)
-              for c in runs for ly in c.layers]
-        step_ms, gemm_ms, _ = _time_steps(torch, runner, lambda: xs, args.steps, args.warmup, flush, stream,
-                                          timed, world)
-        w_bytes = sum((ly.m + proto.sum_r) * ly.n_pad * 4 for c in runs for ly in c.layers)
+        bufs = [dict(Xp=torch.empty(l, ly.n_pad, dtype=torch.int32, device=dev),
+                     s_x=torch.empty(l, dtype=torch.float32, device=dev),
+                     Xpl=(torch.empty(4, l, ly.n_pad, dtype=torch.int16, device=dev)
+                          if ly.use_planes and l > M.SKINNY_MAX_M else None),
+                     Z=torch.empty(l, ly.m + proto.sum_r, dtype=torch.int32, device=dev),
+                     Y=torch.empty(l, ly.m, dtype=torch.float32, device=dev)) for ly in layers]
+        xs = [torch.from_numpy(wl.activations(l, ly.n, seed=wl.SEED_X + l)).to(dev) for ly in layers]
+        # Init X for every step's tokens at once (fresh randomness per token).
+        flush.fill_(0)
+        a = torch.cuda.Event(enable_timing=True); b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        masks = [ly.init_x(l * nsteps, 1_000_000 * (rank + 1) + 10_000 * l + i) for i, ly in enumerate(layers)]
+        b.record(stream)
+        torch.cuda.synchronize()
+        initx_ms = a.elapsed_time(b) / nsteps
+
+        class _Online:
+            ring_macs = sum(l * (ly.m + proto.sum_r) * ly.n_pad for ly in layers)
+
+            def step(self, x_unused, i):
+                k = i % nsteps
+                for ly, bf, mp, x in zip(layers, bufs, masks, xs):
+                    part = PR.PassMask(mp.pass_id, l, mp.Ux[k * l:(k + 1) * l], mp.K[k * l:(k + 1) * l])
+                    ly.mask_input(x, part, bf["Xp"], bf["s_x"], bf["Xpl"])
+                    ly.server(bf["Xp"], bf["Xpl"], bf["Z"])
+                    ly.unmask(bf["Z"], part, bf["s_x"], bf["Y"])
+
+        runner = _Online()
+        eager_ms, gemm_ms, launches = _time_steps(torch, runner, lambda: None, args.steps, args.warmup, flush,
+                                                  stream, timed, world, M.mosaic_kernel_launches)
+        # The same steps as CUDA graphs (one per step: each reads its own rows
+        # of the drawn masks), replayed without the Python launch overhead.
+        graphs = []
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        for k in range(nsteps):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=side):
+                runner.step(None, k)
+            graphs.append(g)
+        torch.cuda.synchronize()
+
+        class _Replay:
+            def step(self, x_unused, i):
+                graphs[i % nsteps].replay()
+
+        online_ms, _, _ = _time_steps(torch, _Replay(), lambda: None, args.steps, args.warmup, flush, stream,
+                                      timed, world)
+        del graphs
+        step_ms = online_ms + initx_ms
+        del masks
+        w_bytes = sum((ly.m + proto.sum_r) * ly.n_pad * 4 for ly in layers)
         # up to SKINNY_MAX_M tokens the server streams uint32 W' (4 B an element),
         # beyond that the tensor cores read its bf16 digit planes (8 B an element)
         skinny = variant != M.GEMM_IMAD and l <= M.SKINNY_MAX_M
         read_bytes = w_bytes if skinny or variant == M.GEMM_IMAD else 2 * w_bytes
         sweep.append({"l": l, "ms_per_step": round(step_ms, 4), "tokens_s": round(world * l / (step_ms / 1e3), 1),
+                      "online_ms": round(online_ms, 4), "online_ms_eager": round(eager_ms, 4),
+                      "init_x_ms_per_step": round(initx_ms, 4),
+                      "gpu_launches_per_step": int(round(launches / args.steps)),
                       "gemm_ms": round(gemm_ms, 4), "ring_tops": round(2 * runner.ring_macs / (gemm_ms / 1e3) / 1e12, 2),
                       "server_kernel": "ring_gemm_skinny" if skinny else
                                        ("ring_gemm_imad" if variant == M.GEMM_IMAD else "ring_gemm_tc"),
@@ -436,8 +460,12 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
            "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights)",
            "config": {"workload": args.workload, "batches": list(wk.decode_batches),
                       "linears": [{"name": x.name, "m": x.m, "n": x.n} for x in wk.linears],
-                      "params": "Example 3.1", "l2": "flushed between timed steps (256 MiB write)"},
+                      "params": "Example 3.1", "l2": "flushed between timed steps (256 MiB write)",
+                      "step": "online part (encode, server product, unmask) of every linear, one CUDA "
+                              "graph per step, + Init X of the step's tokens, drawn ahead for all steps in "
+                              "one call per linear and charged pro rata"},
            "init_w_s": round(init_w_s, 3), "sweep": sweep,
+           "gpu_launches": first["gpu_launches_per_step"] * args.steps,
            "roofline": {"bound": "hbm", "achieved": first["server_read_gbs"], "peak": hbm, "unit": "GB/s",
                         "frac": first["server_hbm_frac"], "traffic": None, "peak_source": peak_src,
                         "kernel": first["server_kernel"] + " at %d token(s): reads of the server operand"

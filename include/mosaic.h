@@ -301,6 +301,21 @@ mosaic_status mosaic_mask_activation_planes(const mosaic_params *p, const mosaic
                                             uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
                                             void *stream);
 
+/* General form of Init X: cj_planes as in mosaic_mask_activation_planes
+ * (nullable: split per call), and the pass id is pass_id + *pass_dev when
+ * pass_dev (a device word) is given -- read on the device when the samplers
+ * run, so that a CUDA graph captured around this call (and around
+ * mosaic_advance_pass) draws a fresh pass on every replay.  With pass_dev
+ * NULL it is mosaic_mask_activation(_planes). */
+mosaic_status mosaic_mask_activation_ex(const mosaic_params *p, const mosaic_key *key, uint64_t pass_id,
+                                        const uint64_t *pass_dev, int64_t m, int64_t n_pad, int64_t l,
+                                        const uint32_t *C, const uint32_t *J, const uint16_t *cj_planes,
+                                        uint32_t *Ux_tm, uint32_t *K_tm, int variant, void *ws,
+                                        size_t ws_bytes, void *stream);
+
+/* *pass_dev += delta, enqueued on `stream` (one-thread kernel). */
+mosaic_status mosaic_advance_pass(uint64_t *pass_dev, uint64_t delta, void *stream);
+
 /* ------------------------------------------------------------------------ */
 /* Unmask and decode (Approx-MatMul Online step 5; Pi_Sec-Linear Online      */
 /* step 3).                                                                  */

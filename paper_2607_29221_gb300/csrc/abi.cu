@@ -464,10 +464,10 @@ namespace {
 // Init X; `cj` (nullable) holds the digit planes of [C-factor; J-factor] made
 // by mosaic_prepare_activation.
 mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key, uint64_t pass_id,
-                                   int64_t m, int64_t n_pad, int64_t l, const uint32_t *C,
-                                   const uint32_t *J, const uint16_t *cj, uint32_t *Ux_tm,
-                                   uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
-                                   void *stream) {
+                                   const uint64_t *pass_dev, int64_t m, int64_t n_pad, int64_t l,
+                                   const uint32_t *C, const uint32_t *J, const uint16_t *cj,
+                                   uint32_t *Ux_tm, uint32_t *K_tm, int variant, void *ws,
+                                   size_t ws_bytes, void *stream) {
     MOSAIC_TRY(check_params(p));
     if (!key) return MOSAIC_ERR_ARG;
     if (!npad_ok(n_pad) || m < 1 || l < 0 || l >= ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
@@ -484,21 +484,21 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
     Carve cv{static_cast<char *>(ws), ws_bytes, 0};
     uint32_t *Rt = cv.take<uint32_t>((size_t)(l * rd));
     if (!Rt) return MOSAIC_ERR_WORKSPACE;
-    MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_R, 0), pass_id, R, l, rd, Rt, rd, st));
+    MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_R, 0), pass_id, R, l, rd, Rt, rd, st, pass_dev));
     SparseLevel lev[2];
     for (uint32_t i = 1; i < d; i++) {
         const uint32_t t = p->t[i], ri = p->r[i - 1];
         uint32_t *ti = cv.take<uint32_t>((size_t)(l * t));
         uint32_t *tv = cv.take<uint32_t>((size_t)(l * t));
         if (!ti || !tv) return MOSAIC_ERR_WORKSPACE;
-        MOSAIC_TRY(prg_sparse(k, tag_of(MOSAIC_TAG_T, i + 1), pass_id, R, l, ri, t, ti, tv, nullptr, st));
+        MOSAIC_TRY(prg_sparse(k, tag_of(MOSAIC_TAG_T, i + 1), pass_id, R, l, ri, t, ti, tv, nullptr, st, pass_dev));
         lev[i - 1] = SparseLevel{ti, tv, (int)t, off_r(p, i), ri};
     }
     // U_x^T = E_x^T + R^T C_d^T + sum_i T_{i+1}^T C_i^T and
     // K^T = R^T J_d^T + sum_i T_{i+1}^T J_i^T: the two dense products share
     // R^T, so on the tensor cores they run as one product against the stacked
     // [C_d; J_d] (planes cached by mosaic_prepare_activation, or split here).
-    MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EX, 0), pass_id, R, p->sigma, l * n_pad, Ux_tm, st));
+    MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EX, 0), pass_id, R, p->sigma, l * n_pad, Ux_tm, st, pass_dev));
     const bool want_tc = variant == MOSAIC_GEMM_TC || (variant == MOSAIC_GEMM_AUTO && tc_available());
     const int64_t Kp = kpad8(rd), bplane = (n_pad + m) * Kp;
     const size_t need = up(8 * (size_t)(l * Kp)) + (cj ? 0 : up(8 * (size_t)bplane));
@@ -542,8 +542,8 @@ mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *k
                                      const uint32_t *C, const uint32_t *J, uint32_t *Ux_tm,
                                      uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
                                      void *stream) {
-    return mask_activation_impl(p, key, pass_id, m, n_pad, l, C, J, nullptr, Ux_tm, K_tm, variant, ws,
-                                ws_bytes, stream);
+    return mask_activation_impl(p, key, pass_id, nullptr, m, n_pad, l, C, J, nullptr, Ux_tm, K_tm, variant,
+                                ws, ws_bytes, stream);
 }
 
 mosaic_status mosaic_mask_activation_planes(const mosaic_params *p, const mosaic_key *key,
@@ -553,8 +553,23 @@ mosaic_status mosaic_mask_activation_planes(const mosaic_params *p, const mosaic
                                             uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
                                             void *stream) {
     if (!cj_planes || !aligned16(cj_planes)) return MOSAIC_ERR_ARG;
-    return mask_activation_impl(p, key, pass_id, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm, variant, ws,
-                                ws_bytes, stream);
+    return mask_activation_impl(p, key, pass_id, nullptr, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm,
+                                variant, ws, ws_bytes, stream);
+}
+
+mosaic_status mosaic_mask_activation_ex(const mosaic_params *p, const mosaic_key *key, uint64_t pass_id,
+                                        const uint64_t *pass_dev, int64_t m, int64_t n_pad, int64_t l,
+                                        const uint32_t *C, const uint32_t *J, const uint16_t *cj_planes,
+                                        uint32_t *Ux_tm, uint32_t *K_tm, int variant, void *ws,
+                                        size_t ws_bytes, void *stream) {
+    if (cj_planes && !aligned16(cj_planes)) return MOSAIC_ERR_ALIGN;
+    return mask_activation_impl(p, key, pass_id, pass_dev, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm,
+                                variant, ws, ws_bytes, stream);
+}
+
+mosaic_status mosaic_advance_pass(uint64_t *pass_dev, uint64_t delta, void *stream) {
+    if (!pass_dev) return MOSAIC_ERR_ARG;
+    return add_u64(pass_dev, delta, as_stream(stream));
 }
 
 mosaic_status mosaic_prepare_activation(const mosaic_params *p, int64_t m, int64_t n_pad,

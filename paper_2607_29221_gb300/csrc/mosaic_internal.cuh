@@ -76,16 +76,21 @@ inline bool is_pow2(int64_t v) { return v > 0 && (v & (v - 1)) == 0; }
 
 // ---- internal launchers (all enqueue on `st`, validate nothing beyond what they state) ----
 
+// The samplers draw from stream id sid + (*sid_dev if sid_dev is given; read
+// on the device when the kernel runs).
 // Uniform words: out[i * ldo + j] = word (i * cols + j).
 mosaic_status prg_uniform(const Key &key, uint32_t tag, uint64_t sid, int rounds, int64_t rows,
-                          int64_t cols, uint32_t *out, int64_t ldo, cudaStream_t st);
+                          int64_t cols, uint32_t *out, int64_t ldo, cudaStream_t st,
+                          const uint64_t *sid_dev = nullptr);
 // Discrete Gaussian elements.
 mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int rounds, float sigma,
-                           int64_t count, uint32_t *out, cudaStream_t st);
+                           int64_t count, uint32_t *out, cudaStream_t st, const uint64_t *sid_dev = nullptr);
 // Sparse rows.
 mosaic_status prg_sparse(const Key &key, uint32_t tag, uint64_t sid, int rounds, int64_t rows,
                          uint32_t r, uint32_t t, uint32_t *idx, uint32_t *val, uint32_t *fail,
-                         cudaStream_t st);
+                         cudaStream_t st, const uint64_t *sid_dev = nullptr);
+// *p += delta on the stream (advances a device-side pass counter).
+mosaic_status add_u64(uint64_t *p, uint64_t delta, cudaStream_t st);
 // Host-side Gaussian CDF table (long double), B = ceil(12 sigma); returns B.
 int gaussian_table_host(float sigma, unsigned long long *table /* 2*kMaxGaussBound+1 */);
 

@@ -12,8 +12,18 @@ namespace {
 constexpr int kThreads = 256;
 
 // One thread per 64-byte ChaCha block: 16 consecutive stream words.
-__global__ void uniform_kernel(Key key, uint32_t tag, uint32_t sid_lo, uint32_t sid_hi, int rounds,
+// Stream id of a launch: sid, plus *sid_dev when given (read on the device,
+// so that a captured graph draws a fresh stream on every replay).
+__device__ __forceinline__ void stream_id(uint64_t sid, const uint64_t *sid_dev, uint32_t &lo, uint32_t &hi) {
+    const uint64_t s = sid + (sid_dev ? *sid_dev : 0ull);
+    lo = (uint32_t)s;
+    hi = (uint32_t)(s >> 32);
+}
+
+__global__ void uniform_kernel(Key key, uint32_t tag, uint64_t sid, const uint64_t *sid_dev, int rounds,
                                int64_t cols, int64_t total, uint32_t *out, int64_t ldo) {
+    uint32_t sid_lo, sid_hi;
+    stream_id(sid, sid_dev, sid_lo, sid_hi);
     const int64_t nblk = (total + 15) / 16;
     for (int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; b < nblk;
          b += (int64_t)gridDim.x * blockDim.x) {
@@ -40,9 +50,11 @@ struct GaussTable {
 // One thread per block: 8 samples, each from two consecutive words.  The
 // sample is k = (number of table entries <= u) - B, capped at B, i.e. the
 // smallest k_j with u < table[j] (table is non-decreasing).
-__global__ void gaussian_kernel(Key key, uint32_t tag, uint32_t sid_lo, uint32_t sid_hi, int rounds,
+__global__ void gaussian_kernel(Key key, uint32_t tag, uint64_t sid, const uint64_t *sid_dev, int rounds,
                                 GaussTable tab, int64_t count, uint32_t *out) {
     __shared__ unsigned long long st[2 * kMaxGaussBound + 1];
+    uint32_t sid_lo, sid_hi;
+    stream_id(sid, sid_dev, sid_lo, sid_hi);
     for (int i = threadIdx.x; i < tab.n; i += blockDim.x) st[i] = tab.t[i];
     __syncthreads();
     const int64_t nblk = (count + 7) / 8;
@@ -80,9 +92,11 @@ __global__ void gaussian_kernel(Key key, uint32_t tag, uint32_t sid_lo, uint32_t
 constexpr int kSparseWarps = 4;
 
 __global__ void __launch_bounds__(kSparseWarps * 32)
-    sparse_kernel(Key key, uint32_t tag, uint32_t sid_lo, uint32_t sid_hi, int rounds, int64_t rows,
+    sparse_kernel(Key key, uint32_t tag, uint64_t sid, const uint64_t *sid_dev, int rounds, int64_t rows,
                   uint32_t r, int t, uint32_t *idx, uint32_t *val, uint32_t *fail, int bitmap_words) {
     extern __shared__ uint32_t sm[];
+    uint32_t sid_lo, sid_hi;
+    stream_id(sid, sid_dev, sid_lo, sid_hi);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t j = (int64_t)blockIdx.x * kSparseWarps + warp;
     if (j >= rows) return;
@@ -177,17 +191,17 @@ int gaussian_table_host(float sigma, unsigned long long *table) {
 }
 
 mosaic_status prg_uniform(const Key &key, uint32_t tag, uint64_t sid, int rounds, int64_t rows,
-                          int64_t cols, uint32_t *out, int64_t ldo, cudaStream_t st) {
+                          int64_t cols, uint32_t *out, int64_t ldo, cudaStream_t st, const uint64_t *sid_dev) {
     const int64_t total = rows * cols;
     if (total == 0) return MOSAIC_OK;
     const int64_t nblk = (total + 15) / 16;
     uniform_kernel<<<grid_for(nblk, kThreads), kThreads, 0, st>>>(
-        key, tag, (uint32_t)sid, (uint32_t)(sid >> 32), rounds, cols, total, out, ldo);
+        key, tag, sid, sid_dev, rounds, cols, total, out, ldo);
     return launch_status();
 }
 
 mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int rounds, float sigma,
-                           int64_t count, uint32_t *out, cudaStream_t st) {
+                           int64_t count, uint32_t *out, cudaStream_t st, const uint64_t *sid_dev) {
     if (count == 0) return MOSAIC_OK;
     if (sigma == 0.0f) {
         return cudaMemsetAsync(out, 0, sizeof(uint32_t) * (size_t)count, st) == cudaSuccess
@@ -198,13 +212,13 @@ mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int round
     tab.n = 2 * tab.bound + 1;
     const int64_t nblk = (count + 7) / 8;
     gaussian_kernel<<<grid_for(nblk, kThreads), kThreads, 0, st>>>(
-        key, tag, (uint32_t)sid, (uint32_t)(sid >> 32), rounds, tab, count, out);
+        key, tag, sid, sid_dev, rounds, tab, count, out);
     return launch_status();
 }
 
 mosaic_status prg_sparse(const Key &key, uint32_t tag, uint64_t sid, int rounds, int64_t rows,
                          uint32_t r, uint32_t t, uint32_t *idx, uint32_t *val, uint32_t *fail,
-                         cudaStream_t st) {
+                         cudaStream_t st, const uint64_t *sid_dev) {
     if (rows == 0) return MOSAIC_OK;
     const int bitmap_words = (int)((r + 31) / 32);
     const size_t smem = (size_t)kSparseWarps * (512 + bitmap_words) * sizeof(uint32_t);
@@ -213,9 +227,19 @@ mosaic_status prg_sparse(const Key &key, uint32_t tag, uint64_t sid, int rounds,
             cudaSuccess)
         return MOSAIC_ERR_CUDA;
     sparse_kernel<<<(unsigned)((rows + kSparseWarps - 1) / kSparseWarps), kSparseWarps * 32, smem, st>>>(
-        key, tag, (uint32_t)sid, (uint32_t)(sid >> 32), rounds, rows, r, (int)t, idx, val, fail,
-        bitmap_words);
+        key, tag, sid, sid_dev, rounds, rows, r, (int)t, idx, val, fail, bitmap_words);
     return launch_status();
 }
 
+}  // namespace mosaic
+
+namespace mosaic {
+namespace {
+__global__ void add_u64_kernel(uint64_t *p, uint64_t delta) { *p += delta; }
+}  // namespace
+
+mosaic_status add_u64(uint64_t *p, uint64_t delta, cudaStream_t st) {
+    add_u64_kernel<<<1, 1, 0, st>>>(p, delta);
+    return launch_status();
+}
 }  // namespace mosaic

@@ -432,6 +432,91 @@ mosaic_status launch_pgather(const GatherArgs &a, cudaStream_t st) {
     return launch_status();
 }
 
+// ---------------------------------------------------------------------------
+// Few staged rows (g_count <= 4, e.g. the unmask of a decode step): one warp
+// per list entity.  Each block stages the g_count rows of the level's segment
+// once and its warps walk entities; the 32 lanes read an entity's (position,
+// value) list with coalesced loads, each lane sums its share of the pairs for
+// every staged row, and a butterfly sums the lanes.  The cost is one pass
+// over the lists.
+// ---------------------------------------------------------------------------
+constexpr int kFewRows = 8;
+constexpr int kFewWarps = 8;
+
+template <bool LIST_IS_COL, bool CLAMP>
+__global__ void __launch_bounds__(kFewWarps * 32) gather_few_kernel(GatherArgs a) {
+    extern __shared__ uint32_t sf[];
+    const int G = (int)a.g_count, r = (int)a.r, t = a.t;
+    for (int i = threadIdx.x; i < G * r; i += blockDim.x) {
+        const int g = i / r, p = i - g * r;
+        sf[i] = a.src[(int64_t)g * a.lds + a.col0 + p];
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rlast = a.r - 1;
+    const int64_t stride = (int64_t)gridDim.x * kFewWarps;
+    for (int64_t e = (int64_t)blockIdx.x * kFewWarps + warp; e < a.nlist; e += stride) {
+        uint32_t acc[kFewRows];
+#pragma unroll
+        for (int k = 0; k < kFewRows; k++) acc[k] = 0u;
+        const uint32_t *ip = a.idx + e * t;
+        const uint32_t *vp = a.val + e * t;
+        for (int q = lane; q < t; q += 32) {
+            uint32_t p = ip[q];
+            if (CLAMP) p = min(p, rlast);
+            const uint32_t v = vp[q];
+#pragma unroll
+            for (int k = 0; k < kFewRows; k++)
+                if (k < G) acc[k] += v * sf[k * r + p];
+        }
+#pragma unroll
+        for (int k = 0; k < kFewRows; k++) {
+            if (k >= G) break;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) acc[k] += __shfl_xor_sync(0xffffffffu, acc[k], o);
+        }
+        // lane k finishes staged row k
+        uint32_t mine = 0u;
+#pragma unroll
+        for (int k = 0; k < kFewRows; k++)
+            if (lane == k) mine = acc[k];
+        if (lane < G) {
+            const int64_t row = LIST_IS_COL ? lane : e;
+            const int64_t col = LIST_IS_COL ? e : lane;
+            uint32_t res = a.sgn >= 0 ? mine : 0u - mine;
+            if (a.a) res += a.a[row * a.lda + col];
+            if (a.b) res -= a.b[row * a.ldb + col];
+            if (a.out) a.out[row * a.ldo + col] = res;
+            if (a.decode) {
+                float y = __fmul_rn(__fmul_rn(__int2float_rn((int32_t)res), a.s_w[col]), a.s_x[row]);
+                if (a.bias) y = __fadd_rn(y, a.bias[col]);
+                a.Y[row * a.ldy + col] = y;
+            }
+        }
+    }
+}
+
+template <bool LIST_IS_COL, bool CLAMP>
+mosaic_status launch_few(const GatherArgs &a, cudaStream_t st) {
+    const size_t smem = (size_t)a.g_count * a.r * sizeof(uint32_t);
+    auto kern = gather_few_kernel<LIST_IS_COL, CLAMP>;
+    static unsigned long long attr_set = 0;   // one bit per device ordinal
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return MOSAIC_ERR_CUDA;
+    if (!(attr_set & (1ull << (dev & 63)))) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 192 * 1024) != cudaSuccess)
+            return MOSAIC_ERR_CUDA;
+        attr_set |= 1ull << (dev & 63);
+    }
+    // Enough warps to stream the lists; every block stages the rows once.
+    const int64_t need = (a.nlist + kFewWarps - 1) / kFewWarps;
+    const int64_t cap = (int64_t)sms * 4;
+    kern<<<(unsigned)(need < cap ? need : cap), kFewWarps * 32, smem, st>>>(a);
+    return launch_status();
+}
+
 template <int TG, bool LIST_IS_COL, bool CLAMP>
 mosaic_status launch_gather(const GatherArgs &a, cudaStream_t st) {
     const size_t smem = gather_smem(TG, a.segp);
@@ -447,6 +532,10 @@ mosaic_status launch_gather(const GatherArgs &a, cudaStream_t st) {
 
 template <bool LIST_IS_COL, bool CLAMP>
 mosaic_status dispatch_gather(GatherArgs a, cudaStream_t st) {
+    // Up to 4 staged rows the lists dominate and one pass over them wins; from
+    // about 8 rows on the tiled gather's line reads win despite its padding.
+    if (a.t > 0 && a.r >= 1 && a.g_count <= 4 && a.g_count * (int64_t)a.r <= 48 * 1024)
+        return launch_few<LIST_IS_COL, CLAMP>(a, st);
     const bool lists_vec = a.t > 0 && (a.t & 3) == 0 &&
                            ((reinterpret_cast<uintptr_t>(a.idx) | reinterpret_cast<uintptr_t>(a.val)) & 15u) == 0;
     if (lists_vec && a.r >= 1 && a.r <= kPgMaxR) return launch_pgather<LIST_IS_COL, CLAMP>(a, st);

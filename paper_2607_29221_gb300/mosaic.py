@@ -81,6 +81,9 @@ _SIGS = {
     "mosaic_prepare_activation": ([_PP, _I64, _I64, _P, _P, _P, _P], _INT),
     "mosaic_mask_activation_planes": ([_PP, _PK, _U64, _I64, _I64, _I64, _P, _P, _P, _P, _P, _INT, _P,
                                        _SZ, _P], _INT),
+    "mosaic_mask_activation_ex": ([_PP, _PK, _U64, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _INT, _P, _SZ,
+                                   _P], _INT),
+    "mosaic_advance_pass": ([_P, _U64, _P], _INT),
     "mosaic_prepare_unmask": ([_PP, _I64, _P, _P, _P], _INT),
     "mosaic_unmask_planes": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
                               _INT, _P, _SZ, _P], _INT),
@@ -300,3 +303,14 @@ def mosaic_unmask_planes(params, l, m, Z, ldz, K_tm, L, L_planes, S_idx, S_val, 
     _call("mosaic_unmask_planes", ctypes.byref(params), l, m, _ptr(Z), ldz, _ptr(K_tm), _ptr(L),
           _ptr(L_planes), _ptr(S_idx), _ptr(S_val), _ptr(s_w), _ptr(s_x), _ptr(bias), _ptr(Y), _ptr(Yhat),
           ldy, variant, _ptr(ws), 0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
+
+
+def mosaic_mask_activation_ex(params, key, pass_id, pass_dev, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm,
+                              variant, ws, stream=None):
+    _call("mosaic_mask_activation_ex", ctypes.byref(params), ctypes.byref(key), pass_id, _ptr(pass_dev), m,
+          n_pad, l, _ptr(C), _ptr(J), _ptr(cj_planes), _ptr(Ux_tm), _ptr(K_tm), variant, _ptr(ws),
+          0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
+
+
+def mosaic_advance_pass(pass_dev, delta=1, stream=None):
+    _call("mosaic_advance_pass", _ptr(pass_dev), delta, _stream(stream))

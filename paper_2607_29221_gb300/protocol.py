@@ -129,19 +129,18 @@ class SecureLinear:
             M.mosaic_prepare_unmask(p, m, self.L, self.L_planes)
 
     # Init X ---------------------------------------------------------------
-    def init_x(self, l: int, pass_id: int) -> PassMask:
+    def init_x(self, l: int, pass_id: int, pass_dev=None, out: PassMask | None = None) -> PassMask:
+        """Init X for one pass.  pass_dev (a device int64 word, optional) is
+        added to pass_id on the device, so that a captured CUDA graph draws a
+        fresh pass on every replay; `out` reuses preallocated U_x / K buffers."""
         p, dev = self.proto.params, self.proto.device
-        Ux = _u32(l, self.n_pad, device=dev)
-        K = _u32(l, self.m, device=dev)
+        Ux = _u32(l, self.n_pad, device=dev) if out is None else out.Ux
+        K = _u32(l, self.m, device=dev) if out is None else out.K
         ws = self.proto.workspace(
             M.mosaic_workspace_bytes(M.OP_MASK_ACTIVATION, self.m, self.n_pad, l, p))
-        if self.cj_planes is not None:
-            M.mosaic_mask_activation_planes(p, self.proto.key, pass_id, self.m, self.n_pad, l, self.chains.C,
-                                            self.J, self.cj_planes, Ux, K, self.proto.variant, ws)
-        else:
-            M.mosaic_mask_activation(p, self.proto.key, pass_id, self.m, self.n_pad, l,
-                                     self.chains.C, self.J, Ux, K, self.proto.variant, ws)
-        return PassMask(pass_id, l, Ux, K)
+        M.mosaic_mask_activation_ex(p, self.proto.key, pass_id, pass_dev, self.m, self.n_pad, l,
+                                    self.chains.C, self.J, self.cj_planes, Ux, K, self.proto.variant, ws)
+        return PassMask(pass_id, l, Ux, K) if out is None else out
 
     # Online ---------------------------------------------------------------
     def mask_input(self, X_tm: torch.Tensor, mp: PassMask, Xp=None, s_x=None, Xplanes=None):

@@ -312,15 +312,17 @@ def test_layer_tiled_gather_shapes(r, t):
         _check_layer(g, ref, op, m, l)
 
 
-def test_unmask_clamps_out_of_range_positions():
+@pytest.mark.parametrize("l", [40, 3])
+def test_unmask_clamps_out_of_range_positions(l):
     """Caller-supplied S positions at or beyond r_i are read as r_i - 1 (no
     read leaves the staged segment): the unmask with positions 2^32 - 1 gives
-    the same Y_hat as with positions r_i - 1."""
+    the same Y_hat as with positions r_i - 1 (tiled gather at 40 tokens, the
+    few-rows gather at 3)."""
     from paper_2607_29221_gb300 import protocol as PR
     M = M_()
     gp, op = _params(3, (96, 64, 40), (8, 4))
     proto = PR.Protocol(KEY, gp, variant=M.GEMM_AUTO)
-    m, n, l = 70, 128, 40
+    m, n = 70, 128
     ch = PR.Chains(proto, PR.pad_width(n))
     layer = PR.SecureLinear(proto, dev(wl.weights(m, n, std=1.0)), 9, ch)
     mp = layer.init_x(l, 3)
@@ -407,3 +409,57 @@ def test_layer_attn_proj_7b_full():
     g, ref, op, m, l = _run_layer(3, (1536, 1024, 652), (80, 80), m=4096, n=4096, l=512,
                                   w_std=0.02, variant=_variants()[-1])
     _check_layer(g, ref, op, m, l)
+
+
+def test_mask_activation_entry_points_and_device_pass_id():
+    """mosaic_mask_activation, _planes and _ex give the same U_x, K; with a
+    device pass word the pass is pass_id + *pass_dev, and a CUDA graph
+    captured around _ex and mosaic_advance_pass draws passes k, k+1, ... on
+    its replays."""
+    from paper_2607_29221_gb300 import protocol as PR
+    M = M_()
+    gp, _ = _params(3, (96, 64, 40), (8, 4))
+    proto = PR.Protocol(KEY, gp, variant=M.GEMM_AUTO)
+    m, n, l = 200, 256, 48
+    ch = PR.Chains(proto, PR.pad_width(n))
+    layer = PR.SecureLinear(proto, dev(wl.weights(m, n, std=1.0)), 6, ch)
+    n_pad = layer.n_pad
+    ws = proto.workspace(M.mosaic_workspace_bytes(M.OP_MASK_ACTIVATION, m, n_pad, l, gp))
+
+    def bufs():
+        return (torch.empty(l, n_pad, dtype=torch.int32, device="cuda"),
+                torch.empty(l, m, dtype=torch.int32, device="cuda"))
+
+    want = {}
+    for pid in (40, 41, 42):
+        U, K = bufs()
+        M.mosaic_mask_activation(gp, proto.key, pid, m, n_pad, l, ch.C, layer.J, U, K, proto.variant, ws)
+        want[pid] = (host_u32(U), host_u32(K))
+    if layer.cj_planes is not None:
+        U, K = bufs()
+        M.mosaic_mask_activation_planes(gp, proto.key, 40, m, n_pad, l, ch.C, layer.J, layer.cj_planes, U, K,
+                                        proto.variant, ws)
+        assert np.array_equal(host_u32(U), want[40][0]) and np.array_equal(host_u32(K), want[40][1])
+    ctr = torch.tensor([1], dtype=torch.int64, device="cuda")
+    U, K = bufs()
+    M.mosaic_mask_activation_ex(gp, proto.key, 40, ctr, m, n_pad, l, ch.C, layer.J, layer.cj_planes, U, K,
+                                proto.variant, ws)
+    assert np.array_equal(host_u32(U), want[41][0]) and np.array_equal(host_u32(K), want[41][1])
+    # graph: replay r draws pass 40 + r
+    ctr.zero_()
+    U, K = bufs()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        M.mosaic_mask_activation_ex(gp, proto.key, 40, ctr, m, n_pad, l, ch.C, layer.J, layer.cj_planes, U, K,
+                                    proto.variant, ws)
+        M.mosaic_advance_pass(ctr, 1)
+    torch.cuda.synchronize()
+    assert int(ctr.item()) == 0          # capturing ran nothing
+    for r in range(3):
+        g.replay()
+        torch.cuda.synchronize()
+        assert np.array_equal(host_u32(U), want[40 + r][0]) and np.array_equal(host_u32(K), want[40 + r][1])
+    assert int(ctr.item()) == 3
+    M.mosaic_device_status()
