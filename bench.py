@@ -485,7 +485,7 @@ def run_matvec_sweep(args, rank, world, torch, M, PR, proto, dev, stream, flush,
         n_pad = PR.pad_width(lin.n)
         ch = PR.Chains(proto, n_pad)
         W = torch.from_numpy(wl.weights(lin.m, lin.n)).to(dev)
-        layer = PR.SecureLinear(proto, W, 1, ch)
+        layer = PR.SecureLinear(proto, W, 1, ch, planes=False)   # one token: no digit planes
         del W
         X = torch.from_numpy(wl.activations(1, lin.n, seed=wl.SEED_X + rank)).to(dev)
         Sr = proto.sum_r

@@ -93,7 +93,7 @@ const char *mosaic_status_string(mosaic_status s);
 
 /* q_max for a rotation width n_pad (Sec. 4 straw-man paragraph: each entry of
  * W_hat X_hat is at most n q_max^2, and n q_max^2 <= 2^(kappa-1)).  Returns 0
- * if n_pad is not a power of two in [32, 32768] or qbits is outside [2, 16]. */
+ * if n_pad is not a power of two in [32, 65536] or qbits is outside [2, 16]. */
 int32_t mosaic_qmax(int64_t n_pad, uint32_t qbits);
 
 /* Writes the inversion table of the discrete Gaussian with parameter sigma
@@ -160,7 +160,9 @@ mosaic_status mosaic_prg_sparse(const mosaic_key *key, uint32_t tag, uint64_t st
  * D = I), transformed by butterflies (a, b) -> (a + b, a - b) in fp32 with
  * stages h = 1, 2, ..., n_pad / 2 in that order, then multiplied by
  * fl32(1 / sqrt(n_pad)).  y: rows x n_pad (leading dimension n_pad); y must
- * not overlap x.  n_pad a power of two in [32, 32768], 1 <= n <= n_pad.
+ * not overlap x.  n_pad a power of two in [32, 65536], 1 <= n <= n_pad
+ * (65536-wide rows run the first 15 stages on their halves, then the last
+ * stage and the scale in a second pass over y; same rounding).
  * x, y 16-byte aligned; ldx a multiple of 4. */
 mosaic_status mosaic_hadamard(const float *x, int64_t ldx, float *y, int64_t rows, int64_t n,
                               int64_t n_pad, const uint32_t *sign_words, void *stream);

@@ -71,7 +71,7 @@ int64_t off_r(const mosaic_params *p, uint32_t i) {
     return s;
 }
 uint32_t tag_of(uint32_t kind, uint32_t level) { return kind | (level << 8); }
-bool npad_ok(int64_t n_pad) { return is_pow2(n_pad) && n_pad >= 32 && n_pad <= 32768; }
+bool npad_ok(int64_t n_pad) { return is_pow2(n_pad) && n_pad >= 32 && n_pad <= 65536; }
 
 // Bytes of digit planes a tensor-core product of an M x K by N x K pair needs.
 size_t ws_gemm(int64_t M, int64_t N, int64_t K) {
@@ -367,7 +367,7 @@ mosaic_status mosaic_mask_chains(const mosaic_params *p, const mosaic_key *key, 
                                  size_t ws_bytes, void *stream) {
     MOSAIC_TRY(check_params(p));
     if (!key) return MOSAIC_ERR_ARG;
-    if (!is_pow2(n_pad) || n_pad > 32768 || n_pad < 32) return MOSAIC_ERR_SHAPE;
+    if (!npad_ok(n_pad)) return MOSAIC_ERR_SHAPE;
     if (!P || !C || !CT) return MOSAIC_ERR_ARG;
     if (ws_bytes < ws_chains(n_pad, p)) return MOSAIC_ERR_WORKSPACE;
     cudaStream_t st = as_stream(stream);

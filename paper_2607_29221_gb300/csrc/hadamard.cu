@@ -40,6 +40,8 @@ struct FwhtArgs {
     float *scale;
     uint16_t *planes;  // [4][rows][n_pad]
     int vec_x;         // x rows 16-byte aligned
+    int64_t ldy;       // mode 0: y row stride
+    int split;         // rows are the halves of rows twice as long (the 65536-wide path)
 };
 
 __device__ __forceinline__ int pad_idx(int i) { return i + (i >> 5); }
@@ -160,8 +162,11 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
 
     float v[E];
     if (active) {
-        const float *xr = a.x + row * a.ldx;
-        if (E % 4 == 0 && a.vec_x && base + E <= a.n) {
+        // Split mode: row = 2 r + h is half h of the 2N-wide row r.
+        const int64_t half = a.split ? (row & 1) : 0;
+        const float *xr = a.split ? a.x + (row >> 1) * a.ldx + half * N : a.x + row * a.ldx;
+        const int64_t nrow = a.split ? (a.n - half * N < 0 ? 0 : (a.n - half * N < N ? a.n - half * N : N)) : a.n;
+        if (E % 4 == 0 && a.vec_x && base + E <= nrow) {
 #pragma unroll
             for (int q = 0; q < E; q += 4) {
                 float4 t = *reinterpret_cast<const float4 *>(xr + base + q);
@@ -169,7 +174,7 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
             }
         } else {
 #pragma unroll
-            for (int e = 0; e < E; e++) v[e] = (base + e < a.n) ? xr[base + e] : 0.0f;
+            for (int e = 0; e < E; e++) v[e] = (base + e < nrow) ? xr[base + e] : 0.0f;
         }
     } else {
 #pragma unroll
@@ -195,7 +200,7 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
 
     if (a.rotate) {
         if (a.signs) {
-            const uint32_t w = a.signs[base >> 5] >> (base & 31);
+            const uint32_t w = a.signs[(a.split ? (row & 1) * (N / 32) : 0) + (base >> 5)] >> (base & 31);
 #pragma unroll
             for (int e = 0; e < E; e++)
                 if ((w >> e) & 1u) v[e] = -v[e];
@@ -272,7 +277,7 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
 
     if (a.mode == 0) {
         if (active) {
-            float *yr = a.y + row * a.n_pad;
+            float *yr = a.split ? a.y + (row >> 1) * a.ldy + (row & 1) * N : a.y + row * a.ldy;
 #pragma unroll
             for (int run = 0; run < RUNS; run++) store_f32<CS>(yr + elem(run), v + run * CS);
         }
@@ -354,6 +359,114 @@ mosaic_status launch(const FwhtArgs &a, cudaStream_t st) {
     return launch_status();
 }
 
+// ---------------------------------------------------------------------------
+// Rows of 65536: the first 15 stages (h = 1 .. 16384) run on the two halves
+// as rows of 32768 (split mode, unscaled, into y or into `out` used as fp32
+// scratch); the last stage h = 32768 pairs the halves elementwise here, then
+// the scale 2^-8 = fl32(1 / sqrt(65536)) (exact), and for encode the row's
+// absmax (atomic max of |v| bits: finite values order like their bits, and a
+// non-finite value exceeds every finite one) and the quantisation.
+// ---------------------------------------------------------------------------
+constexpr int64_t kHalf = 32768;
+
+__global__ void combine_kernel(float *y, int64_t ldy, int64_t rows, int rotate, uint32_t *amax) {
+    const int64_t row = blockIdx.y;
+    const int64_t k = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+    float *lo = y + row * ldy + k, *hi = lo + kHalf;
+    float4 a = *reinterpret_cast<const float4 *>(lo), b = *reinterpret_cast<const float4 *>(hi);
+    float va[4] = {a.x, a.y, a.z, a.w}, vb[4] = {b.x, b.y, b.z, b.w};
+    uint32_t m = 0u;
+#pragma unroll
+    for (int q = 0; q < 4; q++) {
+        if (rotate) {
+            const float p = va[q], r = vb[q];
+            va[q] = __fmul_rn(__fadd_rn(p, r), 0.00390625f);
+            vb[q] = __fmul_rn(__fsub_rn(p, r), 0.00390625f);
+        }
+        m = max(m, max(__float_as_uint(va[q]) & 0x7fffffffu, __float_as_uint(vb[q]) & 0x7fffffffu));
+    }
+    if (rotate) {
+        *reinterpret_cast<float4 *>(lo) = make_float4(va[0], va[1], va[2], va[3]);
+        *reinterpret_cast<float4 *>(hi) = make_float4(vb[0], vb[1], vb[2], vb[3]);
+    }
+    if (amax) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
+        if ((threadIdx.x & 31) == 0) atomicMax(amax + row, m);
+    }
+}
+
+// scale[row] (holding the absmax bits) becomes s = absmax / qmax, or NaN for a
+// row with a non-finite value.
+__global__ void scale_kernel(float *scale, int64_t rows, int32_t qmax) {
+    const int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (row >= rows) return;
+    const uint32_t m = __float_as_uint(scale[row]);
+    scale[row] = m >= 0x7f800000u ? __int_as_float(0x7fc00000) : __fdiv_rn(__uint_as_float(m), (float)qmax);
+}
+
+__global__ void quantize_kernel(uint32_t *out, int64_t ldo, const float *scale, int32_t qmax,
+                                const uint32_t *mask, int64_t ldm, uint16_t *planes, int64_t rows) {
+    const int64_t row = blockIdx.y;
+    const int64_t k = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+    const float s = scale[row];
+    const bool quant = s == s && s != 0.0f;
+    uint32_t *o = out + row * ldo + k;
+    const uint4 bits = *reinterpret_cast<const uint4 *>(o);
+    const uint32_t in[4] = {bits.x, bits.y, bits.z, bits.w};
+    uint32_t code[4];
+#pragma unroll
+    for (int q = 0; q < 4; q++) {
+        const float t = __fadd_rn(__fdiv_rn(__uint_as_float(in[q]), s), 12582912.0f);
+        int32_t c = __float_as_int(t) - 0x4B400000;
+        c = min(max(c, -qmax), qmax);
+        code[q] = quant ? (uint32_t)c : 0u;
+    }
+    if (mask) {
+        const uint4 mk = *reinterpret_cast<const uint4 *>(mask + row * ldm + k);
+        code[0] += mk.x; code[1] += mk.y; code[2] += mk.z; code[3] += mk.w;
+    }
+    *reinterpret_cast<uint4 *>(o) = make_uint4(code[0], code[1], code[2], code[3]);
+    if (planes) store_planes<4>(planes + row * 65536 + k, rows * 65536, code);
+}
+
+mosaic_status fwht65536(FwhtArgs a, cudaStream_t st) {
+    const int64_t rows = a.rows;
+    // Pass 1: stages h = 1 .. 16384 on the halves, unscaled, fp32 into y (mode
+    // 0) or into `out` (mode 1).
+    FwhtArgs h = a;
+    h.split = 1;
+    h.rows = 2 * rows;
+    h.n_pad = kHalf;
+    h.mode = 0;
+    h.inv_sqrt = 1.0f;
+    if (a.mode == 1) {
+        h.y = reinterpret_cast<float *>(a.out);
+        h.ldy = a.ldo;
+    }
+    {
+        const mosaic_status rc = launch<32, 1024>(h, st);
+        if (rc != MOSAIC_OK) return rc;
+    }
+    float *y = h.y;
+    const int64_t ldy = h.ldy;
+    const dim3 grid((unsigned)(kHalf / (256 * 4)), (unsigned)rows);
+    if (rows > 65535) return MOSAIC_ERR_SHAPE;
+    if (a.mode == 0) {
+        combine_kernel<<<grid, 256, 0, st>>>(y, ldy, rows, a.rotate, nullptr);
+        return launch_status();
+    }
+    uint32_t *amax = reinterpret_cast<uint32_t *>(a.scale);
+    if (cudaMemsetAsync(amax, 0, sizeof(uint32_t) * (size_t)rows, st) != cudaSuccess) return MOSAIC_ERR_CUDA;
+    combine_kernel<<<grid, 256, 0, st>>>(y, ldy, rows, a.rotate, amax);
+    MOSAIC_TRY(launch_status());
+    scale_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(a.scale, rows, a.qmax);
+    MOSAIC_TRY(launch_status());
+    const dim3 g2((unsigned)(65536 / (256 * 4)), (unsigned)rows);
+    quantize_kernel<<<g2, 256, 0, st>>>(a.out, a.ldo, a.scale, a.qmax, a.mask, a.ldm, a.planes, rows);
+    return launch_status();
+}
+
 }  // namespace
 
 mosaic_status fwht_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, int64_t n_pad,
@@ -368,6 +481,9 @@ mosaic_status fwht_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, 
     a.y = y; a.qmax = qmax; a.mask = mask; a.ldm = ldm; a.out = out; a.ldo = ldo;
     a.scale = scale; a.planes = planes;
     a.vec_x = aligned16(x) && (ldx % 4 == 0);
+    a.ldy = n_pad;
+    a.split = 0;
+    if (n_pad == 65536) return fwht65536(a, st);
     switch (n_pad) {
         case 32: return launch<1, 32>(a, st);
         case 64: return launch<2, 32>(a, st);

@@ -128,9 +128,10 @@ WORKLOADS = {
         notes="decode sweep at 70B layer shape, pre-masked weights"),
     "matvec_sweep": Workload(
         "matvec_sweep", 1,
-        (Linear("n4096", 4096, 4096), Linear("n8192", 8192, 8192), Linear("n16384", 16384, 16384)),
-        notes="secure mat-vec n x n, one token (the paper's mat-vec figure; n = 36864 would "
-              "need a 65536-wide rotation, beyond this build's 32768)"),
+        (Linear("n4096", 4096, 4096), Linear("n8192", 8192, 8192), Linear("n16384", 16384, 16384),
+         Linear("n36864", 36864, 36864)),
+        notes="secure mat-vec n x n, one token (the paper's mat-vec figure; n = 36864 is "
+              "rotated at width 65536)"),
     "sigma_sweep_7b": Workload(
         "sigma_sweep_7b", 128,
         (Linear("attn", 4096, 4096), Linear("up", 14336, 4096), Linear("down", 4096, 14336)),

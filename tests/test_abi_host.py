@@ -49,9 +49,10 @@ def test_status_strings(lib):
 
 
 def test_qmax_matches_oracle(lib):
-    for k in range(5, 16):
+    for k in range(5, 17):
         assert M.mosaic_qmax(1 << k) == O.qmax_for(1 << k)
-    assert M.mosaic_qmax(1000) == 0 and M.mosaic_qmax(1 << 16) == 0
+    assert M.mosaic_qmax(1 << 16) == 181
+    assert M.mosaic_qmax(1000) == 0 and M.mosaic_qmax(1 << 17) == 0 and M.mosaic_qmax(16) == 0
 
 
 def test_gaussian_table_matches_oracle(lib):

@@ -95,14 +95,15 @@ def test_prg_sparse(rows, r, t):
 # --------------------------------------------------------------------------
 # Rotation and encoding
 # --------------------------------------------------------------------------
-NPADS = [32, 64, 128, 256, 512, 1024, 2048, 4096, 8192, 16384, 32768]
+NPADS = [32, 64, 128, 256, 512, 1024, 2048, 4096, 8192, 16384, 32768, 65536]
 
 
 @pytest.mark.parametrize("n_pad", NPADS)
 def test_hadamard_bit_exact(n_pad):
     M = M_()
     rows = 5 if n_pad >= 8192 else 19
-    for n in sorted({n_pad, max(1, n_pad - 3), n_pad // 2 + 1}):
+    # (n_pad // 2 - 3 leaves the upper half of a 65536 row empty)
+    for n in sorted({n_pad, max(1, n_pad - 3), n_pad // 2 + 1, max(1, n_pad // 2 - 3)}):
         x = wl.activations(rows, n, seed=n)
         words = O.sample_signs(KEY, 11, n_pad)
         y = torch.empty(rows, n_pad, dtype=torch.float32, device="cuda")
@@ -116,7 +117,7 @@ def test_hadamard_bit_exact(n_pad):
     assert np.array_equal(host_f32(y), O.fwht_rows(x[:, :n_pad], n_pad, None))
 
 
-@pytest.mark.parametrize("n_pad", [32, 256, 1024, 4096, 16384, 32768])
+@pytest.mark.parametrize("n_pad", [32, 256, 1024, 4096, 16384, 32768, 65536])
 def test_encode_bit_exact(n_pad):
     M = M_()
     rows = 6 if n_pad >= 16384 else 23
@@ -389,6 +390,15 @@ def test_cached_planes_match_uncached(l):
         outs.append((host_u32(mp.Ux), host_u32(mp.K), host_u32(Yhat), host_f32(Y)))
     for a, b in zip(*outs):
         assert np.array_equal(a, b)
+
+
+def test_layer_rotation_width_65536():
+    """n = 36900 rotates at width 65536 (halves, then the last stage apart):
+    every ring output bit-exact, one token and five tokens."""
+    for l in (1, 5):
+        g, ref, op, m, l_ = _run_layer(3, (96, 64, 40), (8, 4), m=40, n=36900, l=l,
+                                       variant=M_().GEMM_AUTO)
+        _check_layer(g, ref, op, m, l_)
 
 
 def test_layer_zero_noise_and_no_bias():
