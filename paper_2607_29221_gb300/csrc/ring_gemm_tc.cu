@@ -170,6 +170,14 @@ __global__ void __launch_bounds__(THREADS, 1)
         n0 = nchunks;
     }
     const int64_t n_units = n0 + n1;
+    // Shift groups 0 and 1 gather 1 and 2 digit products per K value, so they
+    // stay exact (|sum| <= 2^24) over two 256-wide chunks and are drained every
+    // second chunk of a tile (and at the end of the tile or of a segment);
+    // groups 2 and 3 are drained after every chunk.  `since` counts the chunks
+    // accumulated in groups 0 and 1, including the current one.
+    auto drains01 = [&](int64_t k, int c, int since) {
+        return since >= 2 || c == nchunks - 1 || k == n0 - 1 || k == n_units - 1;
+    };
     // Unit of this CTA's k-th step.
     auto unit_at = [&](int64_t k) -> int64_t {
         if (k >= n0) return s1b + (k - n0);
@@ -234,11 +242,14 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (lane == 0) {
             bool issued_any = false;
             int64_t slot = 0, chunk_count = 0;
+            int since01 = 0;
             for (int64_t k = 0; k < n_units && !*abort_flag; ++k) {
                 const int64_t u = unit_at(k);
                 const int64_t tile = u / nchunks;
                 const int c = (int)(u - tile * nchunks);
                 const int ks0 = c * CHUNK, ks1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
+                const uint32_t keep01 = since01 > 0 ? 1u : 0u;   // groups 0, 1 carry on
+                if (drains01(k, c, ++since01)) since01 = 0;
                 if (chunk_count > 0 && !mbar_wait(acc_empty, (uint32_t)(chunk_count - 1) & 1, abort_flag)) {
                     raise_abort(abort_flag);
                     break;
@@ -263,13 +274,14 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
                         const uint32_t z = (first && kk == 0) ? 0u : 1u;
+                        const uint32_t z01 = (first && kk == 0) ? keep01 : 1u;
                         const uint64_t a0 = sdesc_sw64(a_base + 0 * C::A_PLANE + kk * 32);
                         const uint64_t a1 = sdesc_sw64(a_base + 1 * C::A_PLANE + kk * 32);
                         const uint64_t a2 = sdesc_sw64(a_base + 2 * C::A_PLANE + kk * 32);
                         const uint64_t a3 = sdesc_sw64(a_base + 3 * C::A_PLANE + kk * 32);
                         const uint64_t b0 = sdesc_sw64(b_base + 0 * C::B_PLANE + kk * 32);
                         const uint64_t b2 = sdesc_sw64(b_base + 2 * C::B_PLANE + kk * 32);
-                        umma_bf16(tmem + 0 * BN, a0, b0, C::IDESC2, z);    // d0 e0, d0 e1
+                        umma_bf16(tmem + 0 * BN, a0, b0, C::IDESC2, z01);  // d0 e0, d0 e1
                         umma_bf16(tmem + 2 * BN, a0, b2, C::IDESC2, z);    // d0 e2, d0 e3
                         umma_bf16(tmem + 1 * BN, a1, b0, C::IDESC2, 1u);   // d1 e0, d1 e1
                         umma_bf16(tmem + 3 * BN, a1, b2, C::IDESC, 1u);    // d1 e2
@@ -303,6 +315,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int c = 0; c < HB; ++c) acc[c] = 0u;
         int64_t chunk_count = 0;
+        int since01 = 0;
         for (int64_t k = 0; k < n_units; ++k) {
             const int64_t u = unit_at(k);
             if (!mbar_wait(acc_full, (uint32_t)chunk_count & 1, abort_flag)) {
@@ -310,8 +323,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                 break;
             }
             tc_fence_after();
+            const bool d01 = drains01(k, (int)(u % nchunks), ++since01);
+            if (d01) since01 = 0;
 #pragma unroll
             for (int g = 0; g < 4; ++g) {
+                if (g < 2 && !d01) continue;
 #pragma unroll
                 for (int c0 = 0; c0 < HB; c0 += 32) {
                     uint32_t v[32];
