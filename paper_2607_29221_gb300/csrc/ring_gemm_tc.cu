@@ -332,9 +332,24 @@ __global__ void __launch_bounds__(THREADS, 1)
                 for (int c0 = 0; c0 < HB; c0 += 32) {
                     uint32_t v[32];
                     tmem_ld32(lane_addr + g * BN + c0, v);
+                    if (g == 3) {
+                        // Only the low 8 bits of group 3 survive the shift by 24, so it
+                        // is converted on the FMA pipe (the F2I unit serves the other
+                        // groups): with M = 1.5 * 2^23, q = (x / 256 + M) - M is an
+                        // integer, lo = x - 256 q is exact (|lo| <= 128), and the low
+                        // byte of the bits of lo + M is lo mod 256 (M's low byte is 0).
 #pragma unroll
-                    for (int c = 0; c < 32; ++c)
-                        acc[c0 + c] += ((uint32_t)__float2int_rn(__uint_as_float(v[c]))) << (8 * g);
+                        for (int c = 0; c < 32; ++c) {
+                            const float x = __uint_as_float(v[c]);
+                            const float q = __fsub_rn(__fmaf_rn(x, 0.00390625f, 12582912.0f), 12582912.0f);
+                            const float lo = __fmaf_rn(q, -256.0f, x);
+                            acc[c0 + c] += __float_as_uint(__fadd_rn(lo, 12582912.0f)) << 24;
+                        }
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 32; ++c)
+                            acc[c0 + c] += ((uint32_t)__float2int_rn(__uint_as_float(v[c]))) << (8 * g);
+                    }
                 }
             }
             tc_fence_before();
