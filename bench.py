@@ -75,7 +75,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="mine", choices=["mine", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(wl.WORKLOADS))
-    ap.add_argument("--variant", default="auto", choices=["auto", "tc", "imad"])
+    ap.add_argument("--variant", default="auto", choices=["auto", "tc", "mma_s8", "imad"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     return ap.parse_args()
@@ -257,7 +257,7 @@ def run_mine(args, rank, world):
     G.build()
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
-    variant = {"auto": M.GEMM_AUTO, "tc": M.GEMM_TC, "imad": M.GEMM_IMAD}[args.variant]
+    variant = {"auto": M.GEMM_AUTO, "tc": M.GEMM_TC, "mma_s8": M.GEMM_MMA_S8, "imad": M.GEMM_IMAD}[args.variant]
     if variant == M.GEMM_AUTO:
         variant = M.GEMM_TC if M.mosaic_gemm_variant_available(M.GEMM_TC) else M.GEMM_IMAD
     proto = PR.Protocol(wl.mask_key(), M.default_params(), variant=variant)
@@ -324,11 +324,12 @@ def run_mine(args, rank, world):
     tokens_s = world * l / (step_ms_max / 1e3)
     ring_tops = 2 * runner.ring_macs / (gemm_ms / 1e3) / 1e12
     roof = _roofline(variant, M, runner.ring_macs, gemm_ms, bf16, peak_src,
-                     _traffic("ring_gemm_tc") if args.workload == DEFAULT_WORKLOAD else None)
+                     _traffic("ring_gemm_tc") if args.workload == DEFAULT_WORKLOAD and variant == M.GEMM_TC
+                     else None)
     cfg = {"workload": args.workload, "l": l,
            "linears": [{"name": x.name, "m": x.m, "n": x.n} for x in wk.linears],
            "params": "Example 3.1: d=3, r=1536/1024/652, t=80/80, sigma=0.5, b=16",
-           "gemm_variant": {M.GEMM_TC: "tc", M.GEMM_IMAD: "imad"}[variant],
+           "gemm_variant": {M.GEMM_TC: "tc", M.GEMM_MMA_S8: "mma_s8", M.GEMM_IMAD: "imad"}[variant],
            "l2": "flushed between timed steps (256 MiB write)",
            "parallelism": f"replicas x{world}"}
     if args.workload == "decoder_70b_prefill_2048":
@@ -361,6 +362,13 @@ def _roofline(variant, M, ring_macs, gemm_ms, bf16, peak_src, traffic):
                 "frac": round(achieved / bf16, 4), "traffic": traffic,
                 "kernel": "ring_gemm_tc (10 bf16 digit-pair products per ring MAC)",
                 "peak_source": f"{peak_src} bf16 dense burst"}
+    if variant == M.GEMM_MMA_S8:
+        achieved = 10 * 2 * ring_macs / (gemm_ms / 1e3) / 1e12      # int8 digit-pair ops
+        peak = 2 * bf16                                            # nominal int8 : bf16 = 2 : 1
+        return {"bound": "tensor", "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TOPS",
+                "frac": round(achieved / peak, 4), "traffic": traffic,
+                "kernel": "ring_gemm_s8 (mma.sync m16n8k32, 10 int8 digit-pair products per ring MAC)",
+                "peak_source": f"{peak_src} bf16 dense burst x 2 (nominal int8 ratio)"}
     imad_peak = 152 * 64 * 2 * 2.07e9 / 1e12               # ring-ops/s: 64 IMAD/clk/SM, 2 ops each
     return {"bound": "alu", "achieved": round(ring_tops, 3), "peak": round(imad_peak, 2),
             "unit": "TOPS", "frac": round(ring_tops / imad_peak, 4), "traffic": None,

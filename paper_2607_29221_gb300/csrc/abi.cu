@@ -76,7 +76,9 @@ bool npad_ok(int64_t n_pad) { return is_pow2(n_pad) && n_pad >= 32 && n_pad <= 6
 // Bytes of digit planes a tensor-core product of an M x K by N x K pair needs.
 size_t ws_gemm(int64_t M, int64_t N, int64_t K) {
     const int64_t Kp = (K + 7) / 8 * 8;
-    return up(8 * (size_t)(M * Kp)) + up(8 * (size_t)(N * Kp));
+    const size_t bf16 = up(8 * (size_t)(M * Kp)) + up(8 * (size_t)(N * Kp));
+    const size_t s8 = ws_mma_s8(M, N, K);   // int8 digit planes of the legacy variant
+    return bf16 > s8 ? bf16 : s8;
 }
 
 // Ring product for the internal compositions (uint32 operands):
@@ -302,7 +304,7 @@ mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B
     if (variant == MOSAIC_GEMM_IMAD || (variant == MOSAIC_GEMM_AUTO && (!tc_available() || !tc_layout)))
         return ring_gemm_imad(A, lda, 1, B, ldb, 1, C, ldc, nullptr, 0, 1, M, N, K, st);
     if (variant == MOSAIC_GEMM_MMA_S8)
-        return ring_gemm_mma_s8(A, lda, B, ldb, C, ldc, nullptr, 0, 1, M, N, K, st);
+        return ring_gemm_mma_s8(A, lda, B, ldb, C, ldc, nullptr, 0, 1, M, N, K, ws, ws_bytes, st);
     if (!tc_available()) return MOSAIC_ERR_UNSUPPORTED;
     // A few tokens: the streaming kernel reads B once, no planes needed.
     if (skinny_ok(A, lda, B, ldb, M, K))

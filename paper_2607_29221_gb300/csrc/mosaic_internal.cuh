@@ -73,6 +73,14 @@ inline mosaic_status launch_status() {
 
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline bool is_pow2(int64_t v) { return v > 0 && (v & (v - 1)) == 0; }
+// Blocks for a grid-stride loop over `items`: enough to fill the GPU a few
+// times over, at most 152 x 32.
+inline int grid_for(int64_t items, int threads) {
+    int64_t g = (items + threads - 1) / threads;
+    if (g < 1) g = 1;
+    if (g > 152 * 32) g = 152 * 32;
+    return (int)g;
+}
 
 // ---- internal launchers (all enqueue on `st`, validate nothing beyond what they state) ----
 
@@ -124,10 +132,13 @@ mosaic_status ring_gemm_tc_planes2(const uint16_t *Ap, int64_t ldpa, int64_t a_p
                                    const uint32_t *Cin1, int64_t ldcin1, int64_t N1, uint32_t *C2, int64_t ldc2,
                                    const uint32_t *Cin2, int64_t ldcin2, int64_t N2, int64_t M, int64_t K,
                                    cudaStream_t st);
-// Legacy mma.sync s8 ring GEMM from int8 digits packed in uint32 operands (NT).
+// Legacy mma.sync s8 ring GEMM (NT, uint32 operands split into int8 digit
+// planes in ws, at least ws_mma_s8(M, N, K) bytes).
+size_t ws_mma_s8(int64_t M, int64_t N, int64_t K);
 mosaic_status ring_gemm_mma_s8(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb,
                                uint32_t *C, int64_t ldc, const uint32_t *Cin, int64_t ldcin,
-                               int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st);
+                               int sgn, int64_t M, int64_t N, int64_t K, void *ws, size_t ws_bytes,
+                               cudaStream_t st);
 bool tc_available();
 mosaic_status device_status(cudaStream_t st);
 bool mma_s8_available();

@@ -161,7 +161,8 @@ __global__ void __launch_bounds__(kSparseWarps * 32)
     }
 }
 
-int grid_for(int64_t items, int threads) {
+// Sampler grids: one thread per ChaCha block, up to 152 x 64 blocks.
+int prg_blocks(int64_t items, int threads) {
     int64_t g = (items + threads - 1) / threads;
     if (g < 1) g = 1;
     if (g > 152 * 64) g = 152 * 64;
@@ -195,7 +196,7 @@ mosaic_status prg_uniform(const Key &key, uint32_t tag, uint64_t sid, int rounds
     const int64_t total = rows * cols;
     if (total == 0) return MOSAIC_OK;
     const int64_t nblk = (total + 15) / 16;
-    uniform_kernel<<<grid_for(nblk, kThreads), kThreads, 0, st>>>(
+    uniform_kernel<<<prg_blocks(nblk, kThreads), kThreads, 0, st>>>(
         key, tag, sid, sid_dev, rounds, cols, total, out, ldo);
     return launch_status();
 }
@@ -211,7 +212,7 @@ mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int round
     tab.bound = gaussian_table_host(sigma, tab.t);
     tab.n = 2 * tab.bound + 1;
     const int64_t nblk = (count + 7) / 8;
-    gaussian_kernel<<<grid_for(nblk, kThreads), kThreads, 0, st>>>(
+    gaussian_kernel<<<prg_blocks(nblk, kThreads), kThreads, 0, st>>>(
         key, tag, sid, sid_dev, rounds, tab, count, out);
     return launch_status();
 }

@@ -514,7 +514,6 @@ bool tc_available() {
     return major == 10 && minor == 3 && encode_fn() != nullptr;
 }
 
-bool mma_s8_available() { return false; }
 
 mosaic_status ring_gemm_tc_planes(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const uint16_t *Bp,
                                   int64_t ldpb, int64_t b_plane, uint32_t *Cm, int64_t ldc,
@@ -546,10 +545,6 @@ mosaic_status ring_gemm_tc_planes2(const uint16_t *Ap, int64_t ldpa, int64_t a_p
     return launch_tc<128>(Ap, ldpa, a_plane, Bp, ldpb, b_plane, o1, o2, 1, M, K, st);
 }
 
-mosaic_status ring_gemm_mma_s8(const uint32_t *, int64_t, const uint32_t *, int64_t, uint32_t *, int64_t,
-                               const uint32_t *, int64_t, int, int64_t, int64_t, int64_t, cudaStream_t) {
-    return MOSAIC_ERR_UNSUPPORTED;
-}
 
 mosaic_status device_status(cudaStream_t st) {
     if (cudaStreamSynchronize(st) != cudaSuccess) return MOSAIC_ERR_CUDA;

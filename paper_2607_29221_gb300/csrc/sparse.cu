@@ -668,12 +668,6 @@ __global__ void digit_split_kernel(const uint32_t *a, int64_t lda, int64_t rows,
     }
 }
 
-int grid_for(int64_t items, int threads) {
-    int64_t g = (items + threads - 1) / threads;
-    if (g < 1) g = 1;
-    if (g > 152 * 32) g = 152 * 32;
-    return (int)g;
-}
 
 }  // namespace
 

@@ -169,8 +169,9 @@ class SecureLinear:
                                       self.n_pad, N * self.n_pad, Z, N, l, N, self.n_pad,
                                       M.GEMM_TC)
         else:
+            ws = self.proto.workspace(M.mosaic_workspace_bytes(M.OP_RING_GEMM, l, N, self.n_pad))
             M.mosaic_ring_gemm(Xp, self.n_pad, self.Wp, self.n_pad, Z, N, l, N, self.n_pad,
-                               self.proto.variant)
+                               self.proto.variant, ws)
         return Z
 
     def unmask(self, Z, mp: PassMask, s_x, Y=None, Yhat=None):

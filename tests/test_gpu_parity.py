@@ -269,6 +269,8 @@ def _variants():
     out = [M.GEMM_IMAD]
     if M.mosaic_gemm_variant_available(M.GEMM_TC):
         out.append(M.GEMM_TC)
+    if M.mosaic_gemm_variant_available(M.GEMM_MMA_S8):
+        out.append(M.GEMM_MMA_S8)
     return out
 
 

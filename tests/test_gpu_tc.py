@@ -196,3 +196,31 @@ def test_tc_whole_waves_then_stream_k(N):
     A = wl.uniform_u32(51, 512, 2048)
     B = wl.uniform_u32(52, N, 2048)
     assert np.array_equal(tc_gemm(A, B), ref(A, B))
+
+
+
+# --------------------------------------------------------------------------
+# Legacy mma.sync s8 variant (int8 digit planes, int32 accumulators)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Mm,N,K", [(1, 1, 1), (64, 64, 64), (65, 130, 33), (300, 129, 1000), (128, 257, 2049),
+                                    (17, 999, 4096)])
+def test_mma_s8_random(Mm, N, K):
+    M = _M()
+    if not M.mosaic_gemm_variant_available(M.GEMM_MMA_S8):
+        pytest.skip("mma.sync s8 variant not available")
+    A = wl.uniform_u32(61, Mm, K)
+    B = wl.uniform_u32(62, N, K)
+    assert np.array_equal(ring_gemm_u32(A, B, variant=M.GEMM_MMA_S8), ref(A, B))
+
+
+@pytest.mark.parametrize("va,vb", [(ALL_M128, ALL_M128), (ALL_P127, ALL_M128), (0xFFFFFFFF, 0x80000000)])
+def test_mma_s8_adversarial(va, vb):
+    """Constant digits over K = 5000: the int32 group sums wrap mod 2^32."""
+    M = _M()
+    if not M.mosaic_gemm_variant_available(M.GEMM_MMA_S8):
+        pytest.skip("mma.sync s8 variant not available")
+    Mm, N, K = 70, 90, 5000
+    A = np.full((Mm, K), va, np.uint32)
+    B = np.full((N, K), vb, np.uint32)
+    want = np.uint32((K * va * vb) % (1 << 32))
+    assert np.all(ring_gemm_u32(A, B, variant=M.GEMM_MMA_S8) == want)
