@@ -224,7 +224,8 @@ mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B
  * plane stride of rows_alloc * ldp elements, see mosaic_digit_split /
  * mosaic_encode).  A planes: M rows (plane stride a_plane), B planes: N rows
  * (plane stride b_plane); ldpa, ldpb leading dimensions in elements,
- * multiples of 8; 16-byte aligned.  Variant TC or MMA_S8. */
+ * multiples of 8; 16-byte aligned.  Variant TC (or AUTO); the bf16 planes
+ * feed only the tensor-core kernel (MOSAIC_ERR_UNSUPPORTED otherwise). */
 mosaic_status mosaic_ring_gemm_planes(const uint16_t *A_planes, int64_t ldpa, int64_t a_plane,
                                       const uint16_t *B_planes, int64_t ldpb, int64_t b_plane,
                                       uint32_t *C, int64_t ldc, int64_t M, int64_t N, int64_t K,
