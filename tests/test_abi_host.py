@@ -108,3 +108,32 @@ def test_validation_without_gpu(lib):
     k64 = M.default_params(kappa=64)
     assert _status("mosaic_unmask", ctypes.byref(k64), 1, 1, fake, 4000, fake, fake, fake, fake,
                    fake, fake, None, fake, None, 1, 3, None, 0, None) == 4
+
+
+def test_validation_of_newer_entry_points(lib):
+    """Argument checks of the check, variant and prepared-operand entry points,
+    all decided on the host before any device work."""
+    key = M.make_key(range(8))
+    p = M.default_params()
+    fake = 1 << 40
+    # Freivalds: k out of range, empty token batch
+    assert _status("mosaic_freivalds_check", 0, fake, fake, 8, 32, 4, fake, 8, fake, 32, fake, fake,
+                   None, 0, None) == 1
+    assert _status("mosaic_freivalds_check", 4, fake, fake, 8, 32, 0, fake, 8, fake, 32, fake, fake,
+                   None, 0, None) == 0
+    assert _status("mosaic_freivalds_setup", ctypes.byref(p), ctypes.byref(key), 1, 17, fake, 32, 8, 32,
+                   fake, fake, None) == 1
+    # act_nested must be 0 or 1
+    bad = M.default_params(act_nested=2)
+    assert _status("mosaic_mask_activation_ex", ctypes.byref(bad), ctypes.byref(key), 0, None, 8, 32, 4,
+                   fake, fake, None, fake, fake, 0, None, 0, None) == 1
+    # K above 2^20, rotation widths beyond 65536
+    assert _status("mosaic_ring_gemm", fake, 1 << 21, fake, 1 << 21, fake, 8, 8, 8, (1 << 20) + 1, 3,
+                   None, 0, None) == 2
+    assert _status("mosaic_hadamard", fake, 1 << 17, fake, 1, 1 << 17, 1 << 17, None, None) == 2
+    # prepared planes: empty shapes, missing counter
+    assert _status("mosaic_prepare_activation", ctypes.byref(p), 0, 64, fake, fake, fake, None) == 2
+    assert _status("mosaic_prepare_unmask", ctypes.byref(p), 0, fake, fake, None) == 2
+    assert _status("mosaic_advance_pass", None, 1, None) == 1
+    assert _status("mosaic_unmask_planes", ctypes.byref(p), 1, 8, fake, 3220, fake, fake, None, fake,
+                   fake, fake, fake, None, fake, None, 8, 3, None, 0, None) == 1
