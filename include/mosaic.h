@@ -343,7 +343,9 @@ mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const 
 mosaic_status mosaic_prepare_unmask(const mosaic_params *p, int64_t m, const uint32_t *L,
                                     uint16_t *L_planes, void *stream);
 
-/* mosaic_unmask with the planes of mosaic_prepare_unmask (same results). */
+/* mosaic_unmask with the planes of mosaic_prepare_unmask (same results).
+ * L_planes is required (MOSAIC_ERR_ARG when null, MOSAIC_ERR_ALIGN when not
+ * 16-byte aligned). */
 mosaic_status mosaic_unmask_planes(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z,
                                    int64_t ldz, const uint32_t *K_tm, const uint32_t *L,
                                    const uint16_t *L_planes, const uint32_t *S_idx,

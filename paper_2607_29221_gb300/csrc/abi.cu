@@ -655,7 +655,8 @@ mosaic_status mosaic_unmask_planes(const mosaic_params *p, int64_t l, int64_t m,
                                    const float *s_w, const float *s_x, const float *bias, float *Y,
                                    uint32_t *Yhat, int64_t ldy, int variant, void *ws, size_t ws_bytes,
                                    void *stream) {
-    if (!L_planes || !aligned16(L_planes)) return MOSAIC_ERR_ARG;
+    if (!L_planes) return MOSAIC_ERR_ARG;
+    if (!aligned16(L_planes)) return MOSAIC_ERR_ALIGN;
     return unmask_impl(p, l, m, Z, ldz, K_tm, L, L_planes, S_idx, S_val, s_w, s_x, bias, Y, Yhat, ldy, variant,
                        ws, ws_bytes, stream);
 }

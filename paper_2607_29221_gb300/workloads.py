@@ -80,7 +80,7 @@ def outlier_weights(m: int, n: int, seed: int = SEED_W, std: float = 0.02, chann
 def uniform_u32(seed: int, rows: int, cols: int) -> np.ndarray:
     """Uniform ring elements for ring-only tests (not part of the protocol's PRG)."""
     g = np.random.Generator(np.random.PCG64(seed))
-    return g.integers(0, 1 << 32, size=(rows, cols), dtype=np.uint64).astype(np.uint32)
+    return g.integers(0, 1 << 32, size=(rows, cols), dtype=np.uint32)
 
 
 @dataclass(frozen=True)

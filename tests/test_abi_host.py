@@ -137,3 +137,5 @@ def test_validation_of_newer_entry_points(lib):
     assert _status("mosaic_advance_pass", None, 1, None) == 1
     assert _status("mosaic_unmask_planes", ctypes.byref(p), 1, 8, fake, 3220, fake, fake, None, fake,
                    fake, fake, fake, None, fake, None, 8, 3, None, 0, None) == 1
+    assert _status("mosaic_unmask_planes", ctypes.byref(p), 1, 8, fake, 3220, fake, fake, fake + 2, fake,
+                   fake, fake, fake, None, fake, None, 8, 3, None, 0, None) == 3
