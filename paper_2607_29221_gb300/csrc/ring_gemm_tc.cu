@@ -119,7 +119,8 @@ __device__ __forceinline__ void umma_commit(uint64_t *bar) {
                      smem_u32(bar))
                  : "memory");
 }
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *v) {
+// 32 columns of TMEM for the warp's 32 lanes; the caller waits (tmem_wait).
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t *v) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
         "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
@@ -130,8 +131,8 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *v) {
           "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
           "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
         : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+__device__ __forceinline__ void tmem_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
 template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
@@ -178,11 +179,28 @@ __global__ void __launch_bounds__(THREADS, 1)
     auto drains01 = [&](int64_t k, int c, int since) {
         return since >= 2 || c == nchunks - 1 || k == n0 - 1 || k == n_units - 1;
     };
-    // Unit of this CTA's k-th step.
-    auto unit_at = [&](int64_t k) -> int64_t {
-        if (k >= n0) return s1b + (k - n0);
-        const int64_t w = k / nchunks;
-        return ((int64_t)blockIdx.x + w * (int64_t)gridDim.x) * nchunks + (k - w * nchunks);
+    // Walks this CTA's units in order without divisions: (tile, chunk c) of
+    // unit k (segment 0: tiles blockIdx.x + w * gridDim.x; segment 1: units
+    // s1b, s1b + 1, ...).
+    struct UnitWalk {
+        int64_t k, tile;
+        int c;
+    };
+    const int64_t s1_tile = s1b / nchunks;
+    const int s1_c = (int)(s1b - s1_tile * nchunks);
+    auto walk_init = [&](UnitWalk &w) {
+        w.k = 0;
+        w.tile = n0 > 0 ? (int64_t)blockIdx.x : s1_tile;
+        w.c = n0 > 0 ? 0 : s1_c;
+    };
+    auto walk_next = [&](UnitWalk &w) {
+        if (++w.k == n0) {
+            w.tile = s1_tile;
+            w.c = s1_c;
+        } else if (++w.c == nchunks) {
+            w.c = 0;
+            w.tile += w.k < n0 ? (int64_t)gridDim.x : 1;
+        }
     };
 
     if (threadIdx.x == 0) {
@@ -211,23 +229,31 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 0) {
         if (lane == 0) {
             int64_t slot = 0;
-            for (int64_t k = 0; k < n_units && !*abort_flag; ++k) {
-                const int64_t u = unit_at(k);
-                const int64_t tile = u / nchunks;
-                const int c = (int)(u - tile * nchunks);
-                const int m0 = (int)(tile % a.tiles_m) * BM, n0 = (int)(tile / a.tiles_m) * BN;
+            int s = 0;          // slot % STAGES
+            uint32_t ph = 0;    // parity of the empty phase awaited for slot s (from the second round on)
+            UnitWalk w;
+            walk_init(w);
+            for (; w.k < n_units && !*abort_flag; walk_next(w)) {
+                const int m0 = (int)(w.tile % a.tiles_m) * BM, n0 = (int)(w.tile / a.tiles_m) * BN;
+                const int c = w.c;
                 const int ks1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
+                bool ok = true;
                 for (int ks = c * CHUNK; ks < ks1; ++ks, ++slot) {
-                    const int s = (int)(slot % STAGES);
-                    if (slot >= STAGES && !mbar_wait(&empty[s], (uint32_t)((slot / STAGES) - 1) & 1, abort_flag)) {
+                    if (slot >= STAGES && !mbar_wait(&empty[s], ph, abort_flag)) {
                         raise_abort(abort_flag);
+                        ok = false;
                         break;
                     }
                     uint8_t *st = smem + s * C::STAGE;
                     mbar_expect_tx(&full[s], C::STAGE);
                     tma_load_3d(st, &tmA, &full[s], ks * BK, m0, 0);
                     tma_load_3d(st + C::A_BYTES, &tmB, &full[s], ks * BK, n0, 0);
+                    if (++s == STAGES) {
+                        s = 0;
+                        if (slot >= STAGES) ph ^= 1u;   // slots [STAGES, 2 STAGES) wait parity 0, and so on
+                    }
                 }
+                if (!ok) break;
             }
             if (*abort_flag) {
                 // Let the copies this thread started land before the CTA exits.
@@ -241,12 +267,18 @@ __global__ void __launch_bounds__(THREADS, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             bool issued_any = false;
-            int64_t slot = 0, chunk_count = 0;
+            int64_t chunk_count = 0;
+            int s = 0;          // shared-memory slot of the next stage
+            uint32_t ph = 0;    // parity of its full barrier
             int since01 = 0;
-            for (int64_t k = 0; k < n_units && !*abort_flag; ++k) {
-                const int64_t u = unit_at(k);
-                const int64_t tile = u / nchunks;
-                const int c = (int)(u - tile * nchunks);
+            // Descriptors differ only in the start-address field (address >> 4).
+            const uint64_t desc0 = sdesc_sw64(smem_u32(smem));
+            constexpr uint64_t AP = C::A_PLANE >> 4, BP = C::B_PLANE >> 4;
+            UnitWalk w;
+            walk_init(w);
+            for (; w.k < n_units && !*abort_flag; walk_next(w)) {
+                const int64_t k = w.k;
+                const int c = w.c;
                 const int ks0 = c * CHUNK, ks1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
                 const uint32_t keep01 = since01 > 0 ? 1u : 0u;   // groups 0, 1 carry on
                 if (drains01(k, c, ++since01)) since01 = 0;
@@ -255,16 +287,15 @@ __global__ void __launch_bounds__(THREADS, 1)
                     break;
                 }
                 bool ok = true;
-                for (int ks = ks0; ks < ks1; ++ks, ++slot) {
-                    const int s = (int)(slot % STAGES);
-                    if (!mbar_wait(&full[s], (uint32_t)(slot / STAGES) & 1, abort_flag)) {
+                for (int ks = ks0; ks < ks1; ++ks) {
+                    if (!mbar_wait(&full[s], ph, abort_flag)) {
                         raise_abort(abort_flag);
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a_base = smem_u32(smem + s * C::STAGE);
-                    const uint32_t b_base = a_base + C::A_BYTES;
+                    const uint64_t da = desc0 + (uint64_t)((s * C::STAGE) >> 4);
+                    const uint64_t db = da + (uint64_t)(C::A_BYTES >> 4);
                     const bool first = ks == ks0;
                     // The 10 digit products d_i e_j (i + j <= 3) as 6 MMAs: B planes
                     // j and j + 1 are adjacent in shared memory and the shift
@@ -275,21 +306,20 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int kk = 0; kk < BK / 16; ++kk) {
                         const uint32_t z = (first && kk == 0) ? 0u : 1u;
                         const uint32_t z01 = (first && kk == 0) ? keep01 : 1u;
-                        const uint64_t a0 = sdesc_sw64(a_base + 0 * C::A_PLANE + kk * 32);
-                        const uint64_t a1 = sdesc_sw64(a_base + 1 * C::A_PLANE + kk * 32);
-                        const uint64_t a2 = sdesc_sw64(a_base + 2 * C::A_PLANE + kk * 32);
-                        const uint64_t a3 = sdesc_sw64(a_base + 3 * C::A_PLANE + kk * 32);
-                        const uint64_t b0 = sdesc_sw64(b_base + 0 * C::B_PLANE + kk * 32);
-                        const uint64_t b2 = sdesc_sw64(b_base + 2 * C::B_PLANE + kk * 32);
-                        umma_bf16(tmem + 0 * BN, a0, b0, C::IDESC2, z01);  // d0 e0, d0 e1
-                        umma_bf16(tmem + 2 * BN, a0, b2, C::IDESC2, z);    // d0 e2, d0 e3
-                        umma_bf16(tmem + 1 * BN, a1, b0, C::IDESC2, 1u);   // d1 e0, d1 e1
-                        umma_bf16(tmem + 3 * BN, a1, b2, C::IDESC, 1u);    // d1 e2
-                        umma_bf16(tmem + 2 * BN, a2, b0, C::IDESC2, 1u);   // d2 e0, d2 e1
-                        umma_bf16(tmem + 3 * BN, a3, b0, C::IDESC, 1u);    // d3 e0
+                        const uint64_t a0 = da + 2 * kk, b0 = db + 2 * kk;
+                        umma_bf16(tmem + 0 * BN, a0, b0, C::IDESC2, z01);             // d0 e0, d0 e1
+                        umma_bf16(tmem + 2 * BN, a0, b0 + 2 * BP, C::IDESC2, z);      // d0 e2, d0 e3
+                        umma_bf16(tmem + 1 * BN, a0 + AP, b0, C::IDESC2, 1u);         // d1 e0, d1 e1
+                        umma_bf16(tmem + 3 * BN, a0 + AP, b0 + 2 * BP, C::IDESC, 1u); // d1 e2
+                        umma_bf16(tmem + 2 * BN, a0 + 2 * AP, b0, C::IDESC2, 1u);     // d2 e0, d2 e1
+                        umma_bf16(tmem + 3 * BN, a0 + 3 * AP, b0, C::IDESC, 1u);      // d3 e0
                     }
                     issued_any = true;
                     umma_commit(&empty[s]);
+                    if (++s == STAGES) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
                 }
                 if (!ok) break;
                 umma_commit(acc_full);
@@ -316,40 +346,46 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int c = 0; c < HB; ++c) acc[c] = 0u;
         int64_t chunk_count = 0;
         int since01 = 0;
-        for (int64_t k = 0; k < n_units; ++k) {
-            const int64_t u = unit_at(k);
+        UnitWalk wk;
+        walk_init(wk);
+        for (; wk.k < n_units; walk_next(wk)) {
+            const int64_t k = wk.k, tile = wk.tile;
+            const int c = wk.c;
             if (!mbar_wait(acc_full, (uint32_t)chunk_count & 1, abort_flag)) {
                 raise_abort(abort_flag);
                 break;
             }
             tc_fence_after();
-            const bool d01 = drains01(k, (int)(u % nchunks), ++since01);
+            const bool d01 = drains01(k, c, ++since01);
             if (d01) since01 = 0;
+            // Two groups are loaded before one wait.  Groups 0..2 convert on the
+            // F2I unit; only the low 8 bits of group 3 survive the shift by 24,
+            // so it is split on the FMA pipe instead, interleaved with group 2:
+            // with M = 1.5 * 2^23, q = (x / 256 + M) - M is an integer, lo = x -
+            // 256 q is exact (|lo| <= 128), and the low byte of the bits of
+            // lo + M is lo mod 256 (M's low byte is 0).
 #pragma unroll
-            for (int g = 0; g < 4; ++g) {
-                if (g < 2 && !d01) continue;
+            for (int c0 = 0; c0 < HB; c0 += 32) {
+                uint32_t v0[32], v1[32];
+                if (d01) {
+                    tmem_ld32_nowait(lane_addr + 0 * BN + c0, v0);
+                    tmem_ld32_nowait(lane_addr + 1 * BN + c0, v1);
+                    tmem_wait();
 #pragma unroll
-                for (int c0 = 0; c0 < HB; c0 += 32) {
-                    uint32_t v[32];
-                    tmem_ld32(lane_addr + g * BN + c0, v);
-                    if (g == 3) {
-                        // Only the low 8 bits of group 3 survive the shift by 24, so it
-                        // is converted on the FMA pipe (the F2I unit serves the other
-                        // groups): with M = 1.5 * 2^23, q = (x / 256 + M) - M is an
-                        // integer, lo = x - 256 q is exact (|lo| <= 128), and the low
-                        // byte of the bits of lo + M is lo mod 256 (M's low byte is 0).
+                    for (int cc = 0; cc < 32; ++cc)
+                        acc[c0 + cc] += (uint32_t)__float2int_rn(__uint_as_float(v0[cc])) +
+                                        ((uint32_t)__float2int_rn(__uint_as_float(v1[cc])) << 8);
+                }
+                tmem_ld32_nowait(lane_addr + 2 * BN + c0, v0);
+                tmem_ld32_nowait(lane_addr + 3 * BN + c0, v1);
+                tmem_wait();
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) {
-                            const float x = __uint_as_float(v[c]);
-                            const float q = __fsub_rn(__fmaf_rn(x, 0.00390625f, 12582912.0f), 12582912.0f);
-                            const float lo = __fmaf_rn(q, -256.0f, x);
-                            acc[c0 + c] += __float_as_uint(__fadd_rn(lo, 12582912.0f)) << 24;
-                        }
-                    } else {
-#pragma unroll
-                        for (int c = 0; c < 32; ++c)
-                            acc[c0 + c] += ((uint32_t)__float2int_rn(__uint_as_float(v[c]))) << (8 * g);
-                    }
+                for (int cc = 0; cc < 32; ++cc) {
+                    const float x = __uint_as_float(v1[cc]);
+                    const float q = __fsub_rn(__fmaf_rn(x, 0.00390625f, 12582912.0f), 12582912.0f);
+                    const float lo = __fmaf_rn(q, -256.0f, x);
+                    acc[c0 + cc] += ((uint32_t)__float2int_rn(__uint_as_float(v0[cc])) << 16) +
+                                    (__float_as_uint(__fadd_rn(lo, 12582912.0f)) << 24);
                 }
             }
             tc_fence_before();
@@ -357,8 +393,6 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (lane == 0) mbar_arrive(acc_empty);
             ++chunk_count;
 
-            const int64_t tile = u / nchunks;
-            const int c = (int)(u - tile * nchunks);
             if (c != nchunks - 1 && k != n0 - 1 && k != n_units - 1) continue;
             // End of this CTA's segment of the tile: write it out.
             const bool whole = k < n0 || ((s1b <= tile * nchunks) && (c == nchunks - 1));
