@@ -283,12 +283,17 @@ mosaic_status mosaic_mask_activation(const mosaic_params *p, const mosaic_key *k
                                      uint32_t *K_tm, int variant, void *ws, size_t ws_bytes,
                                      void *stream);
 
-/* Stationary operands of Init X as tensor-core digit planes, made once per
- * weight matrix (after mosaic_mask_weight) so that no pass re-splits them:
- * cj_planes = [4][n_pad + m][Kp] bf16 digits (Kp = r rounded up to a multiple
- * of 8, r = r_d, or r_1 with act_nested = 0): rows [0, n_pad) the C-factor
- * block (C_d, or C_1), rows [n_pad, n_pad + m) the J-factor block (J_d, or
- * J_1).  Size: mosaic_workspace_bytes(MOSAIC_OP_ACTIVATION_PLANES, m, n_pad, 0, p).
+/* Stationary operands of Init X, made once per weight matrix (after
+ * mosaic_mask_weight) so that no pass re-splits or re-stages them.  The
+ * buffer is opaque to the caller; it holds
+ *  - the tensor-core digit planes [4][n_pad + m][Kp] bf16 (Kp = r rounded up
+ *    to a multiple of 8, r = r_d, or r_1 with act_nested = 0): rows [0, n_pad)
+ *    the C-factor block (C_d, or C_1), rows [n_pad, n_pad + m) the J-factor
+ *    block (J_d, or J_1);
+ *  - for each LPN level i of a nested activation mask, the segments C_i and
+ *    J_i in the 32-row tile layout the sparse gathers stage with one bulk
+ *    copy per tile.
+ * Size: mosaic_workspace_bytes(MOSAIC_OP_ACTIVATION_PLANES, m, n_pad, 0, p).
  * 16-byte aligned device buffer. */
 mosaic_status mosaic_prepare_activation(const mosaic_params *p, int64_t m, int64_t n_pad,
                                         const uint32_t *C, const uint32_t *J, uint16_t *cj_planes,

@@ -140,8 +140,31 @@ size_t ws_activation(int64_t m, int64_t n_pad, int64_t l, const mosaic_params *p
     const size_t g = ws_gemm(l, n_pad + m, r_act(p));
     return ws_activation_min(l, p) + g;
 }
+// The activation planes buffer: digit planes of [C-factor; J-factor], then,
+// for each LPN level i of a nested activation mask, the tile images of the
+// segments C_i and J_i that the level's gathers stage (byte offsets; 0 where
+// a level has none).
+struct ActLayout {
+    size_t c_img[2], j_img[2];
+    size_t bytes;
+};
+ActLayout act_layout(int64_t m, int64_t n_pad, const mosaic_params *p) {
+    ActLayout L{{0, 0}, {0, 0}, 0};
+    size_t off = up(8 * (size_t)((n_pad + m) * kpad8(r_act(p))));
+    for (uint32_t i = 1; i <= act_levels(p); i++) {
+        const uint32_t ri = p->r[i - 1];
+        const size_t wc = tile_image_words(n_pad, ri), wj = tile_image_words(m, ri);
+        if (!wc || !wj) continue;
+        L.c_img[i - 1] = off;
+        off += up(4 * wc);
+        L.j_img[i - 1] = off;
+        off += up(4 * wj);
+    }
+    L.bytes = off;
+    return L;
+}
 size_t activation_planes_bytes(int64_t m, int64_t n_pad, const mosaic_params *p) {
-    return 8 * (size_t)((n_pad + m) * kpad8(r_act(p)));
+    return act_layout(m, n_pad, p).bytes;
 }
 size_t unmask_planes_bytes(int64_t m, const mosaic_params *p) {
     return 8 * (size_t)(m * kpad8(p->r[p->d - 1]));
@@ -149,8 +172,17 @@ size_t unmask_planes_bytes(int64_t m, const mosaic_params *p) {
 size_t ws_unmask_min(int64_t m, int64_t l, const mosaic_params *) {
     return up(sizeof(uint32_t) * (size_t)(l * m));
 }
+// Tile images of the Q_i segments of Z for the unmask gathers (tokens are the
+// staged rows); built per call when the workspace has room.
+size_t unmask_images_bytes(int64_t l, const mosaic_params *p) {
+    size_t s = 0;
+    if (l <= 4) return 0;   // a few tokens take the single-pass gather, which stages rows directly
+    for (uint32_t i = 1; i < p->d; i++) s += up(4 * tile_image_words(l, p->r[i - 1]));
+    return s;
+}
 size_t ws_unmask(int64_t m, int64_t l, const mosaic_params *p) {
-    return ws_unmask_min(m, l, p) + ws_gemm(l, m, p->r[p->d - 1]);
+    const size_t g = ws_gemm(l, m, p->r[p->d - 1]), im = unmask_images_bytes(l, p);
+    return ws_unmask_min(m, l, p) + (g > im ? g : im);
 }
 
 }  // namespace
@@ -342,8 +374,10 @@ mosaic_status mosaic_ring_gemm_planes(const uint16_t *A_planes, int64_t ldpa, in
 mosaic_status mosaic_device_status(void *stream) {
     const mosaic_status s = device_status(as_stream(stream));
     const mosaic_status s2 = skinny_status();
+    const mosaic_status s3 = gather_status();
     if (s != MOSAIC_OK) return s;
     if (s2 != MOSAIC_OK) return s2;
+    if (s3 != MOSAIC_OK) return s3;
     return cudaGetLastError() == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
 }
 
@@ -526,12 +560,19 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
                             n_pad, rd, st));
         MOSAIC_TRY(gemm_u32(variant, cv, Rt, rd, 1, J + od, Sr, 1, K_tm, m, nullptr, 0, 1, l, m, rd, st));
     }
-    if (d > 1)
+    // With prepared planes the gathers stage C_i and J_i from their tile images.
+    const ActLayout AL = act_layout(m, n_pad, p);
+    auto image = [&](size_t off) -> const uint32_t * {
+        return cj && off ? reinterpret_cast<const uint32_t *>(reinterpret_cast<const char *>(cj) + off) : nullptr;
+    };
+    if (d > 1) {
+        for (uint32_t i = 1; i < d; i++) lev[i - 1].tiled = image(AL.c_img[i - 1]);
         MOSAIC_TRY(sparse_gather(C, Sr, 0, od, n_pad, l, false, lev, (int)d - 1, Ux_tm, n_pad,
                                  nullptr, 0, 1, Ux_tm, n_pad, st));
-    if (d > 1)
+        for (uint32_t i = 1; i < d; i++) lev[i - 1].tiled = image(AL.j_img[i - 1]);
         MOSAIC_TRY(sparse_gather(J, Sr, 0, od, m, l, false, lev, (int)d - 1, K_tm, m, nullptr, 0, 1,
                                  K_tm, m, st));
+    }
     return MOSAIC_OK;
 }
 
@@ -585,7 +626,18 @@ mosaic_status mosaic_prepare_activation(const mosaic_params *p, int64_t m, int64
     const int64_t Kp = kpad8(rd), bplane = (n_pad + m) * Kp;
     cudaStream_t st = as_stream(stream);
     MOSAIC_TRY(digit_split(C + od, Sr, n_pad, rd, cj_planes, Kp, bplane, st));
-    return digit_split(J + od, Sr, m, rd, cj_planes + n_pad * Kp, Kp, bplane, st);
+    MOSAIC_TRY(digit_split(J + od, Sr, m, rd, cj_planes + n_pad * Kp, Kp, bplane, st));
+    const ActLayout L = act_layout(m, n_pad, p);
+    char *base = reinterpret_cast<char *>(cj_planes);
+    for (uint32_t i = 1; i <= act_levels(p); i++) {
+        if (!L.c_img[i - 1]) continue;
+        const uint32_t ri = p->r[i - 1];
+        MOSAIC_TRY(build_tile_image(C, Sr, off_r(p, i), ri, n_pad,
+                                    reinterpret_cast<uint32_t *>(base + L.c_img[i - 1]), st));
+        MOSAIC_TRY(build_tile_image(J, Sr, off_r(p, i), ri, m, reinterpret_cast<uint32_t *>(base + L.j_img[i - 1]),
+                                    st));
+    }
+    return MOSAIC_OK;
 }
 
 }  // extern "C"
@@ -630,6 +682,17 @@ mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const ui
         const uint32_t t = p->t[i], ri = p->r[i - 1];
         lev[i - 1] = SparseLevel{S_idx + soff, S_val + soff, (int)t, m + off_r(p, i), ri};
         soff += m * t;
+    }
+    // With room in the workspace (the product's planes are free again), the
+    // gathers stage Q_i from tile images made here in one pass over Z.
+    if (d > 1 && unmask_images_bytes(l, p) && cv.used + unmask_images_bytes(l, p) <= cv.cap) {
+        for (uint32_t i = 1; i < d; i++) {
+            const uint32_t ri = p->r[i - 1];
+            if (!tile_image_words(l, ri)) continue;
+            uint32_t *img = cv.take<uint32_t>(tile_image_words(l, ri));
+            MOSAIC_TRY(build_tile_image(Z, ldz, m + off_r(p, i), ri, l, img, st));
+            lev[i - 1].tiled = img;
+        }
     }
     // Y_hat = Y' - tmp - sum_i S_{i+1} Q_i, then decode.
     return unmask_decode(Z, ldz, m, od, l, m, lev, (int)d - 1, tmp, m, s_w, s_x, bias, Y, Yhat, ldy,

@@ -172,7 +172,14 @@ struct SparseLevel {
     int t;
     int64_t off;           // offset of this level's segment (columns of src, or rows of P)
     uint32_t r;            // positions are < r; larger ones are skipped
+    const uint32_t *tiled = nullptr;   // tile images of src's segment (build_tile_image), or null
 };
+// Words of the tile images of a g_count x r segment (0 if the tiled gather
+// does not take r); the images are built by build_tile_image.
+size_t tile_image_words(int64_t g_count, uint32_t r);
+mosaic_status build_tile_image(const uint32_t *src, int64_t lds, int64_t col0, uint32_t r, int64_t g_count,
+                               uint32_t *img, cudaStream_t st);
+mosaic_status gather_status();
 mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, int64_t seg_len,
                             int64_t g_count, int64_t nlist, bool list_is_col, const SparseLevel *lev,
                             int nlev, const uint32_t *a, int64_t lda, const uint32_t *b, int64_t ldb,

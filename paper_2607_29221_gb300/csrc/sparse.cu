@@ -11,9 +11,14 @@
 // gathered word comes from shared memory.
 #include <cuda_bf16.h>
 
+#include "async_copy.cuh"
 #include "mosaic_internal.cuh"
 
 namespace mosaic {
+
+// Set when a tiled gather gave up waiting for its staging copy.
+__device__ uint32_t g_gather_error = 0;
+
 namespace {
 
 constexpr int kMaxLev = 2;
@@ -47,6 +52,7 @@ struct GatherArgs {
     float *Y;
     int64_t ldy;
     int trusted;   // positions known to be < r (drawn by this library)
+    const uint32_t *tiled;   // tile images of the level's segment (build_tile_image) or null
 };
 
 // Staged rows plus the per-warp list rings.
@@ -191,23 +197,33 @@ __global__ void __launch_bounds__(GW * 32) gather_kernel(GatherArgs a) {
 // Staging: a warp loads 4 rows x 32 positions (four 128-byte segments, one
 // 16-byte load a lane) and each of its four 4-byte stores hits 32 distinct
 // banks thanks to the permutation.
-// The (position, value) lists stream through a two-slot per-warp ring in
-// rounds of 16 pairs (cp.async, zero-filled past the end of a list).  Once a
-// round has landed, each lane rewrites two of its entity's positions into
-// line addresses with the permutation bits in place (clamping positions of
-// caller lists to r - 1), so that the gather loop needs one XOR per pair.
-// Work units are (tile, 64 entities), numbered tile-major and split evenly
-// over a persistent grid, so a CTA stages each of its one or two tiles once.
+// The (position, value) lists stream through a per-warp ring in rounds of
+// 16 pairs (cp.async one or two rounds ahead, zero-filled past the end of a
+// list).  Once a round has landed, each lane rewrites two of its entity's
+// positions into line addresses with the permutation bits in place (clamping
+// positions of caller lists to r - 1), so that the gather loop needs one XOR
+// per pair.  Work units are (tile, 64 entities), numbered tile-major and split
+// evenly over a persistent grid, so a CTA stages each of its one or two tiles
+// once; each unit's a - b operands are loaded when it starts and its outputs
+// written when its last round is done (16-byte accesses where the output rows
+// are the list entities and the layout allows).
 // ---------------------------------------------------------------------------
 constexpr int kPgRows = 32;
 constexpr int kPgWarps = 16;
 constexpr int kPgEnts = 4 * kPgWarps;       // entities per unit
 constexpr int kPgSlot = 4 * 36;             // words per ring slot: 4 entities x (16 idx + 16 val + 4 pad)
-constexpr int kPgRing = 2;
-constexpr uint32_t kPgMaxR = 1632;
+constexpr uint32_t kPgMaxR = 1568;          // stage + three-slot rings + barrier + alignment within 227 KB
 
-size_t pgather_smem(uint32_t r) {   // + 128 bytes to align the stage to a line
-    return (size_t)((r + 31) / 32 * 32) * kPgRows * 4 + (size_t)kPgWarps * kPgRing * kPgSlot * 4 + 128;
+// Ring slots per warp: three (lists two rounds ahead) where the outputs are
+// rows of the list entities; two where they are columns, whose scattered
+// a / b reads gain more from the L1 space left beside shared memory.
+template <bool LIST_IS_COL>
+__host__ __device__ constexpr int pg_ring() { return LIST_IS_COL ? 2 : 3; }
+
+// Stage, rings, the staging barrier and abort flag (16 bytes), + 128 bytes
+// to align the stage to a line.
+size_t pgather_smem(uint32_t r, int ring) {
+    return (size_t)((r + 31) / 32 * 32) * kPgRows * 4 + (size_t)kPgWarps * ring * kPgSlot * 4 + 16 + 128;
 }
 
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
@@ -226,40 +242,52 @@ constexpr int kPgStageBatch = 12;  // 16-byte loads a lane keeps in flight while
 
 template <bool LIST_IS_COL, bool CLAMP>
 __global__ void __launch_bounds__(kPgWarps * 32, 1)
-    pgather_kernel(GatherArgs a, int64_t units, int chunks, int vec_src) {
+    pgather_kernel(GatherArgs a, int units, int chunks, int vec_src, int vec_ab) {
+    constexpr int kPgRing = pg_ring<LIST_IS_COL>();
     extern __shared__ __align__(16) uint32_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int grp = lane >> 3, li = lane & 7;
     const int r = (int)a.r, rp = (r + 31) / 32 * 32, t = a.t;
     const uint32_t sm_base = ((uint32_t)__cvta_generic_to_shared(sm) + 127u) & ~127u;
     const uint32_t ring_base = sm_base + 4u * (uint32_t)(rp * kPgRows + warp * (kPgRing * kPgSlot));
-    const int64_t u_begin = units * blockIdx.x / gridDim.x;
-    const int64_t u_end = units * (blockIdx.x + 1) / gridDim.x;
+    // Staging barrier and abort flag after all rings.
+    uint64_t *bar = reinterpret_cast<uint64_t *>(reinterpret_cast<char *>(sm) + (sm_base - smem_u32(sm)) +
+                                                 4 * ((size_t)rp * kPgRows + (size_t)kPgWarps * kPgRing * kPgSlot));
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar + 1);
+    uint32_t bar_phase = 0;
+    if (a.tiled && threadIdx.x == 0) {
+        mbar_init(bar, 1);
+        *abort_flag = 0;
+        mbar_init_fence();
+    }
+    const int u_begin = (int)((int64_t)units * blockIdx.x / gridDim.x);
+    const int u_end = (int)((int64_t)units * (blockIdx.x + 1) / gridDim.x);
     const int R = (t + 15) >> 4;
-    const int64_t steps = (u_end - u_begin) * R;
+    const int steps = (u_end - u_begin) * R;
     const uint32_t rlast = a.r - 1;
     const uint32_t lane_chunk = 16u * (uint32_t)li;   // rows 4 li .. 4 li + 3 of a line, before permutation
 
-    // Prefetch cursor: the (round, entity chunk) of the next list round to copy.
-    int64_t i_step = 0;
-    int i_rr = 0, i_chunk = (int)(u_begin % chunks);
+    // List rounds: lane (grp, li) copies 16 bytes of round rr of entity
+    // (chunk, warp, grp): positions 4 li .. (li < 4) or values 4 (li - 4) ..
+    const uint32_t *lbase = li < 4 ? a.idx : a.val;
+    const int qoff = (li & 3) * 4;
+    const uint32_t st_off = 4u * (uint32_t)(grp * 36 + (li < 4 ? 0 : 16) + qoff);
+    int i_chunk = u_begin % chunks, i_rr = 0, i_s = 0;
     auto issue = [&]() {
-        if (i_step < steps) {
+        if (i_s < steps) {
             const int64_t e = (int64_t)i_chunk * kPgEnts + warp * 4 + grp;
-            const int part = li;   // 0..3: positions, 4..7: values
-            const int q = i_rr * 16 + (part & 3) * 4;
+            const int q = i_rr * 16 + qoff;
             const bool ok = e < a.nlist && q < t;
-            const uint32_t *src = (part < 4 ? a.idx : a.val) + (ok ? e * t + q : 0);
-            const uint32_t dst = ring_base + 4u * (uint32_t)((int)(i_step & 1) * kPgSlot + grp * 36 +
-                                                             (part < 4 ? 0 : 16) + (part & 3) * 4);
-            asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(ok ? 16 : 0)
+            const uint32_t dst = ring_base + 4u * (uint32_t)((i_s % kPgRing) * kPgSlot) + st_off;
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst),
+                         "l"(lbase + (ok ? e * t + q : 0)), "r"(ok ? 16 : 0)
                          : "memory");
             if (++i_rr == R) {
                 i_rr = 0;
                 if (++i_chunk == chunks) i_chunk = 0;
             }
         }
-        ++i_step;
+        ++i_s;
         asm volatile("cp.async.commit_group;" ::: "memory");
     };
 
@@ -268,6 +296,27 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
     // 4 j + gl and stores word p+k in line p+k, chunk j ^ (((p+k) >> 2) & 7):
     // for each k the 32 stores fall in 32 distinct banks.  Each lane keeps
     // kPgStageBatch 16-byte loads in flight.
+    // Tile images (a.tiled) hold exactly this layout: one bulk copy per 32 KB,
+    // all threads wait (bounded) for the barrier.  Returns false if the copy
+    // did not land in time (error word raised).
+    auto stage_tiled = [&](int64_t tile) -> bool {
+        const uint32_t bytes = (uint32_t)rp * 128u;
+        if (threadIdx.x == 0) {
+            // The previous tile's shared-memory reads happen before these async writes.
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_expect_tx(bar, bytes);
+            const char *src = reinterpret_cast<const char *>(a.tiled) + (size_t)tile * bytes;
+            for (uint32_t off = 0; off < bytes; off += 32768u)
+                bulk_load(sm_base + off, src + off, bytes - off < 32768u ? bytes - off : 32768u, bar);
+        }
+        const bool ok = mbar_wait(bar, bar_phase, abort_flag);
+        if (!ok) {
+            *abort_flag = 1;
+            atomicExch(&g_gather_error, 1u);
+        }
+        bar_phase ^= 1u;
+        return ok;
+    };
     auto stage = [&](int64_t tile) {
         const int64_t g0 = tile * kPgRows;
         const int gl = lane >> 3, pq = lane & 7;
@@ -311,93 +360,116 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
         }
     };
 
-    // The epilogue operands a - b of a unit's outputs are loaded when the unit
-    // starts, so that their latency hides behind the unit's rounds.
-    auto prefetch_ab = [&](int64_t tile, int64_t e, uint32_t (&ab)[4]) {
 #pragma unroll
-        for (int c = 0; c < 4; c++) {
-            const int64_t g = tile * kPgRows + li * 4 + c;
-            const int64_t row = LIST_IS_COL ? g : e;
-            const int64_t col = LIST_IS_COL ? e : g;
-            uint32_t v = 0u;
-            if (e < a.nlist && g < a.g_count) {
-                if (a.a) v += a.a[row * a.lda + col];
-                if (a.b) v -= a.b[row * a.ldb + col];
-            }
-            ab[c] = v;
-        }
-    };
-    auto finish = [&](int64_t tile, int64_t e, const uint32_t (&acc)[4], const uint32_t (&ab)[4]) {
-        if (e >= a.nlist) return;
-#pragma unroll
-        for (int c = 0; c < 4; c++) {
-            const int64_t g = tile * kPgRows + li * 4 + c;
-            if (g >= a.g_count) break;
-            const int64_t row = LIST_IS_COL ? g : e;
-            const int64_t col = LIST_IS_COL ? e : g;
-            const uint32_t res = (a.sgn >= 0 ? acc[c] : 0u - acc[c]) + ab[c];
-            if (a.out) a.out[row * a.ldo + col] = res;
-            if (a.decode) {
-                float y = __fmul_rn(__fmul_rn(__int2float_rn((int32_t)res), a.s_w[col]), a.s_x[row]);
-                if (a.bias) y = __fadd_rn(y, a.bias[col]);
-                a.Y[row * a.ldy + col] = y;
-            }
-        }
-    };
-
-    issue();
+    for (int j = 0; j < kPgRing - 1; j++) issue();
+    int s = 0;
     int64_t tile = u_begin / chunks;
-    int chunk = (int)(u_begin % chunks), rr = 0;
-    uint32_t acc[4] = {0u, 0u, 0u, 0u};
-    uint32_t ab[4] = {0u, 0u, 0u, 0u};
-    for (int64_t s = 0; s < steps; s++) {
-        if (rr == 0 && (s == 0 || chunk == 0)) {   // a new tile: the same step for every warp
+    int chunk = u_begin % chunks;
+    for (int u = u_begin; u < u_end; u++) {
+        if (u == u_begin || chunk == 0) {   // a new tile: the same unit for every warp
             __syncthreads();
-            stage(tile);
+            if (a.tiled) {
+                stage_tiled(tile);
+            } else {
+                stage(tile);
+            }
             __syncthreads();
-        }
-        if (rr == 0) prefetch_ab(tile, (int64_t)chunk * kPgEnts + warp * 4 + grp, ab);
-        issue();
-        asm volatile("cp.async.wait_group 1;" ::: "memory");
-        __syncwarp();
-        const uint32_t slot = ring_base + 4u * (uint32_t)((int)(s & 1) * kPgSlot + grp * 36);
-        {
-            // Positions 2 li, 2 li + 1 of the round -> line address | permutation bits.
-            uint32_t p0, p1;
-            asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(p0), "=r"(p1) : "r"(slot + 8u * li) : "memory");
-            if (CLAMP) {
-                p0 = min(p0, rlast);
-                p1 = min(p1, rlast);
+            if (a.tiled && *abort_flag) {
+                // Let this CTA's copy land (bounded) before leaving.
+                if (threadIdx.x == 0) mbar_drain(bar, bar_phase ^ 1u);
+                break;
             }
-            p0 = sm_base + (p0 << 7) + ((p0 << 2) & 0x70u);
-            p1 = sm_base + (p1 << 7) + ((p1 << 2) & 0x70u);
-            asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(slot + 8u * li), "r"(p0), "r"(p1) : "memory");
         }
-        __syncwarp();
+        const int64_t e = (int64_t)chunk * kPgEnts + warp * 4 + grp;
+        const int64_t g = tile * kPgRows + li * 4;
+        const bool e_ok = e < a.nlist;
+        // a - b of the unit's outputs: row e, columns g .. g+3 (or the transpose).
+        const bool vec = vec_ab && !LIST_IS_COL && g + 4 <= a.g_count;
+        uint32_t ab[4] = {0u, 0u, 0u, 0u};
+        if (e_ok) {
+            if (vec) {
+                if (a.a) {
+                    const uint4 x = __ldg(reinterpret_cast<const uint4 *>(a.a + e * a.lda + g));
+                    ab[0] = x.x; ab[1] = x.y; ab[2] = x.z; ab[3] = x.w;
+                }
+                if (a.b) {
+                    const uint4 x = __ldg(reinterpret_cast<const uint4 *>(a.b + e * a.ldb + g));
+                    ab[0] -= x.x; ab[1] -= x.y; ab[2] -= x.z; ab[3] -= x.w;
+                }
+            } else {
 #pragma unroll
-        for (int u4 = 0; u4 < 4; u4++) {
-            const uint4 I = lds128(slot + 16u * u4);
-            const uint4 V = lds128(slot + 64u + 16u * u4);
-            const uint32_t pi[4] = {I.x, I.y, I.z, I.w};
-            const uint32_t vi[4] = {V.x, V.y, V.z, V.w};
-#pragma unroll
-            for (int c = 0; c < 4; c++) {
-                const uint4 x = lds128(pi[c] ^ lane_chunk);
-                acc[0] += vi[c] * x.x;
-                acc[1] += vi[c] * x.y;
-                acc[2] += vi[c] * x.z;
-                acc[3] += vi[c] * x.w;
+                for (int c = 0; c < 4; c++) {
+                    if (g + c >= a.g_count) break;
+                    const int64_t row = LIST_IS_COL ? g + c : e;
+                    const int64_t col = LIST_IS_COL ? e : g + c;
+                    uint32_t v = 0u;
+                    if (a.a) v += a.a[row * a.lda + col];
+                    if (a.b) v -= a.b[row * a.ldb + col];
+                    ab[c] = v;
+                }
             }
         }
-        __syncwarp();
-        if (++rr == R) {
-            finish(tile, (int64_t)chunk * kPgEnts + warp * 4 + grp, acc, ab);
-            acc[0] = acc[1] = acc[2] = acc[3] = 0u;
-            rr = 0;
-            if (++chunk == chunks) {
-                chunk = 0;
-                ++tile;
+        uint32_t acc0 = 0u, acc1 = 0u, acc2 = 0u, acc3 = 0u;
+        for (int rr = 0; rr < R; rr++, s++) {
+            issue();
+            asm volatile("cp.async.wait_group %0;" ::"n"(kPgRing - 1) : "memory");
+            __syncwarp();
+            const uint32_t slot = ring_base + 4u * (uint32_t)((s % kPgRing) * kPgSlot + grp * 36);
+            {
+                // Positions 2 li, 2 li + 1 of the round -> line address | permutation bits.
+                uint32_t p0, p1;
+                asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(p0), "=r"(p1) : "r"(slot + 8u * li) : "memory");
+                if (CLAMP) {
+                    p0 = min(p0, rlast);
+                    p1 = min(p1, rlast);
+                }
+                p0 = sm_base + (p0 << 7) + ((p0 << 2) & 0x70u);
+                p1 = sm_base + (p1 << 7) + ((p1 << 2) & 0x70u);
+                asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(slot + 8u * li), "r"(p0), "r"(p1) : "memory");
             }
+            __syncwarp();
+#pragma unroll
+            for (int u4 = 0; u4 < 4; u4++) {
+                const uint4 I = lds128(slot + 16u * u4);
+                const uint4 V = lds128(slot + 64u + 16u * u4);
+                const uint32_t pi[4] = {I.x, I.y, I.z, I.w};
+                const uint32_t vi[4] = {V.x, V.y, V.z, V.w};
+#pragma unroll
+                for (int c = 0; c < 4; c++) {
+                    const uint4 x = lds128(pi[c] ^ lane_chunk);
+                    acc0 += vi[c] * x.x;
+                    acc1 += vi[c] * x.y;
+                    acc2 += vi[c] * x.z;
+                    acc3 += vi[c] * x.w;
+                }
+            }
+            __syncwarp();
+        }
+        if (e_ok) {
+            const uint32_t acc[4] = {acc0, acc1, acc2, acc3};
+            uint32_t res[4];
+#pragma unroll
+            for (int c = 0; c < 4; c++) res[c] = (a.sgn >= 0 ? acc[c] : 0u - acc[c]) + ab[c];
+            if (vec && a.out && !a.decode) {
+                *reinterpret_cast<uint4 *>(a.out + e * a.ldo + g) = make_uint4(res[0], res[1], res[2], res[3]);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 4; c++) {
+                    if (g + c >= a.g_count) break;
+                    const int64_t row = LIST_IS_COL ? g + c : e;
+                    const int64_t col = LIST_IS_COL ? e : g + c;
+                    if (a.out) a.out[row * a.ldo + col] = res[c];
+                    if (a.decode) {
+                        float y = __fmul_rn(__fmul_rn(__int2float_rn((int32_t)res[c]), a.s_w[col]), a.s_x[row]);
+                        if (a.bias) y = __fadd_rn(y, a.bias[col]);
+                        a.Y[row * a.ldy + col] = y;
+                    }
+                }
+            }
+        }
+        if (++chunk == chunks) {
+            chunk = 0;
+            ++tile;
         }
     }
     asm volatile("cp.async.wait_all;" ::: "memory");
@@ -405,7 +477,7 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
 
 template <bool LIST_IS_COL, bool CLAMP>
 mosaic_status launch_pgather(const GatherArgs &a, cudaStream_t st) {
-    const size_t smem = pgather_smem(a.r);
+    const size_t smem = pgather_smem(a.r, pg_ring<LIST_IS_COL>());
     auto kern = pgather_kernel<LIST_IS_COL, CLAMP>;
     static unsigned long long attr_set = 0;   // one bit per device ordinal
     int dev = 0, sms = 0, per_sm = 0;
@@ -426,9 +498,12 @@ mosaic_status launch_pgather(const GatherArgs &a, cudaStream_t st) {
     const int64_t units = tiles * chunks;
     const int64_t slots = (int64_t)sms * per_sm;
     const int64_t grid = units < slots ? units : slots;
-    if (chunks > 0x7fffffff) return MOSAIC_ERR_SHAPE;
+    if (units > 0x7fffffff) return MOSAIC_ERR_SHAPE;
     const int vec_src = aligned16(a.src) && a.lds % 4 == 0 && a.col0 % 4 == 0;
-    kern<<<(unsigned)grid, kPgWarps * 32, smem, st>>>(a, units, (int)chunks, vec_src);
+    // 16-byte a / b / out accesses (rows = list entities only).
+    const int vec_ab = (!a.a || (aligned16(a.a) && a.lda % 4 == 0)) && (!a.b || (aligned16(a.b) && a.ldb % 4 == 0)) &&
+                       (!a.out || (aligned16(a.out) && a.ldo % 4 == 0));
+    kern<<<(unsigned)grid, kPgWarps * 32, smem, st>>>(a, (int)units, (int)chunks, vec_src, vec_ab);
     return launch_status();
 }
 
@@ -566,8 +641,9 @@ mosaic_status gather_levels(GatherArgs base, bool list_is_col, const SparseLevel
         const bool first = L == 0, last = L == passes - 1;
         if (nlev > 0) {
             g.col0 = lev[L].off; g.r = lev[L].r; g.idx = lev[L].idx; g.val = lev[L].val; g.t = lev[L].t;
+            g.tiled = lev[L].tiled;
         } else {
-            g.col0 = 0; g.r = 0; g.idx = g.val = nullptr; g.t = 0;
+            g.col0 = 0; g.r = 0; g.idx = g.val = nullptr; g.t = 0; g.tiled = nullptr;
         }
         if (!first) {
             g.a = scratch_out; g.lda = ld_scratch; g.b = nullptr;
@@ -669,7 +745,58 @@ __global__ void digit_split_kernel(const uint32_t *a, int64_t lda, int64_t rows,
 }
 
 
+// Tile images for the tiled gather: image t holds rows 32 t .. 32 t + 31 of
+// the segment src[:, col0 .. col0 + r) exactly as pgather_kernel stages them
+// (line p = the 32 rows' words at position p, 16-byte chunk c holding rows
+// 4 (c ^ ((p >> 2) & 7)) .. + 3; zeros past the rows and positions), so that
+// a whole tile is one contiguous copy.  Block (p-block, tile): 32 positions.
+__global__ void tile_image_kernel(const uint32_t *src, int64_t lds, int64_t col0, int r, int64_t g_count, int rp,
+                                  uint32_t *img) {
+    __shared__ uint32_t t[32][33];
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8 threads
+    const int64_t tile = blockIdx.y;
+    const int p0 = blockIdx.x * 32;
+    for (int k = ty; k < 32; k += 8) {
+        const int64_t g = tile * 32 + k;
+        const int p = p0 + tx;
+        t[k][tx] = (g < g_count && p < r) ? src[g * lds + col0 + p] : 0u;
+    }
+    __syncthreads();
+    const int c = tx >> 2, w = tx & 3;
+    for (int k = ty; k < 32; k += 8) {
+        const int p = p0 + k;
+        const int g = ((c ^ ((p >> 2) & 7)) << 2) | w;
+        img[((size_t)tile * rp + p) * 32 + tx] = t[g][k];
+    }
+}
+
 }  // namespace
+
+size_t tile_image_words(int64_t g_count, uint32_t r) {
+    if (r < 1 || r > kPgMaxR || g_count < 1) return 0;
+    return (size_t)((g_count + kPgRows - 1) / kPgRows) * ((r + 31) / 32 * 32) * kPgRows;
+}
+
+mosaic_status build_tile_image(const uint32_t *src, int64_t lds, int64_t col0, uint32_t r, int64_t g_count,
+                               uint32_t *img, cudaStream_t st) {
+    if (!tile_image_words(g_count, r)) return MOSAIC_ERR_SHAPE;
+    const int rp = (int)((r + 31) / 32 * 32);
+    const int64_t tiles = (g_count + kPgRows - 1) / kPgRows;
+    if (tiles > 65535) return MOSAIC_ERR_SHAPE;
+    tile_image_kernel<<<dim3((unsigned)(rp / 32), (unsigned)tiles), 256, 0, st>>>(src, lds, col0, (int)r, g_count,
+                                                                                  rp, img);
+    return launch_status();
+}
+
+mosaic_status gather_status() {
+    uint32_t v = 0, zero = 0;
+    if (cudaMemcpyFromSymbol(&v, g_gather_error, sizeof v) != cudaSuccess) return MOSAIC_ERR_CUDA;
+    if (v) {
+        cudaMemcpyToSymbol(g_gather_error, &zero, sizeof zero);
+        return MOSAIC_ERR_TIMEOUT;
+    }
+    return MOSAIC_OK;
+}
 
 mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, int64_t seg_len,
                             int64_t g_count, int64_t nlist, bool list_is_col, const SparseLevel *lev,
