@@ -1,0 +1,79 @@
+"""A whole masked-linear step (Init X, encode + mask-add, server product,
+unmask + decode) captured as one CUDA graph, as the benchmark runs it: replay
+k draws pass base + k from the device counter, bit-identical in the server
+output Z and the decoded Y to the eager call with that pass id, and
+consecutive replays use different masks.  (Y itself differs slightly between
+passes: the LWE noise E_x of a pass does not cancel in the unmask.)"""
+import numpy as np
+import pytest
+
+from paper_2607_29221_gb300 import workloads as wl
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+KEY = wl.mask_key()
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2607_29221_gb300 import build
+    build.build()
+    from paper_2607_29221_gb300 import mosaic as M
+    M.lib()
+    yield
+
+
+def _bits(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy().view(np.uint32).copy()
+
+
+@pytest.mark.parametrize("l", [48, 8])
+def test_graph_step_matches_eager_passes(l):
+    from paper_2607_29221_gb300 import mosaic as M
+    from paper_2607_29221_gb300 import protocol as PR
+    gp = M.default_params(d=3, r=[96, 64, 40], t=[0, 8, 4])
+    proto = PR.Protocol(KEY, gp, variant=M.GEMM_AUTO)
+    m, n = 200, 256
+    ch = PR.Chains(proto, PR.pad_width(n))
+    layer = PR.SecureLinear(proto, torch.from_numpy(wl.weights(m, n, std=1.0)).cuda(), 3, ch)
+    N = m + proto.sum_r
+    X = torch.from_numpy(wl.activations(l, n)).cuda()
+    bufs = dict(Xp=torch.empty(l, layer.n_pad, dtype=torch.int32, device="cuda"),
+                s_x=torch.empty(l, dtype=torch.float32, device="cuda"),
+                Xpl=torch.empty(4, l, layer.n_pad, dtype=torch.int16, device="cuda"),
+                Z=torch.empty(l, N, dtype=torch.int32, device="cuda"),
+                Y=torch.empty(l, m, dtype=torch.float32, device="cuda"))
+
+    def step(mp):
+        layer.mask_input(X, mp, bufs["Xp"], bufs["s_x"], bufs["Xpl"])
+        layer.server(bufs["Xp"], bufs["Xpl"], bufs["Z"])
+        layer.unmask(bufs["Z"], mp, bufs["s_x"], bufs["Y"])
+
+    base = 5000
+    eager = []
+    for k in range(2):
+        step(layer.init_x(l, base + k))
+        eager.append((_bits(bufs["Z"]), _bits(bufs["Y"])))
+    ctr = torch.zeros(1, dtype=torch.int64, device="cuda")
+    gm = layer.init_x(l, base)
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        step(layer.init_x(l, base, pass_dev=ctr, out=gm))
+        M.mosaic_advance_pass(ctr, 1, stream=side)
+    torch.cuda.synchronize()
+    assert int(ctr.item()) == 0
+    for k in range(2):
+        g.replay()
+        Z, Y = _bits(bufs["Z"]), _bits(bufs["Y"])
+        assert np.array_equal(Z, eager[k][0]), k
+        assert np.array_equal(Y, eager[k][1]), k
+    assert int(ctr.item()) == 2
+    assert not np.array_equal(eager[0][0], eager[1][0])   # fresh masks per pass
+    M.mosaic_device_status()

@@ -305,11 +305,15 @@ def test_layer_one_token_example_params():
 
 
 @pytest.mark.parametrize("r,t", [((98, 70, 37), (8, 4)), ((96, 64, 40), (16, 12)),
-                                 ((1536, 1024, 652), (80, 80))])
+                                 ((1536, 1024, 652), (80, 80)), ((1568, 1544, 96), (12, 20)),
+                                 ((1600, 1560, 96), (12, 20))])
 def test_layer_tiled_gather_shapes(r, t):
     """Hamming weights that are multiples of 4 take the tiled gather: ragged
-    row tiles (m = 131, l = 67), segments that are not multiples of 32 and a
-    segment offset that is not 16-byte aligned (r_1 = 98)."""
+    row tiles (m = 131, l = 67), segments that are not multiples of 32, a
+    segment offset that is not 16-byte aligned (r_1 = 98), the longest
+    segment it stages (1568 words, from prepared tile images for Init X and
+    per-call images of Q for the unmask) and a longer one (1600) that falls
+    back to the row-staged gather."""
     for variant in _variants():
         g, ref, op, m, l = _run_layer(3, r, t, m=131, n=300, l=67, variant=variant)
         _check_layer(g, ref, op, m, l)
