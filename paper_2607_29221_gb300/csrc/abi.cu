@@ -520,31 +520,36 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
     Carve cv{static_cast<char *>(ws), ws_bytes, 0};
     uint32_t *Rt = cv.take<uint32_t>((size_t)(l * rd));
     if (!Rt) return MOSAIC_ERR_WORKSPACE;
-    MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_R, 0), pass_id, R, l, rd, Rt, rd, st, pass_dev));
     SparseLevel lev[2];
+    uint32_t tagT[2] = {0, 0}, rT[2] = {0, 0}, tT[2] = {0, 0};
+    uint32_t *ti[2] = {nullptr, nullptr}, *tv[2] = {nullptr, nullptr};
     for (uint32_t i = 1; i < d; i++) {
         const uint32_t t = p->t[i], ri = p->r[i - 1];
-        uint32_t *ti = cv.take<uint32_t>((size_t)(l * t));
-        uint32_t *tv = cv.take<uint32_t>((size_t)(l * t));
-        if (!ti || !tv) return MOSAIC_ERR_WORKSPACE;
-        MOSAIC_TRY(prg_sparse(k, tag_of(MOSAIC_TAG_T, i + 1), pass_id, R, l, ri, t, ti, tv, nullptr, st, pass_dev));
-        lev[i - 1] = SparseLevel{ti, tv, (int)t, off_r(p, i), ri};
+        ti[i - 1] = cv.take<uint32_t>((size_t)(l * t));
+        tv[i - 1] = cv.take<uint32_t>((size_t)(l * t));
+        if (!ti[i - 1] || !tv[i - 1]) return MOSAIC_ERR_WORKSPACE;
+        tagT[i - 1] = tag_of(MOSAIC_TAG_T, i + 1);
+        rT[i - 1] = ri;
+        tT[i - 1] = t;
+        lev[i - 1] = SparseLevel{ti[i - 1], tv[i - 1], (int)t, off_r(p, i), ri};
     }
     // U_x^T = E_x^T + R^T C_d^T + sum_i T_{i+1}^T C_i^T and
     // K^T = R^T J_d^T + sum_i T_{i+1}^T J_i^T: the two dense products share
     // R^T, so on the tensor cores they run as one product against the stacked
     // [C_d; J_d] (planes cached by mosaic_prepare_activation, or split here).
-    MOSAIC_TRY(prg_gaussian(k, tag_of(MOSAIC_TAG_EX, 0), pass_id, R, p->sigma, l * n_pad, Ux_tm, st, pass_dev));
     const bool want_tc = variant == MOSAIC_GEMM_TC || (variant == MOSAIC_GEMM_AUTO && tc_available());
     const int64_t Kp = kpad8(rd), bplane = (n_pad + m) * Kp;
     const size_t need = up(8 * (size_t)(l * Kp)) + (cj ? 0 : up(8 * (size_t)bplane));
     const bool skinny = skinny_ok(Rt, rd, C + od, Sr, l, rd) && skinny_ok(Rt, rd, J + od, Sr, l, rd);
     const bool fused = want_tc && !skinny && n_pad % 128 == 0 && Sr % 4 == 0 && aligned16(C + od) &&
                        aligned16(J + od) && cv.used + need <= cv.cap;
+    const size_t mark = cv.used;
+    uint16_t *Rp = fused ? cv.take<uint16_t>((size_t)(4 * l * Kp)) : nullptr;
+    // R (with its digit planes for the fused product), the T lists and E_x
+    // (into U_x) in one launch.
+    MOSAIC_TRY(prg_initx(k, R, pass_id, pass_dev, tag_of(MOSAIC_TAG_R, 0), l, rd, Rt, Rp, Kp, (int)d - 1, tagT, rT,
+                         tT, ti, tv, tag_of(MOSAIC_TAG_EX, 0), p->sigma, l * n_pad, Ux_tm, st));
     if (fused) {
-        const size_t mark = cv.used;
-        uint16_t *Rp = cv.take<uint16_t>((size_t)(4 * l * Kp));
-        MOSAIC_TRY(digit_split(Rt, rd, l, rd, Rp, Kp, l * Kp, st));
         const uint16_t *B = cj;
         if (!B) {
             uint16_t *Bw = cv.take<uint16_t>((size_t)(4 * bplane));

@@ -1,6 +1,7 @@
 // Internal declarations shared by the library's translation units.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -45,6 +46,13 @@ __device__ __forceinline__ void chacha_block(const Key &key, uint32_t ctr, uint3
     o[4] = x4 + key.k[0]; o[5] = x5 + key.k[1]; o[6] = x6 + key.k[2]; o[7] = x7 + key.k[3];
     o[8] = x8 + key.k[4]; o[9] = x9 + key.k[5]; o[10] = x10 + key.k[6]; o[11] = x11 + key.k[7];
     o[12] = x12 + ctr; o[13] = x13 + n0; o[14] = x14 + n1; o[15] = x15 + n2;
+}
+
+// Digit d of a as the bf16 bits of the signed value byte_d(a + 0x80808080) - 128
+// (a = sum_d digit_d 2^(8d) mod 2^32); the tensor-core operands' digit planes.
+__device__ __forceinline__ uint32_t digit_bits(uint32_t a, int d) {
+    const int dig = (int)(((a + 0x80808080u) >> (8 * d)) & 0xffu) - 128;
+    return __bfloat16_as_ushort(__float2bfloat16_rn((float)dig));
 }
 
 inline Key to_key(const mosaic_key *k) {
@@ -94,6 +102,13 @@ mosaic_status prg_uniform(const Key &key, uint32_t tag, uint64_t sid, int rounds
 mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int rounds, float sigma,
                            int64_t count, uint32_t *out, cudaStream_t st, const uint64_t *sid_dev = nullptr);
 // Sparse rows.
+// All draws of an Init X call in one launch: R (l x rd, and its digit planes
+// [4][l][Kp] when Rp is not null), nlev <= 2 sparse lists (l rows each) and
+// the Gaussian E (ecount samples), each exactly as the single samplers draw it.
+mosaic_status prg_initx(const Key &key, int rounds, uint64_t sid, const uint64_t *sid_dev, uint32_t tagR,
+                        int64_t l, int64_t rd, uint32_t *R, uint16_t *Rp, int64_t Kp, int nlev, const uint32_t *tagT,
+                        const uint32_t *rT, const uint32_t *tT, uint32_t *const *idx, uint32_t *const *val,
+                        uint32_t tagE, float sigma, int64_t ecount, uint32_t *E, cudaStream_t st);
 mosaic_status prg_sparse(const Key &key, uint32_t tag, uint64_t sid, int rounds, int64_t rows,
                          uint32_t r, uint32_t t, uint32_t *idx, uint32_t *val, uint32_t *fail,
                          cudaStream_t st, const uint64_t *sid_dev = nullptr);

@@ -708,10 +708,6 @@ __global__ void transpose_kernel(const uint32_t *a, int64_t lda, int64_t rows, i
     }
 }
 
-__device__ __forceinline__ uint32_t digit_bits(uint32_t a, int d) {
-    const int dig = (int)(((a + 0x80808080u) >> (8 * d)) & 0xffu) - 128;
-    return __bfloat16_as_ushort(__float2bfloat16_rn((float)dig));
-}
 
 // 4 consecutive elements per thread: one 16-byte load (when aligned and in
 // range) and one 8-byte store per plane; a ragged column tail goes element
