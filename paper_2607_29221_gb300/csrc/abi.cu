@@ -181,8 +181,7 @@ size_t unmask_images_bytes(int64_t l, const mosaic_params *p) {
     return s;
 }
 size_t ws_unmask(int64_t m, int64_t l, const mosaic_params *p) {
-    const size_t g = ws_gemm(l, m, p->r[p->d - 1]), im = unmask_images_bytes(l, p);
-    return ws_unmask_min(m, l, p) + (g > im ? g : im);
+    return ws_unmask_min(m, l, p) + ws_gemm(l, m, p->r[p->d - 1]) + unmask_images_bytes(l, p);
 }
 
 }  // namespace
@@ -671,16 +670,9 @@ mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const ui
     const uint32_t *Qd = Z + m + od;
     const bool want_tc = variant == MOSAIC_GEMM_TC || (variant == MOSAIC_GEMM_AUTO && tc_available());
     const int64_t Kp = kpad8(rd);
-    if (Lp && want_tc && !skinny_ok(Qd, ldz, L, rd, l, rd) && ldz % 4 == 0 && aligned16(Qd) &&
-        cv.used + up(8 * (size_t)(l * Kp)) <= cv.cap) {
-        const size_t mark = cv.used;
-        uint16_t *Qp = cv.take<uint16_t>((size_t)(4 * l * Kp));
-        MOSAIC_TRY(digit_split(Qd, ldz, l, rd, Qp, Kp, l * Kp, st));
-        MOSAIC_TRY(ring_gemm_tc_planes(Qp, Kp, l * Kp, Lp, Kp, m * Kp, tmp, m, K_tm, m, 1, l, m, rd, st));
-        cv.used = mark;
-    } else {
-        MOSAIC_TRY(gemm_u32(variant, cv, Qd, ldz, 1, L, rd, 1, tmp, m, K_tm, m, 1, l, m, rd, st));
-    }
+    const bool tc_planes = Lp && want_tc && !skinny_ok(Qd, ldz, L, rd, l, rd) && ldz % 4 == 0 && aligned16(Qd) &&
+                           cv.used + up(8 * (size_t)(l * Kp)) <= cv.cap;
+    uint16_t *Qp = tc_planes ? cv.take<uint16_t>((size_t)(4 * l * Kp)) : nullptr;
     SparseLevel lev[2];
     int64_t soff = 0;
     for (uint32_t i = 1; i < d; i++) {
@@ -688,16 +680,28 @@ mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const ui
         lev[i - 1] = SparseLevel{S_idx + soff, S_val + soff, (int)t, m + off_r(p, i), ri};
         soff += m * t;
     }
-    // With room in the workspace (the product's planes are free again), the
-    // gathers stage Q_i from tile images made here in one pass over Z.
+    // With room in the workspace, the gathers stage Q_i from tile images made
+    // here, in the same launch that splits Q_d into digit planes.
+    int nimg = 0;
+    int64_t icol[2];
+    uint32_t ir[2];
+    uint32_t *img[2];
     if (d > 1 && unmask_images_bytes(l, p) && cv.used + unmask_images_bytes(l, p) <= cv.cap) {
         for (uint32_t i = 1; i < d; i++) {
             const uint32_t ri = p->r[i - 1];
             if (!tile_image_words(l, ri)) continue;
-            uint32_t *img = cv.take<uint32_t>(tile_image_words(l, ri));
-            MOSAIC_TRY(build_tile_image(Z, ldz, m + off_r(p, i), ri, l, img, st));
-            lev[i - 1].tiled = img;
+            img[nimg] = cv.take<uint32_t>(tile_image_words(l, ri));
+            icol[nimg] = m + off_r(p, i);
+            ir[nimg] = ri;
+            lev[i - 1].tiled = img[nimg];
+            ++nimg;
         }
+    }
+    MOSAIC_TRY(unmask_prep(Z, ldz, l, m + od, rd, Qp, Kp, nimg, icol, ir, img, st));
+    if (Qp) {
+        MOSAIC_TRY(ring_gemm_tc_planes(Qp, Kp, l * Kp, Lp, Kp, m * Kp, tmp, m, K_tm, m, 1, l, m, rd, st));
+    } else {
+        MOSAIC_TRY(gemm_u32(variant, cv, Qd, ldz, 1, L, rd, 1, tmp, m, K_tm, m, 1, l, m, rd, st));
     }
     // Y_hat = Y' - tmp - sum_i S_{i+1} Q_i, then decode.
     return unmask_decode(Z, ldz, m, od, l, m, lev, (int)d - 1, tmp, m, s_w, s_x, bias, Y, Yhat, ldy,

@@ -195,6 +195,12 @@ size_t tile_image_words(int64_t g_count, uint32_t r);
 mosaic_status build_tile_image(const uint32_t *src, int64_t lds, int64_t col0, uint32_t r, int64_t g_count,
                                uint32_t *img, cudaStream_t st);
 mosaic_status gather_status();
+// Before an unmask, in one launch: digit planes [4][l][Kp] of Q_d = columns
+// [qcol, qcol + rd) of Z (when Qp is not null) and the tile images of nimg <= 2
+// segments Z[:, icol[k] .. + ir[k]) (tile_image_words(l, ir[k]) words each).
+mosaic_status unmask_prep(const uint32_t *Z, int64_t ldz, int64_t l, int64_t qcol, int64_t rd, uint16_t *Qp,
+                          int64_t Kp, int nimg, const int64_t *icol, const uint32_t *ir, uint32_t *const *img,
+                          cudaStream_t st);
 mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, int64_t seg_len,
                             int64_t g_count, int64_t nlist, bool list_is_col, const SparseLevel *lev,
                             int nlev, const uint32_t *a, int64_t lda, const uint32_t *b, int64_t ldb,

@@ -746,12 +746,10 @@ __global__ void digit_split_kernel(const uint32_t *a, int64_t lda, int64_t rows,
 // (line p = the 32 rows' words at position p, 16-byte chunk c holding rows
 // 4 (c ^ ((p >> 2) & 7)) .. + 3; zeros past the rows and positions), so that
 // a whole tile is one contiguous copy.  Block (p-block, tile): 32 positions.
-__global__ void tile_image_kernel(const uint32_t *src, int64_t lds, int64_t col0, int r, int64_t g_count, int rp,
-                                  uint32_t *img) {
-    __shared__ uint32_t t[32][33];
+__device__ __forceinline__ void tile_image_block(const uint32_t *src, int64_t lds, int64_t col0, int r,
+                                                 int64_t g_count, int rp, uint32_t *img, int64_t tile, int p0,
+                                                 uint32_t (&t)[32][33]) {
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8 threads
-    const int64_t tile = blockIdx.y;
-    const int p0 = blockIdx.x * 32;
     for (int k = ty; k < 32; k += 8) {
         const int64_t g = tile * 32 + k;
         const int p = p0 + tx;
@@ -763,6 +761,71 @@ __global__ void tile_image_kernel(const uint32_t *src, int64_t lds, int64_t col0
         const int p = p0 + k;
         const int g = ((c ^ ((p >> 2) & 7)) << 2) | w;
         img[((size_t)tile * rp + p) * 32 + tx] = t[g][k];
+    }
+}
+__global__ void tile_image_kernel(const uint32_t *src, int64_t lds, int64_t col0, int r, int64_t g_count, int rp,
+                                  uint32_t *img) {
+    __shared__ uint32_t t[32][33];
+    tile_image_block(src, lds, col0, r, g_count, rp, img, blockIdx.y, blockIdx.x * 32, t);
+}
+
+// Before an unmask: the digit planes of Q_d (the A operand of Q_d L^T) and
+// the tile images of the Q_i segments, in one launch of 256-thread blocks
+// (the first nb_split blocks split, then one block per (image, tile, 32
+// positions)).
+struct UnmaskPrep {
+    const uint32_t *Z;
+    int64_t ldz, l;
+    int64_t qcol, rd;          // Q_d = columns [qcol, qcol + rd)
+    uint16_t *Qp;              // [4][l][Kp] or null
+    int64_t Kp;
+    int vec;
+    int nb_split;
+    int nimg;
+    int64_t icol[2];
+    int ir[2], irp[2], iblocks[2];
+    uint32_t *img[2];
+};
+
+__device__ __forceinline__ void split4(const uint32_t *src, uint16_t *dst, int64_t plane_stride, int64_t c,
+                                       int64_t cols, int vec) {
+    if (vec && c + 4 <= cols) {
+        const uint4 x = *reinterpret_cast<const uint4 *>(src);
+#pragma unroll
+        for (int d = 0; d < 4; d++) {
+            uint2 o;
+            o.x = digit_bits(x.x, d) | (digit_bits(x.y, d) << 16);
+            o.y = digit_bits(x.z, d) | (digit_bits(x.w, d) << 16);
+            *reinterpret_cast<uint2 *>(dst + d * plane_stride) = o;
+        }
+    } else {
+        for (int q = 0; q < 4 && c + q < cols; q++) {
+            const uint32_t w = src[q];
+#pragma unroll
+            for (int d = 0; d < 4; d++) dst[d * plane_stride + q] = (uint16_t)digit_bits(w, d);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256) unmask_prep_kernel(UnmaskPrep a) {
+    __shared__ uint32_t t[32][33];
+    int b = blockIdx.x;
+    if (b < a.nb_split) {
+        const int64_t per_row = (a.rd + 3) / 4, total = a.l * per_row;
+        for (int64_t i = (int64_t)b * 256 + threadIdx.x; i < total; i += (int64_t)a.nb_split * 256) {
+            const int64_t r = i / per_row, c = (i - r * per_row) * 4;
+            split4(a.Z + r * a.ldz + a.qcol + c, a.Qp + r * a.Kp + c, a.l * a.Kp, c, a.rd, a.vec);
+        }
+        return;
+    }
+    b -= a.nb_split;
+    for (int k = 0; k < a.nimg; k++) {
+        if (b < a.iblocks[k]) {
+            const int pb = a.irp[k] / 32;
+            tile_image_block(a.Z, a.ldz, a.icol[k], a.ir[k], a.l, a.irp[k], a.img[k], b / pb, (b % pb) * 32, t);
+            return;
+        }
+        b -= a.iblocks[k];
     }
 }
 
@@ -781,6 +844,45 @@ mosaic_status build_tile_image(const uint32_t *src, int64_t lds, int64_t col0, u
     if (tiles > 65535) return MOSAIC_ERR_SHAPE;
     tile_image_kernel<<<dim3((unsigned)(rp / 32), (unsigned)tiles), 256, 0, st>>>(src, lds, col0, (int)r, g_count,
                                                                                   rp, img);
+    return launch_status();
+}
+
+mosaic_status unmask_prep(const uint32_t *Z, int64_t ldz, int64_t l, int64_t qcol, int64_t rd, uint16_t *Qp,
+                          int64_t Kp, int nimg, const int64_t *icol, const uint32_t *ir, uint32_t *const *img,
+                          cudaStream_t st) {
+    if (l == 0) return MOSAIC_OK;
+    if (nimg < 0 || nimg > 2) return MOSAIC_ERR_UNSUPPORTED;
+    UnmaskPrep a{};
+    a.Z = Z;
+    a.ldz = ldz;
+    a.l = l;
+    a.qcol = qcol;
+    a.rd = rd;
+    a.Qp = Qp;
+    a.Kp = Kp;
+    a.vec = (ldz % 4 == 0) && (qcol % 4 == 0) && (Kp % 4 == 0) && (reinterpret_cast<uintptr_t>(Z) & 15u) == 0 &&
+            (reinterpret_cast<uintptr_t>(Qp) & 7u) == 0;
+    int64_t grid = 0;
+    if (Qp && rd > 0) {
+        const int64_t items = l * ((rd + 3) / 4);
+        a.nb_split = (int)((items + 255) / 256 < 152 * 8 ? (items + 255) / 256 : 152 * 8);
+        grid += a.nb_split;
+    }
+    a.nimg = nimg;
+    for (int k = 0; k < nimg; k++) {
+        if (!tile_image_words(l, ir[k])) return MOSAIC_ERR_SHAPE;
+        a.icol[k] = icol[k];
+        a.ir[k] = (int)ir[k];
+        a.irp[k] = (int)((ir[k] + 31) / 32 * 32);
+        a.img[k] = img[k];
+        const int64_t blocks = ((l + kPgRows - 1) / kPgRows) * (a.irp[k] / 32);
+        if (blocks > 0x3fffffff) return MOSAIC_ERR_SHAPE;
+        a.iblocks[k] = (int)blocks;
+        grid += blocks;
+    }
+    if (grid == 0) return MOSAIC_OK;
+    if (grid > 0x7fffffff) return MOSAIC_ERR_SHAPE;
+    unmask_prep_kernel<<<(unsigned)grid, 256, 0, st>>>(a);
     return launch_status();
 }
 
