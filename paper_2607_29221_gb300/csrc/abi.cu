@@ -546,8 +546,14 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
     uint16_t *Rp = fused ? cv.take<uint16_t>((size_t)(4 * l * Kp)) : nullptr;
     // R (with its digit planes for the fused product), the T lists and E_x
     // (into U_x) in one launch.
+    // The T lists only feed the gathers: when the tiled gather takes every
+    // level, they are drawn as line offsets so that no pass rewrites them.
+    bool lines = d > 1;
+    for (uint32_t i = 1; i < d; i++)
+        lines = lines && pgather_takes(n_pad, rT[i - 1], (int)tT[i - 1]) && pgather_takes(m, rT[i - 1], (int)tT[i - 1]);
+    for (uint32_t i = 1; i < d; i++) lev[i - 1].lines = lines ? 1 : 0;
     MOSAIC_TRY(prg_initx(k, R, pass_id, pass_dev, tag_of(MOSAIC_TAG_R, 0), l, rd, Rt, Rp, Kp, (int)d - 1, tagT, rT,
-                         tT, ti, tv, tag_of(MOSAIC_TAG_EX, 0), p->sigma, l * n_pad, Ux_tm, st));
+                         tT, ti, tv, tag_of(MOSAIC_TAG_EX, 0), p->sigma, l * n_pad, Ux_tm, st, lines));
     if (fused) {
         const uint16_t *B = cj;
         if (!B) {

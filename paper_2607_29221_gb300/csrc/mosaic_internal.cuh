@@ -105,10 +105,11 @@ mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int round
 // All draws of an Init X call in one launch: R (l x rd, and its digit planes
 // [4][l][Kp] when Rp is not null), nlev <= 2 sparse lists (l rows each) and
 // the Gaussian E (ecount samples), each exactly as the single samplers draw it.
+// With `lines`, the lists hold pg_line(position) instead of the position.
 mosaic_status prg_initx(const Key &key, int rounds, uint64_t sid, const uint64_t *sid_dev, uint32_t tagR,
                         int64_t l, int64_t rd, uint32_t *R, uint16_t *Rp, int64_t Kp, int nlev, const uint32_t *tagT,
                         const uint32_t *rT, const uint32_t *tT, uint32_t *const *idx, uint32_t *const *val,
-                        uint32_t tagE, float sigma, int64_t ecount, uint32_t *E, cudaStream_t st);
+                        uint32_t tagE, float sigma, int64_t ecount, uint32_t *E, cudaStream_t st, bool lines = false);
 mosaic_status prg_sparse(const Key &key, uint32_t tag, uint64_t sid, int rounds, int64_t rows,
                          uint32_t r, uint32_t t, uint32_t *idx, uint32_t *val, uint32_t *fail,
                          cudaStream_t st, const uint64_t *sid_dev = nullptr);
@@ -188,7 +189,14 @@ struct SparseLevel {
     int64_t off;           // offset of this level's segment (columns of src, or rows of P)
     uint32_t r;            // positions are < r; larger ones are skipped
     const uint32_t *tiled = nullptr;   // tile images of src's segment (build_tile_image), or null
+    int lines = 0;                     // idx holds pg_line(position) (lists drawn for the tiled gather)
 };
+// Line offset of position p in a staged tile of the tiled gather: 128-byte
+// line p, the permutation bits ((p >> 2) & 7) in the 16-byte chunk field.
+__host__ __device__ __forceinline__ uint32_t pg_line(uint32_t p) { return (p << 7) + ((p << 2) & 0x70u); }
+// True when the tiled gather takes lists of weight t over segments of r words
+// staged in g_count rows (16-byte aligned lists assumed).
+bool pgather_takes(int64_t g_count, uint32_t r, int t);
 // Words of the tile images of a g_count x r segment (0 if the tiled gather
 // does not take r); the images are built by build_tile_image.
 size_t tile_image_words(int64_t g_count, uint32_t r);

@@ -130,7 +130,7 @@ constexpr int kSparseWarps = 4;
 // Row j of the sparse matrix by one warp; sm_warp = the warp's 512 + bitmap_words words.
 __device__ __forceinline__ void sparse_row(const Key &key, uint32_t tag, uint32_t sid_lo, uint32_t sid_hi,
                                            int rounds, int64_t j, uint32_t r, int t, uint32_t *idx, uint32_t *val,
-                                           uint32_t *fail, int bitmap_words, uint32_t *sm_warp) {
+                                           uint32_t *fail, int bitmap_words, uint32_t *sm_warp, bool lines = false) {
     const int lane = threadIdx.x & 31;
     uint32_t *words = sm_warp;
     uint32_t *bits = words + 512;
@@ -166,7 +166,7 @@ __device__ __forceinline__ void sparse_row(const Key &key, uint32_t tag, uint32_
                     val_start = last + 1;
                 }
                 if ((acc >> lane) & 1u) {
-                    ri[got + __popc(acc & lt_mask)] = p;
+                    ri[got + __popc(acc & lt_mask)] = lines ? pg_line(p) : p;
                     atomicOr(&bits[p >> 5], 1u << (p & 31));
                 }
                 got += __popc(acc);
@@ -231,6 +231,7 @@ struct InitxDraws {
     uint32_t *E;
     GaussTable tab;
     int nbU, nbS, nbG;   // blocks per role (nbS per sparse level)
+    int lines;           // lists hold pg_line(position)
 };
 constexpr int kDrawThreads = kSparseWarps * 32;
 
@@ -251,7 +252,7 @@ __global__ void __launch_bounds__(kDrawThreads) initx_draw_kernel(InitxDraws a) 
         const int64_t j = (int64_t)(blk - lv * a.nbS) * kSparseWarps + warp;
         if (j >= a.rowsT) return;
         sparse_row(a.key, a.tagT[lv], sid_lo, sid_hi, a.rounds, j, a.rT[lv], a.tT[lv], a.idx[lv], a.val[lv],
-                   nullptr, a.bitmap_words, sm + warp * (512 + a.bitmap_words));
+                   nullptr, a.bitmap_words, sm + warp * (512 + a.bitmap_words), a.lines != 0);
         return;
     }
     blk -= a.nlev * a.nbS;
@@ -322,7 +323,7 @@ mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int round
 mosaic_status prg_initx(const Key &key, int rounds, uint64_t sid, const uint64_t *sid_dev, uint32_t tagR,
                         int64_t l, int64_t rd, uint32_t *R, uint16_t *Rp, int64_t Kp, int nlev, const uint32_t *tagT,
                         const uint32_t *rT, const uint32_t *tT, uint32_t *const *idx, uint32_t *const *val,
-                        uint32_t tagE, float sigma, int64_t ecount, uint32_t *E, cudaStream_t st) {
+                        uint32_t tagE, float sigma, int64_t ecount, uint32_t *E, cudaStream_t st, bool lines) {
     if (l == 0) return MOSAIC_OK;
     if (nlev < 0 || nlev > 2) return MOSAIC_ERR_UNSUPPORTED;
     InitxDraws a{};
@@ -340,6 +341,7 @@ mosaic_status prg_initx(const Key &key, int rounds, uint64_t sid, const uint64_t
     a.pstride = l * Kp;
     a.nlev = nlev;
     a.rowsT = l;
+    a.lines = lines ? 1 : 0;
     uint32_t rmax = 1;
     for (int i = 0; i < nlev; i++) {
         a.tagT[i] = tagT[i];

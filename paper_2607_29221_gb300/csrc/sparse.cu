@@ -53,6 +53,7 @@ struct GatherArgs {
     int64_t ldy;
     int trusted;   // positions known to be < r (drawn by this library)
     const uint32_t *tiled;   // tile images of the level's segment (build_tile_image) or null
+    int lines;               // positions are already line offsets (p << 7 | chunk bits), see pg_line
 };
 
 // Staged rows plus the per-warp list rings.
@@ -415,19 +416,19 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
             asm volatile("cp.async.wait_group %0;" ::"n"(kPgRing - 1) : "memory");
             __syncwarp();
             const uint32_t slot = ring_base + 4u * (uint32_t)((s % kPgRing) * kPgSlot + grp * 36);
-            {
-                // Positions 2 li, 2 li + 1 of the round -> line address | permutation bits.
+            if (!a.lines) {
+                // Positions 2 li, 2 li + 1 of the round -> line offset | permutation bits.
                 uint32_t p0, p1;
                 asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(p0), "=r"(p1) : "r"(slot + 8u * li) : "memory");
                 if (CLAMP) {
                     p0 = min(p0, rlast);
                     p1 = min(p1, rlast);
                 }
-                p0 = sm_base + (p0 << 7) + ((p0 << 2) & 0x70u);
-                p1 = sm_base + (p1 << 7) + ((p1 << 2) & 0x70u);
+                p0 = pg_line(p0);
+                p1 = pg_line(p1);
                 asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(slot + 8u * li), "r"(p0), "r"(p1) : "memory");
+                __syncwarp();
             }
-            __syncwarp();
 #pragma unroll
             for (int u4 = 0; u4 < 4; u4++) {
                 const uint4 I = lds128(slot + 16u * u4);
@@ -436,7 +437,7 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
                 const uint32_t vi[4] = {V.x, V.y, V.z, V.w};
 #pragma unroll
                 for (int c = 0; c < 4; c++) {
-                    const uint4 x = lds128(pi[c] ^ lane_chunk);
+                    const uint4 x = lds128(sm_base + (pi[c] ^ lane_chunk));
                     acc0 += vi[c] * x.x;
                     acc1 += vi[c] * x.y;
                     acc2 += vi[c] * x.z;
@@ -609,11 +610,12 @@ template <bool LIST_IS_COL, bool CLAMP>
 mosaic_status dispatch_gather(GatherArgs a, cudaStream_t st) {
     // Up to 4 staged rows the lists dominate and one pass over them wins; from
     // about 8 rows on the tiled gather's line reads win despite its padding.
-    if (a.t > 0 && a.r >= 1 && a.g_count <= 4 && a.g_count * (int64_t)a.r <= 48 * 1024)
+    if (a.t > 0 && a.r >= 1 && a.g_count <= 4 && a.g_count * (int64_t)a.r <= 48 * 1024 && !a.lines)
         return launch_few<LIST_IS_COL, CLAMP>(a, st);
     const bool lists_vec = a.t > 0 && (a.t & 3) == 0 &&
                            ((reinterpret_cast<uintptr_t>(a.idx) | reinterpret_cast<uintptr_t>(a.val)) & 15u) == 0;
     if (lists_vec && a.r >= 1 && a.r <= kPgMaxR) return launch_pgather<LIST_IS_COL, CLAMP>(a, st);
+    if (a.lines) return MOSAIC_ERR_UNSUPPORTED;   // line-offset lists are for the tiled gather only
     a.segp = (int64_t)(a.r + 31) / 32 * 32 + 1;
     // The largest row tile with which two CTAs fit on an SM (one CTA stages
     // while the other gathers); else the largest that fits at all.
@@ -642,6 +644,7 @@ mosaic_status gather_levels(GatherArgs base, bool list_is_col, const SparseLevel
         if (nlev > 0) {
             g.col0 = lev[L].off; g.r = lev[L].r; g.idx = lev[L].idx; g.val = lev[L].val; g.t = lev[L].t;
             g.tiled = lev[L].tiled;
+            g.lines = lev[L].lines;
         } else {
             g.col0 = 0; g.r = 0; g.idx = g.val = nullptr; g.t = 0; g.tiled = nullptr;
         }
@@ -830,6 +833,10 @@ __global__ void __launch_bounds__(256) unmask_prep_kernel(UnmaskPrep a) {
 }
 
 }  // namespace
+
+bool pgather_takes(int64_t g_count, uint32_t r, int t) {
+    return t > 0 && (t & 3) == 0 && r >= 1 && r <= kPgMaxR && g_count > 4;
+}
 
 size_t tile_image_words(int64_t g_count, uint32_t r) {
     if (r < 1 || r > kPgMaxR || g_count < 1) return 0;
