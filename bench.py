@@ -707,9 +707,14 @@ def run_kernels_hbm(args, rank, world, torch, M, PR, proto, dev, stream, flush, 
     rows = []
     sampler = ClockSampler(_smi_index(dev.index))
     sampler.start()
+    # Two batches per width: the workload's, and 4x as many rows, where the
+    # fixed cost of a launch (a few us) no longer hides the streaming rate.
+    shapes = []
     for lin in wk.linears:
         n_pad = PR.pad_width(lin.n)
-        l = wk.l if n_pad <= 16384 else wk.l // 2
+        l0 = wk.l if n_pad <= 16384 else wk.l // 2
+        shapes += [(n_pad, l0), (n_pad, 4 * l0)]
+    for n_pad, l in shapes:
         x = torch.from_numpy(wl.activations(l, n_pad, seed=wl.SEED_X)).to(dev)
         y = torch.empty_like(x)
         mask = torch.randint(-2**31, 2**31 - 1, (l, n_pad), dtype=torch.int32, device=dev)
