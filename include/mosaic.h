@@ -45,7 +45,7 @@ typedef enum {
     MOSAIC_ERR_UNSUPPORTED = 4,  /* valid request this build does not implement      */
     MOSAIC_ERR_CUDA = 5,         /* a CUDA runtime call or launch failed             */
     MOSAIC_ERR_WORKSPACE = 6,    /* ws too small (see mosaic_workspace_bytes)        */
-    MOSAIC_ERR_TIMEOUT = 7       /* a bounded device wait expired (tensor GEMM)      */
+    MOSAIC_ERR_TIMEOUT = 7       /* a bounded device wait expired (read back by mosaic_device_status) */
 } mosaic_status;
 
 /* Protocol parameters (Example 3.1 defaults, lambda = 140).
@@ -358,10 +358,18 @@ mosaic_status mosaic_unmask_planes(const mosaic_params *p, int64_t l, int64_t m,
                                    const float *bias, float *Y, uint32_t *Yhat, int64_t ldy,
                                    int variant, void *ws, size_t ws_bytes, void *stream);
 
+/* Self-test of the timeout path: launches a kernel whose bounded wait on a
+ * barrier phase that nothing completes gives up after limit_us microseconds
+ * (1 .. 10^6) and raises a device error word, as a copy or product that
+ * never arrives would; the next mosaic_device_status returns
+ * MOSAIC_ERR_TIMEOUT (and clears the word).  No fault, no hang: the context
+ * stays usable. */
+mosaic_status mosaic_selftest_wait(int64_t limit_us, void *stream);
+
 /* Synchronises `stream` and reports device-side failures of earlier calls:
- * MOSAIC_ERR_TIMEOUT if a tensor-core product gave up a bounded wait (the
- * device error word is cleared by this call), MOSAIC_ERR_CUDA if a CUDA error
- * is pending, else MOSAIC_OK. */
+ * MOSAIC_ERR_TIMEOUT if a tensor-core product, a streaming product or a tiled
+ * gather gave up a bounded wait (the device error words are cleared by this
+ * call), MOSAIC_ERR_CUDA if a CUDA error is pending, else MOSAIC_OK. */
 mosaic_status mosaic_device_status(void *stream);
 
 /* mosaic_unmask for callers that cannot allocate device memory (the paper

@@ -370,6 +370,11 @@ mosaic_status mosaic_ring_gemm_planes(const uint16_t *A_planes, int64_t ldpa, in
                                1, M, N, K, as_stream(stream));
 }
 
+mosaic_status mosaic_selftest_wait(int64_t limit_us, void *stream) {
+    if (limit_us < 1 || limit_us > 1000000) return MOSAIC_ERR_ARG;
+    return wait_probe((unsigned long long)limit_us * 1000ull, as_stream(stream));
+}
+
 mosaic_status mosaic_device_status(void *stream) {
     const mosaic_status s = device_status(as_stream(stream));
     const mosaic_status s2 = skinny_status();

@@ -203,6 +203,9 @@ size_t tile_image_words(int64_t g_count, uint32_t r);
 mosaic_status build_tile_image(const uint32_t *src, int64_t lds, int64_t col0, uint32_t r, int64_t g_count,
                                uint32_t *img, cudaStream_t st);
 mosaic_status gather_status();
+// Launches a bounded wait that runs out after limit_ns (the self-test of the
+// timeout path: reported by the next device status as MOSAIC_ERR_TIMEOUT).
+mosaic_status wait_probe(unsigned long long limit_ns, cudaStream_t st);
 // Before an unmask, in one launch: digit planes [4][l][Kp] of Q_d = columns
 // [qcol, qcol + rd) of Z (when Qp is not null) and the tile images of nimg <= 2
 // segments Z[:, icol[k] .. + ir[k]) (tile_image_words(l, ir[k]) words each).

@@ -893,6 +893,26 @@ mosaic_status unmask_prep(const uint32_t *Z, int64_t ldz, int64_t l, int64_t qco
     return launch_status();
 }
 
+namespace {
+// Self-test of the bounded waits: one thread waits on a barrier phase that
+// nothing completes, gives up after limit_ns and raises the gather's error
+// word exactly as a staging copy that never lands would.
+__global__ void wait_probe_kernel(unsigned long long limit_ns) {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x != 0) return;
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    mbar_init_fence();
+    if (!mbar_wait(&bar, 0u, &abort_flag, limit_ns)) atomicExch(&g_gather_error, 1u);
+}
+}  // namespace
+
+mosaic_status wait_probe(unsigned long long limit_ns, cudaStream_t st) {
+    wait_probe_kernel<<<1, 32, 0, st>>>(limit_ns);
+    return launch_status();
+}
+
 mosaic_status gather_status() {
     uint32_t v = 0, zero = 0;
     if (cudaMemcpyFromSymbol(&v, g_gather_error, sizeof v) != cudaSuccess) return MOSAIC_ERR_CUDA;

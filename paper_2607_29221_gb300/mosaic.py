@@ -87,6 +87,7 @@ _SIGS = {
     "mosaic_prepare_unmask": ([_PP, _I64, _P, _P, _P], _INT),
     "mosaic_unmask_planes": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
                               _INT, _P, _SZ, _P], _INT),
+    "mosaic_selftest_wait": ([_I64, _P], _INT),
     "mosaic_freivalds_setup": ([_PP, _PK, _U64, _INT, _P, _I64, _I64, _I64, _P, _P, _P], _INT),
     "mosaic_freivalds_check": ([_INT, _P, _P, _I64, _I64, _I64, _P, _I64, _P, _I64, _P, _P, _P, _SZ,
                                 _P], _INT),
@@ -182,6 +183,12 @@ def mosaic_gemm_variant_available(variant: int) -> bool:
 
 def mosaic_device_status(stream=None):
     _call("mosaic_device_status", _stream(stream))
+
+
+def mosaic_selftest_wait(limit_us: int, stream=None):
+    """Launches a bounded wait that runs out after limit_us (the timeout path's
+    self-test); the next mosaic_device_status raises MOSAIC_ERR_TIMEOUT."""
+    _call("mosaic_selftest_wait", limit_us, _stream(stream))
 
 
 def mosaic_workspace_bytes(op: int, m: int, n_pad: int, l: int, params: mosaic_params = None) -> int:

@@ -139,3 +139,8 @@ def test_validation_of_newer_entry_points(lib):
                    fake, fake, fake, None, fake, None, 8, 3, None, 0, None) == 1
     assert _status("mosaic_unmask_planes", ctypes.byref(p), 1, 8, fake, 3220, fake, fake, fake + 2, fake,
                    fake, fake, fake, None, fake, None, 8, 3, None, 0, None) == 3
+
+
+def test_selftest_wait_validates_its_limit(lib):
+    assert _status("mosaic_selftest_wait", 0, None) == 1
+    assert _status("mosaic_selftest_wait", 1000001, None) == 1

@@ -132,3 +132,22 @@ def test_largest_contraction_is_exact(Mm, N, adversarial):
         _gemm(dA, dB, C, Mm, N, K, v)
         assert np.array_equal(host(C), ref), v
     _M().mosaic_device_status()
+
+
+def test_bounded_wait_expiry_is_reported_and_the_context_survives():
+    """A bounded device wait on a barrier that nothing completes runs out after
+    2 ms; the next device status reports the timeout (and clears it), and the
+    context keeps working (a product afterwards is still exact)."""
+    M = _M()
+    M.mosaic_device_status()
+    M.mosaic_selftest_wait(2000)
+    with pytest.raises(M.MosaicError) as ei:
+        M.mosaic_device_status()
+    assert ei.value.status == 7
+    M.mosaic_device_status()          # cleared
+    A = wl.uniform_u32(81, 5, 33)
+    B = wl.uniform_u32(82, 7, 33)
+    C = sentinel(5, 7)
+    _gemm(dev(A), dev(B), C, 5, 7, 33, M.GEMM_AUTO)
+    assert np.array_equal(host(C), O.matmul(A, B.T.copy()))
+    M.mosaic_device_status()
