@@ -14,15 +14,16 @@
 //     two digits is at most 2^14 in magnitude, so a group that has summed at
 //     most 1024 products is still an exact integer (|sum| <= 2^24).  Every
 //     CHUNK * BK = 256 values of K (group 3 then holds 1024 products) the
-//     epilogue warps drain all four groups to int32 registers:
-//     acc += (int32)g_s << 8s, with 32-bit wraparound, which is exact mod 2^32.
+//     epilogue warps drain groups 2 and 3, every 512 values of K groups 0 and
+//     1, into int32 registers: acc += g_s << 8s mod 2^32 (drain_01 and
+//     drain_23 below convert the fp32 sums exactly).
 //
 // Pipeline (128 x BN output tiles, 10 warps):
 //   warp 0      TMA producer: per stage one 3-D box {32 K, rows, 4 planes}
 //               for A and one for B (64-byte swizzle), mbarrier complete_tx
 //   warp 1      TMEM allocation (512 columns) and the single-thread MMA issuer
 //               (12 tcgen05.mma per stage: 8 of 128 x 2BN x 16, 4 of 128 x BN x 16)
-//   warps 2..9  epilogue: tcgen05.ld 32x32b, fp32 -> int32, shift-add (each lane
+//   warps 2..9  epilogue: tcgen05.ld 32x32b, exact fp32 -> int32, shift-add (each lane
 //               quarter of TMEM twice, half of the columns each)
 // Every wait is bounded (about 2 s of %globaltimer); on expiry the kernel
 // raises a device error word, stops issuing work, waits (bounded) for its
@@ -46,6 +47,42 @@ constexpr int CHUNK = 8;        // stages between drains: 256 K
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int THREADS = 320;   // warp 0 TMA, warp 1 MMA, warps 2..9 epilogue
 constexpr int EPI_WARPS = 8;
+
+// Drain conversions.  The fp32 group sums are integers with |x| <= 2^24 and
+// the F2I unit converts 16 values per clock per SM while the tensor pipe
+// idles, so each pair of groups is folded into ONE exact fp32 value first
+// (FMA pipe).  kM = 1.5 * 2^23: for an integer y with |y| <= 2^22 the bits of
+// y + kM are bits(kM) + y, so fma(x, 2^-8, kM) - kM is h = round(x / 2^8)
+// exactly and fma(h, -2^8, x) = x - 2^8 h is exact (|x - 2^8 h| <= 2^7).
+constexpr float kM = 12582912.0f;
+
+// Groups 0 and 1 (|x0| <= 2^23, |x1| <= 2^24 after 512 K): with h =
+// round(x1 / 2^8), x0 + 2^8 x1 = s + 2^16 h where s = x0 + 2^8 (x1 - 2^8 h)
+// is exact (|s| < 2^24) and goes through F2I; h << 16 is the bits of
+// x1 / 2^8 + kM shifted by 16, since bits(kM) << 16 = 0 mod 2^32.
+__device__ __forceinline__ void drain_01(uint32_t *acc, const uint32_t *v0, const uint32_t *v1) {
+#pragma unroll
+    for (int cc = 0; cc < 32; ++cc) {
+        const float x0 = __uint_as_float(v0[cc]), x1 = __uint_as_float(v1[cc]);
+        const float t = __fmaf_rn(x1, 0.00390625f, kM);
+        const float lo = __fmaf_rn(__fsub_rn(t, kM), -256.0f, x1);
+        const float s = __fmaf_rn(lo, 256.0f, x0);
+        acc[cc] += (uint32_t)__float2int_rn(s) + (__float_as_uint(t) << 16);
+    }
+}
+
+// Groups 2 and 3 (|x2| <= 3 * 2^22, |x3| <= 2^24 after 256 K): (x2 << 16) +
+// (x3 << 24) = s << 16 mod 2^32 with s = x2 + 2^8 (x3 - 2^8 round(x3 / 2^8)),
+// exact (|s| < 2^24).
+__device__ __forceinline__ void drain_23(uint32_t *acc, const uint32_t *v0, const uint32_t *v1) {
+#pragma unroll
+    for (int cc = 0; cc < 32; ++cc) {
+        const float x3 = __uint_as_float(v1[cc]);
+        const float lo3 = __fmaf_rn(__fsub_rn(__fmaf_rn(x3, 0.00390625f, kM), kM), -256.0f, x3);
+        const float s = __fmaf_rn(lo3, 256.0f, __uint_as_float(v0[cc]));
+        acc[cc] += (uint32_t)__float2int_rn(s) << 16;
+    }
+}
 
 template <int BN>
 struct Cfg {
@@ -358,12 +395,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc_fence_after();
             const bool d01 = drains01(k, c, ++since01);
             if (d01) since01 = 0;
-            // Two groups are loaded before one wait.  Groups 0..2 convert on the
-            // F2I unit; only the low 8 bits of group 3 survive the shift by 24,
-            // so it is split on the FMA pipe instead, interleaved with group 2:
-            // with M = 1.5 * 2^23, q = (x / 256 + M) - M is an integer, lo = x -
-            // 256 q is exact (|lo| <= 128), and the low byte of the bits of
-            // lo + M is lo mod 256 (M's low byte is 0).
+            // Two groups are loaded before one wait.
 #pragma unroll
             for (int c0 = 0; c0 < HB; c0 += 32) {
                 uint32_t v0[32], v1[32];
@@ -371,22 +403,12 @@ __global__ void __launch_bounds__(THREADS, 1)
                     tmem_ld32_nowait(lane_addr + 0 * BN + c0, v0);
                     tmem_ld32_nowait(lane_addr + 1 * BN + c0, v1);
                     tmem_wait();
-#pragma unroll
-                    for (int cc = 0; cc < 32; ++cc)
-                        acc[c0 + cc] += (uint32_t)__float2int_rn(__uint_as_float(v0[cc])) +
-                                        ((uint32_t)__float2int_rn(__uint_as_float(v1[cc])) << 8);
+                    drain_01(acc + c0, v0, v1);
                 }
                 tmem_ld32_nowait(lane_addr + 2 * BN + c0, v0);
                 tmem_ld32_nowait(lane_addr + 3 * BN + c0, v1);
                 tmem_wait();
-#pragma unroll
-                for (int cc = 0; cc < 32; ++cc) {
-                    const float x = __uint_as_float(v1[cc]);
-                    const float q = __fsub_rn(__fmaf_rn(x, 0.00390625f, 12582912.0f), 12582912.0f);
-                    const float lo = __fmaf_rn(q, -256.0f, x);
-                    acc[c0 + cc] += ((uint32_t)__float2int_rn(__uint_as_float(v0[cc])) << 16) +
-                                    (__float_as_uint(__fadd_rn(lo, 12582912.0f)) << 24);
-                }
+                drain_23(acc + c0, v0, v1);
             }
             tc_fence_before();
             __syncwarp();
