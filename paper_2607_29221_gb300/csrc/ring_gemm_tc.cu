@@ -196,38 +196,40 @@ __global__ void __launch_bounds__(THREADS, 1)
     // Segment 0: whole tiles blockIdx.x + w * gridDim.x for every whole wave w
     // (dp_tiles = waves * gridDim.x; CTAs in step read the same B tiles at the
     // same K); segment 1: this CTA's even share of the remaining tiles' units
-    // (stream-K).  Without split, segment 0 is the CTA's one tile.
-    int64_t n0 = 0, s1b = 0, n1 = 0;
+    // (stream-K).  Without split, segment 0 is every tile blockIdx.x + w *
+    // gridDim.x (one tile when the grid covers them all).
+    // Unit counts fit in 32 bits (tiles * nchunks < 2^31, checked by the host).
+    int n0 = 0, s1b = 0, n1 = 0;
+    const int tiles = a.tiles_m * a.tiles_n;
     if (a.split) {
-        const int64_t dp_units = (int64_t)a.dp_tiles * nchunks;
-        n0 = (int64_t)(a.dp_tiles / (int)gridDim.x) * nchunks;
-        const int64_t U = (int64_t)a.tiles_m * a.tiles_n * nchunks - dp_units;
-        s1b = dp_units + U * blockIdx.x / gridDim.x;
-        n1 = dp_units + U * (blockIdx.x + 1) / gridDim.x - s1b;
+        const int dp_units = a.dp_tiles * nchunks;
+        n0 = (a.dp_tiles / (int)gridDim.x) * nchunks;
+        const int64_t U = (int64_t)tiles * nchunks - dp_units;
+        s1b = dp_units + (int)(U * blockIdx.x / gridDim.x);
+        n1 = dp_units + (int)(U * (blockIdx.x + 1) / gridDim.x) - s1b;
     } else {
-        n0 = nchunks;
+        n0 = ((tiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x) * nchunks;
     }
-    const int64_t n_units = n0 + n1;
+    const int n_units = n0 + n1;
     // Shift groups 0 and 1 gather 1 and 2 digit products per K value, so they
     // stay exact (|sum| <= 2^24) over two 256-wide chunks and are drained every
     // second chunk of a tile (and at the end of the tile or of a segment);
     // groups 2 and 3 are drained after every chunk.  `since` counts the chunks
     // accumulated in groups 0 and 1, including the current one.
-    auto drains01 = [&](int64_t k, int c, int since) {
+    auto drains01 = [&](int k, int c, int since) {
         return since >= 2 || c == nchunks - 1 || k == n0 - 1 || k == n_units - 1;
     };
     // Walks this CTA's units in order without divisions: (tile, chunk c) of
     // unit k (segment 0: tiles blockIdx.x + w * gridDim.x; segment 1: units
     // s1b, s1b + 1, ...).
     struct UnitWalk {
-        int64_t k, tile;
-        int c;
+        int k, tile, c;
     };
-    const int64_t s1_tile = s1b / nchunks;
+    const int s1_tile = s1b / nchunks;
     const int s1_c = (int)(s1b - s1_tile * nchunks);
     auto walk_init = [&](UnitWalk &w) {
         w.k = 0;
-        w.tile = n0 > 0 ? (int64_t)blockIdx.x : s1_tile;
+        w.tile = n0 > 0 ? (int)blockIdx.x : s1_tile;
         w.c = n0 > 0 ? 0 : s1_c;
     };
     auto walk_next = [&](UnitWalk &w) {
@@ -236,7 +238,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             w.c = s1_c;
         } else if (++w.c == nchunks) {
             w.c = 0;
-            w.tile += w.k < n0 ? (int64_t)gridDim.x : 1;
+            w.tile += w.k < n0 ? (int)gridDim.x : 1;
         }
     };
 
@@ -265,7 +267,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     if (warp == 0) {
         if (lane == 0) {
-            int64_t slot = 0;
+            int slot = 0;
             int s = 0;          // slot % STAGES
             uint32_t ph = 0;    // parity of the empty phase awaited for slot s (from the second round on)
             UnitWalk w;
@@ -294,7 +296,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             if (*abort_flag) {
                 // Let the copies this thread started land before the CTA exits.
-                for (int64_t q = slot > STAGES ? slot - STAGES : 0; q < slot; ++q) {
+                for (int q = slot > STAGES ? slot - STAGES : 0; q < slot; ++q) {
                     const unsigned long long t0 = gtime();
                     while (!mbar_try(&full[q % STAGES], (uint32_t)(q / STAGES) & 1) && gtime() - t0 < kWaitNs) {
                     }
@@ -304,7 +306,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             bool issued_any = false;
-            int64_t chunk_count = 0;
+            uint32_t chunk_count = 0;
             int s = 0;          // shared-memory slot of the next stage
             uint32_t ph = 0;    // parity of its full barrier
             int since01 = 0;
@@ -314,7 +316,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             UnitWalk w;
             walk_init(w);
             for (; w.k < n_units && !*abort_flag; walk_next(w)) {
-                const int64_t k = w.k;
+                const int k = w.k;
                 const int c = w.c;
                 const int ks0 = c * CHUNK, ks1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
                 const uint32_t keep01 = since01 > 0 ? 1u : 0u;   // groups 0, 1 carry on
@@ -381,12 +383,12 @@ __global__ void __launch_bounds__(THREADS, 1)
         uint32_t acc[HB];
 #pragma unroll
         for (int c = 0; c < HB; ++c) acc[c] = 0u;
-        int64_t chunk_count = 0;
+        uint32_t chunk_count = 0;
         int since01 = 0;
         UnitWalk wk;
         walk_init(wk);
         for (; wk.k < n_units; walk_next(wk)) {
-            const int64_t k = wk.k, tile = wk.tile;
+            const int k = wk.k, tile = wk.tile;
             const int c = wk.c;
             if (!mbar_wait(acc_full, (uint32_t)chunk_count & 1, abort_flag)) {
                 raise_abort(abort_flag);
@@ -534,19 +536,20 @@ mosaic_status launch_tc(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const
     }
     const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = (N + BN - 1) / BN, tiles = tiles_m * tiles_n;
     const int64_t nk = (K + BK - 1) / BK, nchunks = (nk + CHUNK - 1) / CHUNK;
+    if (tiles * nchunks > (int64_t)INT32_MAX) return MOSAIC_ERR_SHAPE;   // 32-bit unit numbers
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
         return MOSAIC_ERR_CUDA;
-    // One CTA per tile unless the last wave would leave more than 10% of the
-    // SMs idle; then a persistent grid shares the (tile, chunk) units evenly.
-    // Short products (fewer than 8 chunks, K < 2048) keep one CTA per tile:
-    // there the preparation of C and the split-tile atomics cost more than
-    // the idle SMs.
+    // Whole tiles on a persistent grid (at most one CTA per SM) unless the
+    // last wave would leave more than 10% of the SMs idle; then the grid also
+    // shares the remaining tiles' (tile, chunk) units evenly.  Short products
+    // (fewer than 8 chunks, K < 2048) keep whole tiles only: there the
+    // preparation of C and the split-tile atomics cost more than the idle SMs.
     const int64_t waves = (tiles + sms - 1) / sms;
     const bool split = nchunks >= 8 && (double)tiles / (double)(waves * sms) < 0.9;
     TcArgs args{Cm, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)K, (int)tiles_m, (int)tiles_n, split ? 1 : 0,
                 0, (int)o1.cols, o2.C, o2.ldc, o2.Cin, o2.ldcin};
-    int64_t grid = tiles;
+    int64_t grid = tiles < sms ? tiles : sms;
     if (split) {
         if (prepare_split(o1, M, st) != cudaSuccess || prepare_split(o2, M, st) != cudaSuccess)
             return MOSAIC_ERR_CUDA;
