@@ -180,8 +180,16 @@ size_t unmask_images_bytes(int64_t l, const mosaic_params *p) {
     for (uint32_t i = 1; i < p->d; i++) s += up(4 * tile_image_words(l, p->r[i - 1]));
     return s;
 }
+// Line-offset copies of the S lists for the levels that take the tiled gather.
+size_t unmask_lines_bytes(int64_t m, int64_t l, const mosaic_params *p) {
+    size_t s = 0;
+    for (uint32_t i = 1; i < p->d; i++)
+        if (pgather_takes(l, p->r[i - 1], (int)p->t[i])) s += up(4 * (size_t)(m * p->t[i]));
+    return s;
+}
 size_t ws_unmask(int64_t m, int64_t l, const mosaic_params *p) {
-    return ws_unmask_min(m, l, p) + ws_gemm(l, m, p->r[p->d - 1]) + unmask_images_bytes(l, p);
+    return ws_unmask_min(m, l, p) + ws_gemm(l, m, p->r[p->d - 1]) + unmask_images_bytes(l, p) +
+           unmask_lines_bytes(m, l, p);
 }
 
 }  // namespace
@@ -708,7 +716,22 @@ mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const ui
             ++nimg;
         }
     }
-    MOSAIC_TRY(unmask_prep(Z, ldz, l, m + od, rd, Qp, Kp, nimg, icol, ir, img, st));
+    // With room, the tiled gathers read line-offset copies of the S lists made
+    // in the same launch, instead of converting every round.
+    int nlin = 0;
+    LineCopy lin[2];
+    for (uint32_t i = 1; i < d; i++) {
+        SparseLevel &lv = lev[i - 1];
+        const size_t bytes = up(4 * (size_t)(m * lv.t));
+        if (!pgather_takes(l, lv.r, lv.t) || !aligned16(lv.idx) || !aligned16(lv.val) ||
+            !aligned16(cv.base + cv.used) || cv.used + bytes > cv.cap)
+            continue;
+        uint32_t *buf = cv.take<uint32_t>((size_t)(m * lv.t));
+        lin[nlin++] = LineCopy{lv.idx, buf, m * lv.t, lv.r};
+        lv.idx = buf;
+        lv.lines = 1;
+    }
+    MOSAIC_TRY(unmask_prep(Z, ldz, l, m + od, rd, Qp, Kp, nimg, icol, ir, img, nlin, lin, st));
     if (Qp) {
         MOSAIC_TRY(ring_gemm_tc_planes(Qp, Kp, l * Kp, Lp, Kp, m * Kp, tmp, m, K_tm, m, 1, l, m, rd, st));
     } else {

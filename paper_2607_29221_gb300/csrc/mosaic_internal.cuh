@@ -206,12 +206,22 @@ mosaic_status gather_status();
 // Launches a bounded wait that runs out after limit_ns (the self-test of the
 // timeout path: reported by the next device status as MOSAIC_ERR_TIMEOUT).
 mosaic_status wait_probe(unsigned long long limit_ns, cudaStream_t st);
+// A caller's position list turned into the tiled gather's line offsets:
+// dst[i] = pg_line(min(src[i], r - 1)) for count entries (a multiple of 4;
+// both pointers 16-byte aligned).
+struct LineCopy {
+    const uint32_t *src;
+    uint32_t *dst;
+    int64_t count;
+    uint32_t r;
+};
 // Before an unmask, in one launch: digit planes [4][l][Kp] of Q_d = columns
-// [qcol, qcol + rd) of Z (when Qp is not null) and the tile images of nimg <= 2
-// segments Z[:, icol[k] .. + ir[k]) (tile_image_words(l, ir[k]) words each).
+// [qcol, qcol + rd) of Z (when Qp is not null), the tile images of nimg <= 2
+// segments Z[:, icol[k] .. + ir[k]) (tile_image_words(l, ir[k]) words each)
+// and the line-offset copies of nlin <= 2 S lists.
 mosaic_status unmask_prep(const uint32_t *Z, int64_t ldz, int64_t l, int64_t qcol, int64_t rd, uint16_t *Qp,
                           int64_t Kp, int nimg, const int64_t *icol, const uint32_t *ir, uint32_t *const *img,
-                          cudaStream_t st);
+                          int nlin, const LineCopy *lin, cudaStream_t st);
 mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, int64_t seg_len,
                             int64_t g_count, int64_t nlist, bool list_is_col, const SparseLevel *lev,
                             int nlev, const uint32_t *a, int64_t lda, const uint32_t *b, int64_t ldb,

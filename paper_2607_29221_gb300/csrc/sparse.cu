@@ -788,6 +788,13 @@ struct UnmaskPrep {
     int64_t icol[2];
     int ir[2], irp[2], iblocks[2];
     uint32_t *img[2];
+    // Line-offset copies of caller lists: dst[i] = pg_line(min(src[i], r - 1)).
+    int nlin;
+    const uint32_t *lsrc[2];
+    uint32_t *ldst[2];
+    int64_t lcount[2];   // entries, a multiple of 4
+    uint32_t lr[2];
+    int lblocks[2];
 };
 
 __device__ __forceinline__ void split4(const uint32_t *src, uint16_t *dst, int64_t plane_stride, int64_t c,
@@ -830,6 +837,21 @@ __global__ void __launch_bounds__(256) unmask_prep_kernel(UnmaskPrep a) {
         }
         b -= a.iblocks[k];
     }
+    for (int k = 0; k < a.nlin; k++) {
+        if (b < a.lblocks[k]) {
+            const uint32_t rlast = a.lr[k] - 1;
+            const int64_t quads = a.lcount[k] / 4;
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.lsrc[k]);
+            uint4 *dst = reinterpret_cast<uint4 *>(a.ldst[k]);
+            for (int64_t i = (int64_t)b * 256 + threadIdx.x; i < quads; i += (int64_t)a.lblocks[k] * 256) {
+                const uint4 v = src[i];
+                dst[i] = make_uint4(pg_line(min(v.x, rlast)), pg_line(min(v.y, rlast)), pg_line(min(v.z, rlast)),
+                                    pg_line(min(v.w, rlast)));
+            }
+            return;
+        }
+        b -= a.lblocks[k];
+    }
 }
 
 }  // namespace
@@ -856,9 +878,9 @@ mosaic_status build_tile_image(const uint32_t *src, int64_t lds, int64_t col0, u
 
 mosaic_status unmask_prep(const uint32_t *Z, int64_t ldz, int64_t l, int64_t qcol, int64_t rd, uint16_t *Qp,
                           int64_t Kp, int nimg, const int64_t *icol, const uint32_t *ir, uint32_t *const *img,
-                          cudaStream_t st) {
+                          int nlin, const LineCopy *lin, cudaStream_t st) {
     if (l == 0) return MOSAIC_OK;
-    if (nimg < 0 || nimg > 2) return MOSAIC_ERR_UNSUPPORTED;
+    if (nimg < 0 || nimg > 2 || nlin < 0 || nlin > 2) return MOSAIC_ERR_UNSUPPORTED;
     UnmaskPrep a{};
     a.Z = Z;
     a.ldz = ldz;
@@ -886,6 +908,18 @@ mosaic_status unmask_prep(const uint32_t *Z, int64_t ldz, int64_t l, int64_t qco
         if (blocks > 0x3fffffff) return MOSAIC_ERR_SHAPE;
         a.iblocks[k] = (int)blocks;
         grid += blocks;
+    }
+    a.nlin = nlin;
+    for (int k = 0; k < nlin; k++) {
+        if (lin[k].count % 4 != 0 || lin[k].r < 1 || !aligned16(lin[k].src) || !aligned16(lin[k].dst))
+            return MOSAIC_ERR_UNSUPPORTED;
+        a.lsrc[k] = lin[k].src;
+        a.ldst[k] = lin[k].dst;
+        a.lcount[k] = lin[k].count;
+        a.lr[k] = lin[k].r;
+        const int64_t quads = lin[k].count / 4;
+        a.lblocks[k] = (int)((quads + 255) / 256 < 152 * 4 ? (quads + 255) / 256 : 152 * 4);
+        grid += a.lblocks[k];
     }
     if (grid == 0) return MOSAIC_OK;
     if (grid > 0x7fffffff) return MOSAIC_ERR_SHAPE;
