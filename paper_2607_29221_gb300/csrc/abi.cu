@@ -685,7 +685,8 @@ mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const ui
     Carve cv{static_cast<char *>(ws), ws_bytes, 0};
     uint32_t *tmp = cv.take<uint32_t>((size_t)(l * m));
     if (!tmp) return MOSAIC_ERR_WORKSPACE;
-    // tmp = K + Q_d L^T  (token-major: Q_d^T is the column block [m + od, m + Sr) of Z).
+    // tmp = K + Q_d L^T, or with the tensor-core product tmp = Y' - K - Q_d L^T
+    // (token-major: Q_d^T is the column block [m + od, m + Sr) of Z).
     const uint32_t *Qd = Z + m + od;
     const bool want_tc = variant == MOSAIC_GEMM_TC || (variant == MOSAIC_GEMM_AUTO && tc_available());
     const int64_t Kp = kpad8(rd);
@@ -733,13 +734,14 @@ mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const ui
     }
     MOSAIC_TRY(unmask_prep(Z, ldz, l, m + od, rd, Qp, Kp, nimg, icol, ir, img, nlin, lin, st));
     if (Qp) {
-        MOSAIC_TRY(ring_gemm_tc_planes(Qp, Kp, l * Kp, Lp, Kp, m * Kp, tmp, m, K_tm, m, 1, l, m, rd, st));
+        MOSAIC_TRY(ring_gemm_tc_planes_diff(Qp, Kp, l * Kp, Lp, Kp, m * Kp, tmp, m, Z, ldz, K_tm, m, -1, l, m, rd,
+                                            st));
     } else {
         MOSAIC_TRY(gemm_u32(variant, cv, Qd, ldz, 1, L, rd, 1, tmp, m, K_tm, m, 1, l, m, rd, st));
     }
-    // Y_hat = Y' - tmp - sum_i S_{i+1} Q_i, then decode.
-    return unmask_decode(Z, ldz, m, od, l, m, lev, (int)d - 1, tmp, m, s_w, s_x, bias, Y, Yhat, ldy,
-                         st);
+    // Y_hat = Y' - tmp - sum_i S_{i+1} Q_i (tmp - sum_i ... after the folded product), then decode.
+    return unmask_decode(Z, ldz, m, od, l, m, lev, (int)d - 1, tmp, m, s_w, s_x, bias, Y, Yhat, ldy, st,
+                         Qp != nullptr);
 }
 
 }  // namespace

@@ -148,6 +148,12 @@ mosaic_status ring_gemm_tc_planes2(const uint16_t *Ap, int64_t ldpa, int64_t a_p
                                    const uint32_t *Cin1, int64_t ldcin1, int64_t N1, uint32_t *C2, int64_t ldc2,
                                    const uint32_t *Cin2, int64_t ldcin2, int64_t N2, int64_t M, int64_t K,
                                    cudaStream_t st);
+// C = Cin - Csub + sgn * A B^T from planes, one output (K > 0; never split
+// into stream-K units).
+mosaic_status ring_gemm_tc_planes_diff(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const uint16_t *Bp,
+                                       int64_t ldpb, int64_t b_plane, uint32_t *C, int64_t ldc,
+                                       const uint32_t *Cin, int64_t ldcin, const uint32_t *Csub, int64_t ldcsub,
+                                       int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st);
 // Legacy mma.sync s8 ring GEMM (NT, uint32 operands split into int8 digit
 // planes in ws, at least ws_mma_s8(M, N, K) bytes).
 size_t ws_mma_s8(int64_t M, int64_t N, int64_t K);
@@ -227,11 +233,13 @@ mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, i
                             int nlev, const uint32_t *a, int64_t lda, const uint32_t *b, int64_t ldb,
                             int sgn, uint32_t *out, int64_t ldo, cudaStream_t st);
 // Unmask epilogue: list = output column j; staged rows = tokens k of Z.
+// Y_hat = Y' - tmp - sum_i S_{i+1} Q_i, or tmp - sum_i S_{i+1} Q_i when
+// `folded` (tmp already holds Y' - K - L Q_d), then decode.
 mosaic_status unmask_decode(const uint32_t *Z, int64_t ldz, int64_t seg_off, int64_t seg_len,
                             int64_t l, int64_t m, const SparseLevel *lev, int nlev,
                             const uint32_t *tmp, int64_t ldt, const float *s_w, const float *s_x,
                             const float *bias, float *Y, uint32_t *Yhat, int64_t ldy,
-                            cudaStream_t st);
+                            cudaStream_t st, bool folded = false);
 // out[j][c] = a[j][c] + sum_lev sum_q val[j][q] * P[(row_off_lev + idx[j][q]) * ldp + c]
 mosaic_status sparse_rowgather(const uint32_t *P, int64_t ldp, const SparseLevel *lev, int nlev,
                                int64_t m, int64_t ncols, const uint32_t *a, int64_t lda,

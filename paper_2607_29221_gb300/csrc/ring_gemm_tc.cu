@@ -120,6 +120,9 @@ struct TcArgs {
     int64_t ldc2;
     const uint32_t *Cin2;
     int64_t ldcin2;
+    // Plain mode, first output: C = Cin - Csub + sgn * A B^T (Csub nullable).
+    const uint32_t *Csub;
+    int64_t ldcsub;
 };
 
 __device__ __forceinline__ void raise_abort(volatile int *abort_flag) {
@@ -432,13 +435,15 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const uint32_t *cin = cin0 ? cin0 + (int64_t)gm * (second ? a.ldcin2 : a.ldcin) : nullptr;
                 const int64_t ldc_o = second ? a.ldc2 : a.ldc;
                 const int64_t ldcin_o = second ? a.ldcin2 : a.ldcin;
+                const uint32_t *sub = (!second && a.Csub) ? a.Csub + (int64_t)gm * a.ldcsub : nullptr;
                 if (a.sgn < 0) {
 #pragma unroll
                     for (int cc = 0; cc < HB; ++cc) acc[cc] = 0u - acc[cc];
                 }
                 const bool vec = (n0 + HB <= nout) && ((ldc_o & 3) == 0) &&
                                  ((reinterpret_cast<uintptr_t>(crow) & 15u) == 0) &&
-                                 (!cin || (((ldcin_o & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin) & 15u) == 0)));
+                                 (!cin || (((ldcin_o & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin) & 15u) == 0))) &&
+                                 (!sub || (((a.ldcsub & 3) == 0) && ((reinterpret_cast<uintptr_t>(sub) & 15u) == 0)));
                 if (a.split && !whole) {
                     // Other CTAs add into this tile too: exact and order-free in Z_{2^32}.
 #pragma unroll
@@ -454,6 +459,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                             const uint4 i4 = *reinterpret_cast<const uint4 *>(base + n0 + cc);
                             o.x += i4.x; o.y += i4.y; o.z += i4.z; o.w += i4.w;
                         }
+                        if (sub) {
+                            const uint4 s4 = *reinterpret_cast<const uint4 *>(sub + n0 + cc);
+                            o.x -= s4.x; o.y -= s4.y; o.z -= s4.z; o.w -= s4.w;
+                        }
                         *reinterpret_cast<uint4 *>(crow + n0 + cc) = o;
                     }
                 } else {
@@ -461,7 +470,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
                     for (int cc = 0; cc < HB; ++cc) {
                         const int gn = n0 + cc;
-                        if (gn < nout) crow[gn] = acc[cc] + (base ? base[gn] : 0u);
+                        if (gn < nout) crow[gn] = acc[cc] + (base ? base[gn] : 0u) - (sub ? sub[gn] : 0u);
                     }
                 }
             }
@@ -499,6 +508,8 @@ struct TcOut {
     const uint32_t *Cin;
     int64_t ldcin;
     int64_t cols;
+    const uint32_t *Csub = nullptr;   // first output only, plain mode
+    int64_t ldcsub = 0;
 };
 
 // Prepares a stream-K output: its tiles are summed with atomic adds, so it
@@ -546,9 +557,10 @@ mosaic_status launch_tc(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const
     // (fewer than 8 chunks, K < 2048) keep whole tiles only: there the
     // preparation of C and the split-tile atomics cost more than the idle SMs.
     const int64_t waves = (tiles + sms - 1) / sms;
-    const bool split = nchunks >= 8 && (double)tiles / (double)(waves * sms) < 0.9;
+    // A subtracted input is read in plain mode only (stream-K prepares C from Cin alone).
+    const bool split = !o1.Csub && nchunks >= 8 && (double)tiles / (double)(waves * sms) < 0.9;
     TcArgs args{Cm, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)K, (int)tiles_m, (int)tiles_n, split ? 1 : 0,
-                0, (int)o1.cols, o2.C, o2.ldc, o2.Cin, o2.ldcin};
+                0, (int)o1.cols, o2.C, o2.ldc, o2.Cin, o2.ldcin, o1.Csub, o1.ldcsub};
     int64_t grid = tiles < sms ? tiles : sms;
     if (split) {
         if (prepare_split(o1, M, st) != cudaSuccess || prepare_split(o2, M, st) != cudaSuccess)
@@ -604,6 +616,19 @@ mosaic_status ring_gemm_tc_planes2(const uint16_t *Ap, int64_t ldpa, int64_t a_p
     return launch_tc<128>(Ap, ldpa, a_plane, Bp, ldpb, b_plane, o1, o2, 1, M, K, st);
 }
 
+
+mosaic_status ring_gemm_tc_planes_diff(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const uint16_t *Bp,
+                                       int64_t ldpb, int64_t b_plane, uint32_t *Cm, int64_t ldc,
+                                       const uint32_t *Cin, int64_t ldcin, const uint32_t *Csub, int64_t ldcsub,
+                                       int sgn, int64_t M, int64_t N, int64_t K, cudaStream_t st) {
+    if (M == 0 || N == 0) return MOSAIC_OK;
+    if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX || K == 0 || !Cin || !Csub) return MOSAIC_ERR_SHAPE;
+    TcOut o1{Cm, ldc, Cin, ldcin, N};
+    o1.Csub = Csub;
+    o1.ldcsub = ldcsub;
+    const TcOut none{nullptr, 0, nullptr, 0, 0};
+    return launch_tc<128>(Ap, ldpa, a_plane, Bp, ldpb, b_plane, o1, none, sgn, M, K, st);
+}
 
 mosaic_status device_status(cudaStream_t st) {
     if (cudaStreamSynchronize(st) != cudaSuccess) return MOSAIC_ERR_CUDA;

@@ -974,11 +974,16 @@ mosaic_status unmask_decode(const uint32_t *Z, int64_t ldz, int64_t seg_off, int
                             int64_t l, int64_t m, const SparseLevel *lev, int nlev,
                             const uint32_t *tmp, int64_t ldt, const float *s_w, const float *s_x,
                             const float *bias, float *Y, uint32_t *Yhat, int64_t ldy,
-                            cudaStream_t st) {
+                            cudaStream_t st, bool folded) {
     (void)seg_off; (void)seg_len;
     GatherArgs g{};
     g.src = Z; g.lds = ldz; g.g_count = l; g.nlist = m;
-    g.a = Z; g.lda = ldz; g.b = tmp; g.ldb = ldt; g.sgn = -1; g.out = Yhat; g.ldo = ldy;
+    if (folded) {
+        g.a = tmp; g.lda = ldt; g.b = nullptr; g.ldb = 0;
+    } else {
+        g.a = Z; g.lda = ldz; g.b = tmp; g.ldb = ldt;
+    }
+    g.sgn = -1; g.out = Yhat; g.ldo = ldy;
     g.decode = 1; g.s_w = s_w; g.s_x = s_x; g.bias = bias; g.Y = Y; g.ldy = ldy;
     // The partial Y_hat between levels lives in tmp (each element is read and
     // then overwritten by the same thread).
