@@ -589,12 +589,15 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
         return cj && off ? reinterpret_cast<const uint32_t *>(reinterpret_cast<const char *>(cj) + off) : nullptr;
     };
     if (d > 1) {
-        for (uint32_t i = 1; i < d; i++) lev[i - 1].tiled = image(AL.c_img[i - 1]);
-        MOSAIC_TRY(sparse_gather(C, Sr, 0, od, n_pad, l, false, lev, (int)d - 1, Ux_tm, n_pad,
-                                 nullptr, 0, 1, Ux_tm, n_pad, st));
-        for (uint32_t i = 1; i < d; i++) lev[i - 1].tiled = image(AL.j_img[i - 1]);
-        MOSAIC_TRY(sparse_gather(J, Sr, 0, od, m, l, false, lev, (int)d - 1, K_tm, m, nullptr, 0, 1,
-                                 K_tm, m, st));
+        // U_x += sum_i C_i T_{i+1} and K += sum_i J_i T_{i+1} read the same lists:
+        // one launch per level serves both.
+        const uint32_t *cimg[2] = {nullptr, nullptr}, *jimg[2] = {nullptr, nullptr};
+        for (uint32_t i = 1; i < d; i++) {
+            cimg[i - 1] = image(AL.c_img[i - 1]);
+            jimg[i - 1] = image(AL.j_img[i - 1]);
+        }
+        MOSAIC_TRY(sparse_gather_pair(C, Sr, n_pad, Ux_tm, n_pad, cimg, J, Sr, m, K_tm, m, jimg, l, lev, (int)d - 1,
+                                      st));
     }
     return MOSAIC_OK;
 }

@@ -232,6 +232,15 @@ mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, i
                             int64_t g_count, int64_t nlist, bool list_is_col, const SparseLevel *lev,
                             int nlev, const uint32_t *a, int64_t lda, const uint32_t *b, int64_t ldb,
                             int sgn, uint32_t *out, int64_t ldo, cudaStream_t st);
+// The two Init X gathers of the same T lists in one launch per level:
+// out[j][.] += sum_q val[j][q] * src[.][off + idx[j][q]] over g_count staged
+// rows (tile images img[L]), and the same for (src2, g_count2, out2, img2[L]).
+// Falls back to two sparse_gather calls when a job would not take the tiled
+// gather.
+mosaic_status sparse_gather_pair(const uint32_t *src, int64_t lds, int64_t g_count, uint32_t *out, int64_t ldo,
+                                 const uint32_t *const *img, const uint32_t *src2, int64_t lds2, int64_t g_count2,
+                                 uint32_t *out2, int64_t ldo2, const uint32_t *const *img2, int64_t nlist,
+                                 const SparseLevel *lev, int nlev, cudaStream_t st);
 // Unmask epilogue: list = output column j; staged rows = tokens k of Z.
 // Y_hat = Y' - tmp - sum_i S_{i+1} Q_i, or tmp - sum_i S_{i+1} Q_i when
 // `folded` (tmp already holds Y' - K - L Q_d), then decode.

@@ -54,6 +54,13 @@ struct GatherArgs {
     int trusted;   // positions known to be < r (drawn by this library)
     const uint32_t *tiled;   // tile images of the level's segment (build_tile_image) or null
     int lines;               // positions are already line offsets (p << 7 | chunk bits), see pg_line
+    // Tiled gather only: a second job on the same lists and segment columns.
+    // Its units follow the first job's; they stage rows of src2 (tiled2)
+    // and read a2 / write out2 (no b, no decode).
+    int two;
+    const uint32_t *src2, *tiled2, *a2;
+    int64_t lds2, g_count2, lda2, ldo2;
+    uint32_t *out2;
 };
 
 // Staged rows plus the per-warp list rings.
@@ -243,7 +250,7 @@ constexpr int kPgStageBatch = 12;  // 16-byte loads a lane keeps in flight while
 
 template <bool LIST_IS_COL, bool CLAMP>
 __global__ void __launch_bounds__(kPgWarps * 32, 1)
-    pgather_kernel(GatherArgs a, int units, int chunks, int vec_src, int vec_ab) {
+    pgather_kernel(GatherArgs a, int units, int units0, int chunks, int vec_src, int vec_ab) {
     constexpr int kPgRing = pg_ring<LIST_IS_COL>();
     extern __shared__ __align__(16) uint32_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -300,13 +307,13 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
     // Tile images (a.tiled) hold exactly this layout: one bulk copy per 32 KB,
     // all threads wait (bounded) for the barrier.  Returns false if the copy
     // did not land in time (error word raised).
-    auto stage_tiled = [&](int64_t tile) -> bool {
+    auto stage_tiled = [&](const uint32_t *img, int64_t tile) -> bool {
         const uint32_t bytes = (uint32_t)rp * 128u;
         if (threadIdx.x == 0) {
             // The previous tile's shared-memory reads happen before these async writes.
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             mbar_expect_tx(bar, bytes);
-            const char *src = reinterpret_cast<const char *>(a.tiled) + (size_t)tile * bytes;
+            const char *src = reinterpret_cast<const char *>(img) + (size_t)tile * bytes;
             for (uint32_t off = 0; off < bytes; off += 32768u)
                 bulk_load(sm_base + off, src + off, bytes - off < 32768u ? bytes - off : 32768u, bar);
         }
@@ -318,7 +325,7 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
         bar_phase ^= 1u;
         return ok;
     };
-    auto stage = [&](int64_t tile) {
+    auto stage = [&](const uint32_t *src, int64_t lds, int64_t g_count, int64_t tile) {
         const int64_t g0 = tile * kPgRows;
         const int gl = lane >> 3, pq = lane & 7;
         const int total = 8 * (rp / 32);
@@ -330,8 +337,8 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
                 const int g = (it & 7) * 4 + gl;
                 const int p = (it >> 3) * 32 + pq * 4;
                 w[j] = make_uint4(0u, 0u, 0u, 0u);
-                if (it < total && g0 + g < a.g_count && p < r) {
-                    const uint32_t *srow = a.src + (g0 + g) * a.lds + a.col0;
+                if (it < total && g0 + g < g_count && p < r) {
+                    const uint32_t *srow = src + (g0 + g) * lds + a.col0;
                     if (vec_src && p + 4 <= r) {
                         w[j] = __ldg(reinterpret_cast<const uint4 *>(srow + p));
                     } else {
@@ -364,18 +371,23 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
 #pragma unroll
     for (int j = 0; j < kPgRing - 1; j++) issue();
     int s = 0;
-    int64_t tile = u_begin / chunks;
+    // units0 (a multiple of chunks) is where the second job's units start.
+    int64_t tile = (u_begin >= units0 ? u_begin - units0 : u_begin) / chunks;
     int chunk = u_begin % chunks;
     for (int u = u_begin; u < u_end; u++) {
+        const bool j1 = u >= units0;   // the same for every thread
+        if (u == units0) tile = 0;
+        const int64_t g_count = j1 ? a.g_count2 : a.g_count;
         if (u == u_begin || chunk == 0) {   // a new tile: the same unit for every warp
             __syncthreads();
-            if (a.tiled) {
-                stage_tiled(tile);
+            const uint32_t *img = j1 ? a.tiled2 : a.tiled;
+            if (img) {
+                stage_tiled(img, tile);
             } else {
-                stage(tile);
+                stage(j1 ? a.src2 : a.src, j1 ? a.lds2 : a.lds, g_count, tile);
             }
             __syncthreads();
-            if (a.tiled && *abort_flag) {
+            if (img && *abort_flag) {
                 // Let this CTA's copy land (bounded) before leaving.
                 if (threadIdx.x == 0) mbar_drain(bar, bar_phase ^ 1u);
                 break;
@@ -385,12 +397,14 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
         const int64_t g = tile * kPgRows + li * 4;
         const bool e_ok = e < a.nlist;
         // a - b of the unit's outputs: row e, columns g .. g+3 (or the transpose).
-        const bool vec = vec_ab && !LIST_IS_COL && g + 4 <= a.g_count;
+        const bool vec = vec_ab && !LIST_IS_COL && g + 4 <= g_count;
+        const uint32_t *ja = j1 ? a.a2 : a.a;
+        const int64_t jlda = j1 ? a.lda2 : a.lda;
         uint32_t ab[4] = {0u, 0u, 0u, 0u};
         if (e_ok) {
             if (vec) {
-                if (a.a) {
-                    const uint4 x = __ldg(reinterpret_cast<const uint4 *>(a.a + e * a.lda + g));
+                if (ja) {
+                    const uint4 x = __ldg(reinterpret_cast<const uint4 *>(ja + e * jlda + g));
                     ab[0] = x.x; ab[1] = x.y; ab[2] = x.z; ab[3] = x.w;
                 }
                 if (a.b) {
@@ -400,11 +414,11 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
             } else {
 #pragma unroll
                 for (int c = 0; c < 4; c++) {
-                    if (g + c >= a.g_count) break;
+                    if (g + c >= g_count) break;
                     const int64_t row = LIST_IS_COL ? g + c : e;
                     const int64_t col = LIST_IS_COL ? e : g + c;
                     uint32_t v = 0u;
-                    if (a.a) v += a.a[row * a.lda + col];
+                    if (ja) v += ja[row * jlda + col];
                     if (a.b) v -= a.b[row * a.ldb + col];
                     ab[c] = v;
                 }
@@ -451,15 +465,17 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
             uint32_t res[4];
 #pragma unroll
             for (int c = 0; c < 4; c++) res[c] = (a.sgn >= 0 ? acc[c] : 0u - acc[c]) + ab[c];
-            if (vec && a.out && !a.decode) {
-                *reinterpret_cast<uint4 *>(a.out + e * a.ldo + g) = make_uint4(res[0], res[1], res[2], res[3]);
+            uint32_t *jout = j1 ? a.out2 : a.out;
+            const int64_t jldo = j1 ? a.ldo2 : a.ldo;
+            if (vec && jout && !a.decode) {
+                *reinterpret_cast<uint4 *>(jout + e * jldo + g) = make_uint4(res[0], res[1], res[2], res[3]);
             } else {
 #pragma unroll
                 for (int c = 0; c < 4; c++) {
-                    if (g + c >= a.g_count) break;
+                    if (g + c >= g_count) break;
                     const int64_t row = LIST_IS_COL ? g + c : e;
                     const int64_t col = LIST_IS_COL ? e : g + c;
-                    if (a.out) a.out[row * a.ldo + col] = res[c];
+                    if (jout) jout[row * jldo + col] = res[c];
                     if (a.decode) {
                         float y = __fmul_rn(__fmul_rn(__int2float_rn((int32_t)res[c]), a.s_w[col]), a.s_x[row]);
                         if (a.bias) y = __fadd_rn(y, a.bias[col]);
@@ -495,16 +511,22 @@ mosaic_status launch_pgather(const GatherArgs &a, cudaStream_t st) {
         per_sm < 1)
         return MOSAIC_ERR_CUDA;
     const int64_t tiles = (a.g_count + kPgRows - 1) / kPgRows;
+    const int64_t tiles2 = a.two ? (a.g_count2 + kPgRows - 1) / kPgRows : 0;
     const int64_t chunks = (a.nlist + kPgEnts - 1) / kPgEnts;
-    const int64_t units = tiles * chunks;
+    const int64_t units0 = tiles * chunks, units = (tiles + tiles2) * chunks;
     const int64_t slots = (int64_t)sms * per_sm;
     const int64_t grid = units < slots ? units : slots;
     if (units > 0x7fffffff) return MOSAIC_ERR_SHAPE;
-    const int vec_src = aligned16(a.src) && a.lds % 4 == 0 && a.col0 % 4 == 0;
+    int vec_src = aligned16(a.src) && a.lds % 4 == 0 && a.col0 % 4 == 0;
     // 16-byte a / b / out accesses (rows = list entities only).
-    const int vec_ab = (!a.a || (aligned16(a.a) && a.lda % 4 == 0)) && (!a.b || (aligned16(a.b) && a.ldb % 4 == 0)) &&
-                       (!a.out || (aligned16(a.out) && a.ldo % 4 == 0));
-    kern<<<(unsigned)grid, kPgWarps * 32, smem, st>>>(a, (int)units, (int)chunks, vec_src, vec_ab);
+    int vec_ab = (!a.a || (aligned16(a.a) && a.lda % 4 == 0)) && (!a.b || (aligned16(a.b) && a.ldb % 4 == 0)) &&
+                 (!a.out || (aligned16(a.out) && a.ldo % 4 == 0));
+    if (a.two) {
+        vec_src = vec_src && aligned16(a.src2) && a.lds2 % 4 == 0;
+        vec_ab = vec_ab && (!a.a2 || (aligned16(a.a2) && a.lda2 % 4 == 0)) &&
+                 (!a.out2 || (aligned16(a.out2) && a.ldo2 % 4 == 0));
+    }
+    kern<<<(unsigned)grid, kPgWarps * 32, smem, st>>>(a, (int)units, (int)units0, (int)chunks, vec_src, vec_ab);
     return launch_status();
 }
 
@@ -968,6 +990,49 @@ mosaic_status sparse_gather(const uint32_t *src, int64_t lds, int64_t seg_off, i
     g.trusted = 1;   // the T lists of Init X come from prg_sparse
     // Later levels accumulate in place in `out`.
     return gather_levels(g, list_is_col, lev, nlev, out, ldo, st);
+}
+
+mosaic_status sparse_gather_pair(const uint32_t *src, int64_t lds, int64_t g_count, uint32_t *out, int64_t ldo,
+                                 const uint32_t *const *img, const uint32_t *src2, int64_t lds2, int64_t g_count2,
+                                 uint32_t *out2, int64_t ldo2, const uint32_t *const *img2, int64_t nlist,
+                                 const SparseLevel *lev, int nlev, cudaStream_t st) {
+    // Both jobs on the tiled gather, or two separate calls.
+    bool pair = nlev > 0 && nlev <= kMaxLev;
+    for (int L = 0; pair && L < nlev; L++) {
+        const bool lists_vec = ((reinterpret_cast<uintptr_t>(lev[L].idx) | reinterpret_cast<uintptr_t>(lev[L].val)) &
+                                15u) == 0;
+        pair = lists_vec && pgather_takes(g_count, lev[L].r, lev[L].t) && pgather_takes(g_count2, lev[L].r, lev[L].t) &&
+               (!img[L]) == (!img2[L]);
+    }
+    if (!pair) {
+        SparseLevel l1[kMaxLev], l2[kMaxLev];
+        for (int L = 0; L < nlev && L < kMaxLev; L++) {
+            l1[L] = lev[L];
+            l1[L].tiled = img[L];
+            l2[L] = lev[L];
+            l2[L].tiled = img2[L];
+        }
+        MOSAIC_TRY(sparse_gather(src, lds, 0, 0, g_count, nlist, false, l1, nlev, out, ldo, nullptr, 0, 1, out, ldo,
+                                 st));
+        return sparse_gather(src2, lds2, 0, 0, g_count2, nlist, false, l2, nlev, out2, ldo2, nullptr, 0, 1, out2,
+                             ldo2, st);
+    }
+    if (g_count == 0 && g_count2 == 0) return MOSAIC_OK;
+    if (nlist == 0) return MOSAIC_OK;
+    for (int L = 0; L < nlev; L++) {
+        GatherArgs g{};
+        g.src = src; g.lds = lds; g.g_count = g_count; g.nlist = nlist;
+        g.a = out; g.lda = ldo; g.sgn = 1; g.out = out; g.ldo = ldo;
+        g.trusted = 1;   // the T lists of Init X come from prg_sparse
+        g.col0 = lev[L].off; g.r = lev[L].r; g.idx = lev[L].idx; g.val = lev[L].val; g.t = lev[L].t;
+        g.tiled = img[L];
+        g.lines = lev[L].lines;
+        g.two = 1;
+        g.src2 = src2; g.lds2 = lds2; g.g_count2 = g_count2; g.tiled2 = img2[L];
+        g.a2 = out2; g.lda2 = ldo2; g.out2 = out2; g.ldo2 = ldo2;
+        MOSAIC_TRY((launch_pgather<false, false>(g, st)));
+    }
+    return MOSAIC_OK;
 }
 
 mosaic_status unmask_decode(const uint32_t *Z, int64_t ldz, int64_t seg_off, int64_t seg_len,
