@@ -207,14 +207,18 @@ __global__ void __launch_bounds__(GW * 32) gather_kernel(GatherArgs a) {
 // banks thanks to the permutation.
 // The (position, value) lists stream through a per-warp ring in rounds of
 // 16 pairs (cp.async one or two rounds ahead, zero-filled past the end of a
-// list).  Once a round has landed, each lane rewrites two of its entity's
-// positions into line addresses with the permutation bits in place (clamping
-// positions of caller lists to r - 1), so that the gather loop needs one XOR
-// per pair.  Work units are (tile, 64 entities), numbered tile-major and split
-// evenly over a persistent grid, so a CTA stages each of its one or two tiles
-// once; each unit's a - b operands are loaded when it starts and its outputs
-// written when its last round is done (16-byte accesses where the output rows
-// are the list entities and the layout allows).
+// list).  Lists already given as line addresses (`lines`: drawn that way, or
+// converted once per call) are used as they are; otherwise, once a round has
+// landed, each lane rewrites two of its entity's positions into line
+// addresses with the permutation bits in place (clamping positions of caller
+// lists to r - 1), so that the gather loop needs one XOR per pair.  Work
+// units are (tile, 64 entities), numbered tile-major and split evenly over a
+// persistent grid, so a CTA stages each of its one or two tiles once; with a
+// second job (`two`: another source and output on the same lists) its units
+// follow the first job's.  Each unit's a - b operands are loaded when it
+// starts and its outputs written when its last round is done (16-byte
+// accesses where the output rows are the list entities and the layout
+// allows).
 // ---------------------------------------------------------------------------
 constexpr int kPgRows = 32;
 constexpr int kPgWarps = 16;
