@@ -75,6 +75,17 @@ def test_workspace_sizes(lib):
     assert M.mosaic_workspace_bytes(M.OP_MASK_WEIGHT, 8, 64, 0, bad) == 0
 
 
+def test_unmask_workspace_holds_the_fast_path(lib):
+    """The advertised unmask workspace (Example 3.1, 512 tokens, m = 4096) holds
+    every part the fast path carves: the l x m scratch, the digit planes of Q_d
+    (4 x l x 656 bf16), the tile images of Q_1 and Q_2 (16 tiles x r_i x 32 words)
+    and the line-offset copies of both S lists (m x 80 words each)."""
+    p = M.default_params()
+    l, m = 512, 4096
+    need = (l * m * 4 + 4 * l * 656 * 2 + 16 * 1536 * 32 * 4 + 16 * 1024 * 32 * 4 + 2 * m * 80 * 4)
+    assert M.mosaic_workspace_bytes(M.OP_UNMASK, m, 0, l, p) >= need
+
+
 def _status(fn, *args):
     return getattr(M.lib(), fn)(*args)
 
