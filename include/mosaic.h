@@ -11,8 +11,9 @@
  * Conventions shared by every entry point
  *  - Every matrix pointer is a DEVICE pointer owned by the caller; the
  *    library never allocates, frees or retains memory.  Scratch memory comes
- *    in `ws` (size from mosaic_workspace_bytes) and must not overlap any
- *    other argument.
+ *    in `ws` (size from mosaic_workspace_bytes, for a 256-byte aligned ws as
+ *    cudaMalloc returns; from a misaligned ws the bytes before its first
+ *    256-byte boundary go unused) and must not overlap any other argument.
  *  - Every call is asynchronous on `stream` (a cudaStream_t passed as void*;
  *    NULL is the legacy default stream).  A status of MOSAIC_OK means the
  *    work was validated and enqueued; faults inside a kernel surface at the
@@ -335,7 +336,11 @@ mosaic_status mosaic_advance_pass(uint64_t *pass_dev, uint64_t delta, void *stre
  *   Y[k][j] = ((float)(int32)Y_hat[k][j] * s_w[j]) * s_x[k] + bias[j]
  * (fp32, two roundings of the products, no fused multiply-add; bias
  * nullable).  Y: l x m fp32 (ldy); Yhat (nullable): l x m uint32 (ldy).
- * ws: mosaic_workspace_bytes(MOSAIC_OP_UNMASK, m, 0, l, p). */
+ * ws: mosaic_workspace_bytes(MOSAIC_OP_UNMASK, m, 0, l, p) bytes hold every
+ * optional part (tensor-core digit planes of Q_d, tile images of the Q_i,
+ * line-offset copies of the S lists); any size from 4 l m bytes (rounded up
+ * to 256) works, parts that do not fit are skipped and the result is the
+ * same; less returns MOSAIC_ERR_WORKSPACE. */
 mosaic_status mosaic_unmask(const mosaic_params *p, int64_t l, int64_t m, const uint32_t *Z,
                             int64_t ldz, const uint32_t *K_tm, const uint32_t *L,
                             const uint32_t *S_idx, const uint32_t *S_val, const float *s_w,

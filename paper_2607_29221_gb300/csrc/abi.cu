@@ -35,6 +35,14 @@ struct Carve {
     }
 };
 
+// Carving starts at the first kAlign boundary inside ws, so every part is
+// aligned (TMA operands, 16-byte vector accesses) even when the caller's
+// buffer is not; its leading bytes then go unused.
+Carve carve(void *ws, size_t bytes) {
+    const size_t pad = (size_t)((kAlign - reinterpret_cast<uintptr_t>(ws) % kAlign) % kAlign);
+    return Carve{static_cast<char *>(ws), bytes, pad < bytes ? pad : bytes};
+}
+
 bool rounds_ok(uint32_t r) { return r == 8 || r == 12 || r == 20; }
 
 mosaic_status check_params(const mosaic_params *p) {
@@ -351,7 +359,7 @@ mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B
     // Tensor-core variant: split both operands into digit planes in ws.
     const int64_t Kp = (K + 7) / 8 * 8;
     if (!aligned16(A) || !aligned16(B) || lda % 4 || ldb % 4) return MOSAIC_ERR_ALIGN;
-    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    Carve cv = carve(ws, ws_bytes);
     uint16_t *Ap = cv.take<uint16_t>((size_t)(4 * M * Kp));
     uint16_t *Bp = cv.take<uint16_t>((size_t)(4 * N * Kp));
     if (!Ap || !Bp) return MOSAIC_ERR_WORKSPACE;
@@ -422,7 +430,7 @@ mosaic_status mosaic_mask_chains(const mosaic_params *p, const mosaic_key *key, 
     const Key k = to_key(key);
     const int R = (int)p->rounds;
     const int64_t Sr = sum_r(p);
-    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    Carve cv = carve(ws, ws_bytes);
     // Level 1: M_1 (r_1 x n_pad) is P_1; N_1 (n_pad x r_1) is C_1.
     MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_M, 1), chain_id, R, p->r[0], n_pad, P, n_pad, st));
     MOSAIC_TRY(prg_uniform(k, tag_of(MOSAIC_TAG_N, 1), chain_id, R, n_pad, p->r[0], C, Sr, st));
@@ -463,7 +471,7 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, 
     const int R = (int)p->rounds;
     const uint32_t d = p->d;
     const int64_t Sr = sum_r(p), rd = p->r[d - 1], od = off_r(p, d);
-    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    Carve cv = carve(ws, ws_bytes);
     uint32_t *WE = cv.take<uint32_t>((size_t)(m * n_pad));
     if (!WE) return MOSAIC_ERR_WORKSPACE;
 
@@ -529,7 +537,7 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
     // d - 1 LPN levels.  act_nested = 0: R at rank r_1 against C_1, J_1 only.
     const uint32_t d = act_levels(p) + 1;
     const int64_t Sr = sum_r(p), rd = r_act(p), od = p->act_nested ? off_r(p, p->d) : 0;
-    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    Carve cv = carve(ws, ws_bytes);
     uint32_t *Rt = cv.take<uint32_t>((size_t)(l * rd));
     if (!Rt) return MOSAIC_ERR_WORKSPACE;
     SparseLevel lev[2];
@@ -685,7 +693,7 @@ mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const ui
     if (d > 1 && (!S_idx || !S_val)) return MOSAIC_ERR_ARG;
     if (ws_bytes < ws_unmask_min(m, l, p)) return MOSAIC_ERR_WORKSPACE;
     cudaStream_t st = as_stream(stream);
-    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    Carve cv = carve(ws, ws_bytes);
     uint32_t *tmp = cv.take<uint32_t>((size_t)(l * m));
     if (!tmp) return MOSAIC_ERR_WORKSPACE;
     // tmp = K + Q_d L^T, or with the tensor-core product tmp = Y' - K - Q_d L^T
@@ -803,7 +811,7 @@ mosaic_status mosaic_freivalds_check(int k, const uint32_t *a, const uint32_t *Y
     if (m < 1 || n_pad < 1 || l < 0 || ldz < m || ldx < n_pad) return MOSAIC_ERR_SHAPE;
     if (l == 0) return MOSAIC_OK;
     if (!a || !Ychk || !Z || !Xp || !bad || !n_bad) return MOSAIC_ERR_ARG;
-    Carve cv{static_cast<char *>(ws), ws_bytes, 0};
+    Carve cv = carve(ws, ws_bytes);
     uint32_t *lhs = cv.take<uint32_t>((size_t)(k * l));
     uint32_t *rhs = cv.take<uint32_t>((size_t)(k * l));
     if (!lhs || !rhs) return MOSAIC_ERR_WORKSPACE;

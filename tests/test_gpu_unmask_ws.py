@@ -3,8 +3,9 @@ the result.  With the full workspace the call uses tensor-core digit planes of
 Q_d (the product then writes Y' - K - Q_d L^T), tile images of Q_1, Q_2 and
 line-offset copies of the S lists; without room for the copies the gathers
 convert positions per round; at the minimum size (the l x m scratch only) the
-product runs without planes and the gathers stage rows directly.  Y_hat and Y
-are bit-identical across the three, and Y_hat equals Y' - K - L Q_d -
+product runs without planes and the gathers stage rows directly; a workspace
+that starts off a 256-byte boundary is carved from its first boundary.  Y_hat
+and Y are bit-identical across all four, and Y_hat equals Y' - K - L Q_d -
 sum_i S_{i+1} Q_i computed by the oracle from the same Z."""
 from types import SimpleNamespace
 
@@ -57,17 +58,19 @@ def test_unmask_workspace_sizes_agree(m, l):
     Z = layer.server(Xp, Xpl)
     full = M.mosaic_workspace_bytes(M.OP_UNMASK, m, 0, l, gp)
     lines = sum(_up(4 * m * ti) for ti in t)
-    sizes = {"full": full, "no_line_copies": full - lines, "minimum": _up(4 * l * m)}
+    # (bytes, offset): the misaligned buffer starts 4 bytes past an aligned one.
+    sizes = {"full": (full, 0), "no_line_copies": (full - lines, 0), "minimum": (_up(4 * l * m), 0),
+             "misaligned": (full + 256, 4)}
     got = {}
-    for name, nb in sizes.items():
-        ws = torch.empty(nb, dtype=torch.uint8, device="cuda")
+    for name, (nb, off) in sizes.items():
+        ws = torch.empty(nb + off, dtype=torch.uint8, device="cuda")[off:]
         Y = torch.empty(l, m, dtype=torch.float32, device="cuda")
         Yhat = torch.empty(l, m, dtype=torch.int32, device="cuda")
         M.mosaic_unmask_planes(gp, l, m, Z, Z.stride(0), mp.K, layer.L, layer.L_planes, layer.S_idx,
                                layer.S_val, layer.s_w, s_x, layer.bias, Y, Yhat, m, M.GEMM_AUTO, ws)
         M.mosaic_device_status()
         got[name] = (_host(Yhat), _host(Y))
-    for name in ("no_line_copies", "minimum"):
+    for name in ("no_line_copies", "minimum", "misaligned"):
         assert np.array_equal(got[name][0], got["full"][0]), name
         assert np.array_equal(got[name][1], got["full"][1]), name
     # Y_hat by the oracle's unmask (feature-major) from the same Z, K, L and S lists.
