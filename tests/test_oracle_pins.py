@@ -304,6 +304,80 @@ def test_depth_one_matches_simple_protocol():
     assert np.array_equal(simple, r["Y_hat"])
 
 
+def _sparse_dense(S, rows, r):
+    """(idx, val), rows x t with distinct positions per row -> dense rows x r."""
+    idx, val = S
+    D = np.zeros((rows, r), np.uint32)
+    np.put_along_axis(D, idx.astype(np.int64), val, axis=1)
+    return D
+
+
+def _rank_gf2(A):
+    """Rank over GF(2) of the low bits of A (rows as Python integers)."""
+    rows = [int("".join("1" if b else "0" for b in row) or "0", 2) for row in (A & 1).astype(bool)]
+    rank = 0
+    while rows:
+        piv = max(rows)
+        if piv == 0:
+            break
+        rows.remove(piv)
+        top = piv.bit_length() - 1
+        rows = [x ^ piv if (x >> top) & 1 else x for x in rows]
+        rank += 1
+    return rank
+
+
+@pytest.mark.parametrize("act_nested", [True, False])
+@pytest.mark.parametrize("d", [1, 2, 3])
+def test_masks_follow_the_nested_substitution_form(d, act_nested):
+    """The masks against the nested form they come from, evaluated inside out from the
+    sampled M_i, N_i (not from the oracle's chain products):
+      eq. weight-mask, first line: U_w - E_w = (((L M_d + S_d) M_{d-1} + S_{d-1}) ... + S_2) M_1;
+      eq. activation-mask:         U_x - E_x = N_1 (T_2 + N_2 (T_3 + ... N_d R))
+                                   (N_1 R with the LWE-only activation mask of Sec. 5.2);
+      Init X 1c with J_i = (W_hat + E_w) N_1 ... N_i:  K = (W_hat + E_w)(U_x - E_x).
+    A dropped LPN term, a term at the wrong level or a missing E fails here even when
+    the unmask drops the same term (which the noise identity cannot see)."""
+    p = O.Params(d=d, r=SMALL.r[:d], t=SMALL.t[: d - 1], sigma=1.0, act_nested=act_nested)
+    m, n, l = 40, 100, 12
+    _, r, _, _ = _run(p, m=m, n=n, l=l, seed_off=10 + d)
+    ws, ps, n_pad = r["ws"], r["ps"], r["n_pad"]
+    rk = p.ranks(n_pad)
+    Ms = [O.sample_uniform(KEY, O.tag(O.KIND_M, i), n_pad, rk[i], rk[i - 1]) for i in range(1, d + 1)]
+    Ns = [O.sample_uniform(KEY, O.tag(O.KIND_N, i), n_pad, rk[i - 1], rk[i]) for i in range(1, d + 1)]
+    acc = ws.L
+    for i in range(d, 0, -1):                       # level i: acc <- acc M_i (+ S_i below level 1)
+        acc = acc @ Ms[i - 1]
+        if i > 1:
+            acc = acc + _sparse_dense(ws.S[i], m, rk[i - 1])
+    assert np.array_equal(ws.W_masked - ws.W_hat - ws.E_w, acc)
+    if act_nested:
+        acc = ps.R
+        for i in range(d, 0, -1):                   # acc <- N_i (acc + T_{i+1})
+            if i < d:
+                acc = acc + _sparse_dense(ps.T[i + 1], l, rk[i]).T
+            acc = Ns[i - 1] @ acc
+    else:
+        acc = Ns[0] @ ps.R
+    Ux_noiseless = ps.U_x - ps.E_x
+    assert np.array_equal(Ux_noiseless, acc)
+    assert np.array_equal(ps.K, (ws.W_hat + ws.E_w) @ Ux_noiseless)
+
+
+def test_weight_mask_rank_mod_2():
+    """Rank facts of eq. weight-mask: every term has row space inside that of M_1, so
+    rank(U_w - E_w) <= r_1; without the sparse LPN terms it would be <= r_d, and with
+    them (d >= 2) it exceeds r_d.  Checked over GF(2) on a 256 x 256 case."""
+    for d, r, t in ((3, (96, 64, 40), (6, 5)), (2, (96, 40), (6,)), (1, (96,), ())):
+        p = O.Params(d=d, r=r, t=t, sigma=1.0)
+        _, res, _, _ = _run(p, m=256, n=256, l=4, seed_off=20 + d)
+        ws = res["ws"]
+        rank = _rank_gf2(ws.W_masked - ws.W_hat - ws.E_w)
+        assert rank <= r[0]
+        if d >= 2:
+            assert rank > r[-1]
+
+
 def test_masked_input_is_uniform_when_x_is_zero():
     from scipy import stats
     p = O.Params(d=3, r=(96, 64, 40), t=(6, 5), sigma=0.5)
