@@ -8,10 +8,12 @@ is timed apart (``init_w_s``).
 
 Workloads (``--workload``; seeded synthetic inputs, activations ~ N(0,1),
 weights ~ N(0,0.02), Example 3.1 parameters):
-  attn_proj_7b_512x4096x4096   (default) X 512 x 4096, W 4096 x 4096
+  decoder_70b_prefill_2048     (default) one 70B decoder layer: 4 masked linears
+                               (QKV 8192->10240, O 8192->8192, gate+up 8192->57344,
+                               down 28672->8192) + fp32 RMSNorm / causal GQA
+                               attention / SwiGLU / residuals, 2048 tokens
+  attn_proj_7b_512x4096x4096   X 512 x 4096, W 4096 x 4096
   ffn_7b_2048x4096x14336       up 4096 -> 14336 then down 14336 -> 4096, 2048 tokens
-  decoder_70b_prefill_2048     one 70B decoder layer: 4 masked linears + fp32
-                               RMSNorm / attention / SwiGLU / residuals, 2048 tokens
   decode_70b_sweep             every linear of a 70B layer at 1..256 tokens
 L2 is flushed (256 MiB write) between timed steps.
 
@@ -40,7 +42,8 @@ from paper_2607_29221_gb300 import workloads as wl  # noqa: E402
 
 METRIC = "masked ring-GEMM effective TOPS (Z_2^32) and masked-layer tokens/s; % of roofline"
 L2_FLUSH_BYTES = 256 << 20
-DEFAULT_WORKLOAD = "attn_proj_7b_512x4096x4096"
+DEFAULT_WORKLOAD = "decoder_70b_prefill_2048"
+DECODER_SEED = 11          # weights of the decoder layer: seeds 11..14 (QKV, O, gate+up, down)
 
 
 def _peaks():
@@ -53,19 +56,32 @@ def _peaks():
         return 6800.0, 1900.0, 1700.0, "fallback"
 
 
-def _traffic(kernel: str):
-    """DRAM bytes per launch from the committed ncu capture (profiles/traffic.json),
-    or None if the kernel's source changed since the capture."""
+def _traffic(kernel: str, workload: str):
+    """DRAM bytes of `kernel` per step of `workload` from the committed ncu
+    capture (profiles/traffic.json), or None if there is none or the kernel's
+    source changed since the capture."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
-            rec = json.load(f)[kernel]
+            rec = json.load(f)[f"{kernel}@{workload}"]
         with open(os.path.join(ROOT, rec["source"]), "rb") as f:
             if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
                 return None
-        return float(rec["dram_bytes_per_launch"])
+        return float(rec["dram_bytes_per_step"])
     except Exception:
         return None
+
+
+def _config(wk, world):
+    """The workload as both arms report it (the JSON line's `config`)."""
+    cfg = {"workload": wk.name, "l": wk.l,
+           "linears": [{"name": x.name, "m": x.m, "n": x.n} for x in wk.linears],
+           "params": "Example 3.1: d=3, r=1536/1024/652, t=80/80, sigma=0.5, b=16",
+           "l2": "flushed between timed steps (256 MiB write)",
+           "parallelism": f"replicas x{world}"}
+    if wk.name == "decoder_70b_prefill_2048":
+        cfg["glue"] = "fp32 RMSNorm, causal GQA attention (64 q / 8 kv heads, d 128), SwiGLU, residuals"
+    return cfg
 
 
 def parse():
@@ -142,27 +158,65 @@ class ClockSampler:
 # workloads
 # ---------------------------------------------------------------------------
 class _Timed:
-    """CUDA events around the server products of the steps being timed."""
+    """CUDA events around the server products and the encodes of the steps
+    being timed (on the launching stream)."""
 
     def __init__(self, stream):
         self.stream = stream
         self.active = False
-        self.pairs = []
+        self.pairs = {"server": [], "encode": []}
 
-    def wrap(self, layer):
+    def _wrap(self, fn, key):
         import torch
-        server = layer.server
 
-        def timed_server(*a, **k):
+        def timed(*a, **k):
             if not self.active:
-                return server(*a, **k)
+                return fn(*a, **k)
             e0 = torch.cuda.Event(enable_timing=True); e1 = torch.cuda.Event(enable_timing=True)
             e0.record(self.stream)
-            out = server(*a, **k)
+            out = fn(*a, **k)
             e1.record(self.stream)
-            self.pairs.append((e0, e1))
+            self.pairs[key].append((e0, e1))
             return out
-        layer.server = timed_server
+        return timed
+
+    def wrap(self, layer):
+        layer.server = self._wrap(layer.server, "server")
+        layer.mask_input = self._wrap(layer.mask_input, "encode")
+
+    def ms(self, key, steps):
+        p = self.pairs[key]
+        return float(np.sum([a.elapsed_time(b) for a, b in p])) / steps if p else 0.0
+
+    def clear(self):
+        for v in self.pairs.values():
+            v.clear()
+
+
+class _Parts:
+    """mark(part) records a CUDA event where a part of the step begins; the
+    time to the next mark is charged to that part."""
+
+    def __init__(self, stream):
+        self.stream = stream
+        self.evs = []
+
+    def __call__(self, name):
+        import torch
+        e = torch.cuda.Event(enable_timing=True)
+        e.record(self.stream)
+        self.evs.append((name, e))
+
+    def totals(self):
+        out = {}
+        for (n, a), (_, b) in zip(self.evs[:-1], self.evs[1:]):
+            if n != "end":
+                out[n] = out.get(n, 0.0) + a.elapsed_time(b)
+        return out
+
+
+def _no_mark(name):
+    return None
 
 
 class LinearChain:
@@ -193,13 +247,29 @@ class LinearChain:
                 Y=torch.empty(l, lin.m, dtype=torch.float32, device=dev)))
         self.ring_macs = sum(l * (ly.m + proto.sum_r) * ly.n_pad for ly in self.layers)
         self.n_in, self.m_out = linears[0].n, linears[-1].m
+        self.masks = [ly.init_x(l, 900_000 + c) for c, ly in enumerate(self.layers)]
 
-    def step(self, x, i):
+    def step(self, x, i, mark=None):
+        mark = mark or _no_mark
         for c, (layer, bf) in enumerate(zip(self.layers, self.bufs)):
-            mp = layer.init_x(self.l, 1_000_000 * self.rank + 1000 * c + i)
+            mark("init_x")
+            mp = layer.init_x(self.l, 1_000_000 * self.rank + 1000 * c + i, out=self.masks[c])
+            mark("encode")
             layer.mask_input(x, mp, bf["Xp"], bf["s_x"], bf["Xpl"])
+            mark("server")
             layer.server(bf["Xp"], bf["Xpl"], bf["Z"])
+            mark("unmask")
             layer.unmask(bf["Z"], mp, bf["s_x"], bf["Y"])
+            x = bf["Y"]
+        return x
+
+    def _pass(self, x, mps, ctr, side):
+        from paper_2607_29221_gb300 import mosaic as M
+        for c, (layer, bf) in enumerate(zip(self.layers, self.bufs)):
+            layer.mask_input(x, mps[c], bf["Xp"], bf["s_x"], bf["Xpl"])
+            layer.server(bf["Xp"], bf["Xpl"], bf["Z"])
+            layer.unmask(bf["Z"], mps[c], bf["s_x"], bf["Y"])
+            M.mosaic_advance_pass(ctr[c], 1, stream=side)
             x = bf["Y"]
         return x
 
@@ -208,32 +278,25 @@ class LinearChain:
         a base plus a device counter that the graph advances, so every replay
         draws fresh masks (pass ids disjoint from the eager steps')."""
         import torch
-        from paper_2607_29221_gb300 import mosaic as M
         dev = x.device
         base = [1_000_000 * self.rank + 500_000 + 1000 * c for c in range(len(self.layers))]
-        self.ctr = [torch.zeros(1, dtype=torch.int64, device=dev) for _ in self.layers]
-        self.gmask = [ly.init_x(self.l, b) for ly, b in zip(self.layers, base)]   # buffers, workspace sized
+        ctr = [torch.zeros(1, dtype=torch.int64, device=dev) for _ in self.layers]
+        gmask = [ly.init_x(self.l, b) for ly, b in zip(self.layers, base)]   # buffers, workspace sized
         torch.cuda.synchronize()
         side = torch.cuda.Stream()
         side.wait_stream(torch.cuda.current_stream())
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=side):
-            for c, (layer, bf) in enumerate(zip(self.layers, self.bufs)):
-                mp = layer.init_x(self.l, base[c], pass_dev=self.ctr[c], out=self.gmask[c])
-                layer.mask_input(x, mp, bf["Xp"], bf["s_x"], bf["Xpl"])
-                layer.server(bf["Xp"], bf["Xpl"], bf["Z"])
-                layer.unmask(bf["Z"], mp, bf["s_x"], bf["Y"])
-                M.mosaic_advance_pass(self.ctr[c], 1, stream=side)
-                x = bf["Y"]
+            mps = [ly.init_x(self.l, base[c], pass_dev=ctr[c], out=gmask[c]) for c, ly in enumerate(self.layers)]
+            y = self._pass(x, mps, ctr, side)
         torch.cuda.synchronize()
-        return g
+        return g, y
 
     def graph_e2e(self, X, X_host, Y_host):
         """The step with its host copies as one CUDA graph: the copy of X in
         runs on a forked stream beside every layer's Init X (which does not
         depend on X), the copy of Y out ends the graph."""
         import torch
-        from paper_2607_29221_gb300 import mosaic as M
         dev = X.device
         base = [1_000_000 * self.rank + 700_000 + 1000 * c for c in range(len(self.layers))]
         ctr = [torch.zeros(1, dtype=torch.int64, device=dev) for _ in self.layers]
@@ -248,14 +311,8 @@ class LinearChain:
                 X.copy_(X_host, non_blocking=True)
             mps = [ly.init_x(self.l, base[c], pass_dev=ctr[c], out=gmask[c]) for c, ly in enumerate(self.layers)]
             side.wait_stream(copy)
-            x = X
-            for c, (layer, bf) in enumerate(zip(self.layers, self.bufs)):
-                layer.mask_input(x, mps[c], bf["Xp"], bf["s_x"], bf["Xpl"])
-                layer.server(bf["Xp"], bf["Xpl"], bf["Z"])
-                layer.unmask(bf["Z"], mps[c], bf["s_x"], bf["Y"])
-                M.mosaic_advance_pass(ctr[c], 1, stream=side)
-                x = bf["Y"]
-            Y_host.copy_(x, non_blocking=True)
+            y = self._pass(X, mps, ctr, side)
+            Y_host.copy_(y, non_blocking=True)
         torch.cuda.synchronize()
         return g
 
@@ -266,15 +323,65 @@ class DecoderLayerRun:
     def __init__(self, proto, dev, l, rank, timed):
         from paper_2607_29221_gb300 import decoder as D
         s = D.LayerShape()
-        self.layer = D.SecureDecoderLayer(proto, D.LayerWeights(s, seed=11, device=dev))
-        for lin in self.layer.linears():
+        self.layer = D.SecureDecoderLayer(proto, D.LayerWeights(s, seed=DECODER_SEED, device=dev))
+        self.layers = self.layer.linears()
+        for lin in self.layers:
             timed.wrap(lin)
-        self.ring_macs = sum(l * (lin.m + proto.sum_r) * lin.n_pad for lin in self.layer.linears())
+        self.layer.alloc(l)
+        self.ring_macs = sum(l * (lin.m + proto.sum_r) * lin.n_pad for lin in self.layers)
         self.n_in = self.m_out = s.hidden
-        self.l = l
+        self.l, self.rank = l, rank
+        self.masks = self.layer.init_x(l, 90_000)
 
-    def step(self, x, i):
-        return self.layer.forward(x)
+    def step(self, x, i, mark=None):
+        mark = mark or _no_mark
+        mark("init_x")
+        masks = self.layer.init_x(self.l, 100_000 * self.rank + i, out=self.masks)
+        return self.layer.forward(x, masks, mark=mark)
+
+    def graph(self, x):
+        """The layer's step captured as one CUDA graph (fresh masks per replay
+        from a device pass counter)."""
+        import torch
+        from paper_2607_29221_gb300 import mosaic as M
+        base = 100_000 * self.rank + 50_000
+        ctr = torch.zeros(1, dtype=torch.int64, device=x.device)
+        gm = self.layer.init_x(self.l, base)
+        torch.cuda.synchronize()
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            masks = self.layer.init_x(self.l, base, pass_dev=ctr, out=gm)
+            y = self.layer.forward(x, masks)
+            M.mosaic_advance_pass(ctr, 1, stream=side)
+        torch.cuda.synchronize()
+        return g, y
+
+    def graph_e2e(self, X, X_host, Y_host):
+        """The step with its host copies as one CUDA graph: the copy of X in
+        runs on a forked stream beside the four calls' Init X (independent of
+        X), the copy of Y out ends the graph."""
+        import torch
+        from paper_2607_29221_gb300 import mosaic as M
+        base = 100_000 * self.rank + 70_000
+        ctr = torch.zeros(1, dtype=torch.int64, device=X.device)
+        gm = self.layer.init_x(self.l, base)
+        torch.cuda.synchronize()
+        side, copy = torch.cuda.Stream(), torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            copy.wait_stream(side)
+            with torch.cuda.stream(copy):
+                X.copy_(X_host, non_blocking=True)
+            masks = self.layer.init_x(self.l, base, pass_dev=ctr, out=gm)
+            side.wait_stream(copy)
+            y = self.layer.forward(X, masks)
+            M.mosaic_advance_pass(ctr, 1, stream=side)
+            Y_host.copy_(y, non_blocking=True)
+        torch.cuda.synchronize()
+        return g
 
 
 def _time_steps(torch, runner, make_input, steps, warmup, flush, stream, timed, world, counter=None):
@@ -299,9 +406,18 @@ def _time_steps(torch, runner, make_input, steps, warmup, flush, stream, timed, 
     torch.cuda.synchronize()
     _barrier(world)
     step_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
-    gemm_ms = float(np.sum([a.elapsed_time(b) for a, b in timed.pairs])) / steps if timed.pairs else 0.0
-    timed.pairs.clear()
-    return step_ms, gemm_ms, launches
+    gemm_ms = timed.ms("server", steps)
+    enc_ms = timed.ms("encode", steps)
+    timed.clear()
+    return step_ms, gemm_ms, launches, enc_ms
+
+
+class _Replay:
+    def __init__(self, g):
+        self.g = g
+
+    def step(self, x_unused, i):
+        self.g.replay()
 
 
 def run_mine(args, rank, world):
@@ -350,56 +466,54 @@ def run_mine(args, rank, world):
     sampler = ClockSampler(_smi_index(dev.index))
     sampler.start()
     time.sleep(0.3)
-    # our kernels launched inside the timed region, from the library's own counter
-    eager_ms, gemm_ms, launches_timed = _time_steps(torch, runner, lambda: X, args.steps, args.warmup, flush,
-                                                    stream, timed, world, M.mosaic_kernel_launches)
-    step_ms = eager_ms
-    graph_ms = None
-    if isinstance(runner, LinearChain):
-        # The step as one CUDA graph (same kernels; replays draw fresh passes).
-        g = runner.graph(X)
-
-        class _Replay:
-            def step(self, x_unused, i):
-                g.replay()
-
-        graph_ms, _, _ = _time_steps(torch, _Replay(), lambda: X, args.steps, args.warmup, flush, stream,
-                                     timed, world)
-        step_ms = graph_ms
-        del g
-
-    # end to end through the public API with host buffers
-    Y_host = torch.empty(l, runner.m_out, dtype=torch.float32).pin_memory()
-    e2e = []
-    for i in range(max(3, args.steps // 2)):
+    # Eager steps: our kernels launched inside the timed region (the library's
+    # own counter), and CUDA events around every server product and encode.
+    eager_ms, gemm_ms, launches_timed, enc_ms = _time_steps(
+        torch, runner, lambda: X, args.steps, args.warmup, flush, stream, timed, world,
+        M.mosaic_kernel_launches)
+    # The step as one CUDA graph (same kernels; replays draw fresh passes).
+    g, _ = runner.graph(X)
+    step_ms, _, _, _ = _time_steps(torch, _Replay(g), lambda: X, args.steps, args.warmup, flush, stream,
+                                   timed, world)
+    del g
+    # Where the step's time goes: CUDA events where each part begins (eager).
+    part_steps = max(3, args.steps // 4)
+    parts = _Parts(stream)
+    for i in range(part_steps):
         flush.fill_(i & 0xFF)
-        a = torch.cuda.Event(enable_timing=True); c = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        X.copy_(X_host, non_blocking=True)
-        Y = runner.step(X, 10_000 + i)
-        Y_host.copy_(Y, non_blocking=True)
-        c.record(stream)
-        e2e.append((a, c))
+        runner.step(X, 20_000 + i, mark=parts)
+        parts("end")
     torch.cuda.synchronize()
-    e2e_ms = float(np.mean([a.elapsed_time(c) for a, c in e2e]))
-    e2e_eager_ms = e2e_ms
-    if isinstance(runner, LinearChain):
-        # The same through one CUDA graph per step, the copy of X overlapping Init X.
-        ge = runner.graph_e2e(X, X_host, Y_host)
-        for i in range(3):
-            ge.replay()
-        torch.cuda.synchronize()
-        e2e = []
-        for i in range(max(3, args.steps // 2)):
+    part_ms = {k: round(v / part_steps, 4) for k, v in parts.totals().items()}
+
+    # End to end through the public API with host buffers: the copy of X in
+    # and of Y out inside the timed region, every step.
+    Y_host = torch.empty(l, runner.m_out, dtype=torch.float32).pin_memory()
+    e2e_steps = max(3, args.steps // 2)
+
+    def _e2e(step_fn):
+        ev = []
+        for i in range(e2e_steps):
             flush.fill_(i & 0xFF)
             a = torch.cuda.Event(enable_timing=True); c = torch.cuda.Event(enable_timing=True)
             a.record(stream)
-            ge.replay()
+            step_fn(i)
             c.record(stream)
-            e2e.append((a, c))
+            ev.append((a, c))
         torch.cuda.synchronize()
-        e2e_ms = float(np.mean([a.elapsed_time(c) for a, c in e2e]))
-        del ge
+        return float(np.mean([a.elapsed_time(c) for a, c in ev]))
+
+    def _eager_e2e(i):
+        X.copy_(X_host, non_blocking=True)
+        Y = runner.step(X, 10_000 + i)
+        Y_host.copy_(Y, non_blocking=True)
+    e2e_eager_ms = _e2e(_eager_e2e)
+    ge = runner.graph_e2e(X, X_host, Y_host)
+    for i in range(3):
+        ge.replay()
+    torch.cuda.synchronize()
+    e2e_ms = _e2e(lambda i: ge.replay())
+    del ge
     clocks = sampler.stop()
     M.mosaic_device_status()
 
@@ -414,38 +528,43 @@ def run_mine(args, rank, world):
     tokens_s = world * l / (step_ms_max / 1e3)
     ring_tops = 2 * runner.ring_macs / (gemm_ms / 1e3) / 1e12
     roof = _roofline(variant, M, runner.ring_macs, gemm_ms, bf16, peak_src,
-                     _traffic("ring_gemm_tc") if args.workload == DEFAULT_WORKLOAD and variant == M.GEMM_TC
-                     else None)
-    cfg = {"workload": args.workload, "l": l,
-           "linears": [{"name": x.name, "m": x.m, "n": x.n} for x in wk.linears],
-           "params": "Example 3.1: d=3, r=1536/1024/652, t=80/80, sigma=0.5, b=16",
-           "gemm_variant": {M.GEMM_TC: "tc", M.GEMM_MMA_S8: "mma_s8", M.GEMM_IMAD: "imad"}[variant],
-           "l2": "flushed between timed steps (256 MiB write)",
-           "parallelism": f"replicas x{world}",
-           "launch": "one CUDA graph per step (fresh pass ids from a device counter)" if graph_ms is not None
-                     else "eager"}
-    if args.workload == "decoder_70b_prefill_2048":
-        cfg["glue"] = "fp32 RMSNorm, causal GQA attention (64 q / 8 kv heads, d 128), SwiGLU, residuals"
+                     _traffic("ring_gemm_tc", args.workload) if variant == M.GEMM_TC else None)
+    roof["per"] = (f"the {len(runner.layers)} server-product launches of one step"
+                   if len(runner.layers) > 1 else "one server-product launch")
+    if variant == M.GEMM_TC:
+        roof["frac_of_sustained"] = round(roof["achieved"] / bf16_sus, 4)
+    enc_bytes = sum(l * (4 * ly.n + (16 if ly.use_planes and l > M.SKINNY_MAX_M else 8) * ly.n_pad)
+                    for ly in runner.layers)
+    enc_gbs = enc_bytes / (enc_ms / 1e3) / 1e9 if enc_ms > 0 else 0.0
+    rooflines = [dict(roof, kernel=roof["kernel"]),
+                 {"kernel": "fwht_kernel (encode: rotate, quantise, + U_x, digit planes)", "bound": "hbm",
+                  "achieved": round(enc_gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(enc_gbs / hbm, 4),
+                  "traffic": None, "bytes_per_step": enc_bytes, "ms_per_step": round(enc_ms, 4),
+                  "peak_source": f"{peak_src} copy bandwidth"}]
     out = {
         "metric": METRIC, "value": round(tokens_s, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms_max, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
         "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights)",
-        "config": cfg,
+        "config": _config(wk, world),
+        "implementation": {"gemm_variant": {M.GEMM_TC: "tc", M.GEMM_MMA_S8: "mma_s8",
+                                            M.GEMM_IMAD: "imad"}[variant],
+                           "launch": "one CUDA graph per step (fresh pass ids from a device counter)"},
         "ms_per_step_eager": round(eager_ms_max, 4),
+        "parts_ms_per_step": part_ms,
         "ring_tops": round(ring_tops, 2),
         "gemm_ms": round(gemm_ms, 4),
         "init_w_s": round(init_w_s, 3),
         "roofline": roof,
+        "rooflines": rooflines,
         "e2e": {"value": round(world * l / (e2e_ms_max / 1e3), 1), "unit": "tokens/s",
                 "h2d_bytes_per_step": l * runner.n_in * 4, "d2h_bytes_per_step": l * runner.m_out * 4,
-                "launch": "one CUDA graph per step, the copy of X overlapping Init X"
-                          if isinstance(runner, LinearChain) else "eager",
+                "launch": "one CUDA graph per step, the copy of X overlapping Init X",
                 "value_eager": round(world * l / (e2e_eager_ms_max / 1e3), 1)},
         "gpu_launches": int(launches_timed),
         "clocks": clocks,
     }
-    if world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD:
+    if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(wk, args.cpu_budget_s)
     print(json.dumps(out), flush=True)
 
@@ -515,7 +634,7 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
                     ly.unmask(bf["Z"], part, bf["s_x"], bf["Y"])
 
         runner = _Online()
-        eager_ms, gemm_ms, launches = _time_steps(torch, runner, lambda: None, args.steps, args.warmup, flush,
+        eager_ms, gemm_ms, launches, _ = _time_steps(torch, runner, lambda: None, args.steps, args.warmup, flush,
                                                   stream, timed, world, M.mosaic_kernel_launches)
         # The same steps as CUDA graphs (one per step: each reads its own rows
         # of the drawn masks), replayed without the Python launch overhead.
@@ -529,11 +648,11 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
             graphs.append(g)
         torch.cuda.synchronize()
 
-        class _Replay:
+        class _StepReplay:
             def step(self, x_unused, i):
                 graphs[i % nsteps].replay()
 
-        online_ms, _, _ = _time_steps(torch, _Replay(), lambda: None, args.steps, args.warmup, flush, stream,
+        online_ms, _, _, _ = _time_steps(torch, _StepReplay(), lambda: None, args.steps, args.warmup, flush, stream,
                                       timed, world)
         del graphs
         step_ms = online_ms + initx_ms
@@ -850,76 +969,120 @@ def _max_over_ranks(v, world, dev):
 # ---------------------------------------------------------------------------
 # CPU oracle as baseline / reference arm
 # ---------------------------------------------------------------------------
-def _oracle_setup(wk):
+ORACLE_TOKENS = 16           # tokens per sampled oracle step
+ORACLE_ROWS = 256            # output rows per linear where Init W in full is out of reach
+ORACLE_FULL_INIT_MACS = 6e10  # Init W (J = (W_hat + E_w) C) up to this many MACs runs on every row
+
+
+def _linear_weights_seed(wk, i):
+    """Seed and std of linear i's float weights, as the GPU arm draws them."""
+    if wk.name == "decoder_70b_prefill_2048":
+        return DECODER_SEED + i, 0.02
+    return wl.SEED_W + i, wk.linears[i].w_std
+
+
+def _oracle_setup(wk, tokens):
+    """One-time oracle state of every linear of the workload: the public chains
+    in full, and Init W on all rows or on ORACLE_ROWS evenly spaced rows
+    (oracle.sampled).  Not timed (the GPU arm's Init W is timed apart too)."""
     import oracle as O
-    lin = wk.linears[0]
-    m, n = lin.m, lin.n
-    n_pad = 1 << max(0, (n - 1).bit_length())
+    from oracle import sampled as OS
     key = wl.mask_key()
     p = O.Params()
+    chains = {}
+    plan = []
     t0 = time.perf_counter()
-    P, C = O.chains(key, p, n_pad)
-    W = wl.weights(m, n, std=lin.w_std)
-    ws = O.init_w(key, p, W, 1, P, C, n_pad)
-    return O, key, p, P, C, ws, time.perf_counter() - t0
+    for i, lin in enumerate(wk.linears):
+        n_pad = 1 << max(5, (lin.n - 1).bit_length())
+        if n_pad not in chains:
+            chains[n_pad] = O.chains(key, p, n_pad)
+        P, C = chains[n_pad]
+        if lin.m * n_pad * sum(p.r) <= ORACLE_FULL_INIT_MACS:
+            rows = np.arange(lin.m)
+        else:
+            rows = np.unique(np.linspace(0, lin.m - 1, ORACLE_ROWS).astype(np.int64))
+        seed, std = _linear_weights_seed(wk, i)
+        W_rows = wl.weight_rows(lin.m, lin.n, rows, seed=seed, std=std)
+        wr = OS.weight_rows(key, p, W_rows, rows, 1 + i, P, C, n_pad)
+        X = wl.activations(tokens, lin.n, seed=wl.SEED_X + i)
+        b = wl.bias(lin.m, seed=wl.SEED_B + i)[rows]
+        plan.append(dict(lin=lin, n_pad=n_pad, P=P, C=C, wr=wr, X=X, b=b, rows=rows))
+    return O, OS, key, p, plan, time.perf_counter() - t0
 
 
-def _oracle_step(O, key, p, P, C, ws, X, pass_id, b):
-    ps = O.init_x(key, p, X.shape[1], pass_id, C, ws.J, ws.n_pad)
-    _, s_x, Xm = O.mask_input(X, ws, ps.U_x)
-    Ym, Q = O.server(ws, P, Xm)
-    Yh = O.unmask(p, ws, ps, Ym, Q)
-    return O.decode(Yh, ws.s_w, s_x, b)
+def _oracle_step(O, OS, key, p, plan, pass_id):
+    """One sampled oracle step: every linear's Init X, encode + mask-add, server
+    product, unmask and decode for the sample's tokens, over the sampled rows.
+    Returns the seconds the whole step (all rows) takes for those tokens: the
+    per-token part (Init X draws and U_x, encode, Q_i = P_i X') as measured,
+    the per-(row, token) part (K, Y', unmask, decode) scaled by m / rows."""
+    total = 0.0
+    for st in plan:
+        k = st["X"].shape[0]
+        wr = st["wr"]
+        t0 = time.perf_counter()
+        tc = OS.token_cols(key, p, st["X"], np.arange(k), pass_id, wr.sign_words, wr.qmax, st["C"], st["n_pad"])
+        Q = OS.server_q(tc, st["P"])
+        t1 = time.perf_counter()
+        K = OS.k_entries(p, wr, tc)
+        Ym = OS.server_rows(wr, tc)
+        Yh = OS.unmask_entries(p, wr, K, Ym, Q)
+        O.decode(Yh, wr.s_w, tc.s_x, st["b"])
+        t2 = time.perf_counter()
+        total += (t1 - t0) + (t2 - t1) * st["lin"].m / len(st["rows"])
+    return total
 
 
-def cpu_baseline(wk, budget_s, tokens=None):
-    O, key, p, P, C, ws, init_s = _oracle_setup(wk)
-    l = wk.l if tokens is None else tokens
-    X = wl.activations(l, wk.linears[0].n).T.copy()
-    b = wl.bias(wk.linears[0].m)
-    done, t0 = 0, time.perf_counter()
+def _oracle_sample_text(wk, plan, k, extra=""):
+    rows = ", ".join(f"{st['lin'].name} {len(st['rows'])}/{st['lin'].m}" for st in plan)
+    glue = "; fp32 glue not included" if wk.name == "decoder_70b_prefill_2048" else ""
+    return (f"{k} of {wk.l} tokens per step through every linear (rows computed: {rows}); "
+            f"per-token work (Init X draws, U_x, encode, Q_i = P_i X') timed as run, per-(row, token) "
+            f"work (K, Y', unmask, decode) scaled by m / rows computed{glue}; seeded N(0,1) inputs of "
+            f"each linear's width; one-time chains + Init W excluded like the GPU value{extra}")
+
+
+def cpu_baseline(wk, budget_s):
+    O, OS, key, p, plan, init_s = _oracle_setup(wk, ORACLE_TOKENS)
+    k = ORACLE_TOKENS
+    done, secs, t0 = 0, 0.0, time.perf_counter()
     while True:
-        _oracle_step(O, key, p, P, C, ws, X, 500 + done, b)
+        secs += _oracle_step(O, OS, key, p, plan, 500 + done)
         done += 1
         if time.perf_counter() - t0 >= budget_s:
             break
-    dt = time.perf_counter() - t0
-    return {"value": round(done * l / dt, 2), "unit": "tokens/s", "cores": O.num_threads(),
+    return {"value": round(done * k / secs, 3), "unit": "tokens/s", "cores": O.num_threads(),
             "kind": "oracle",
-            "sample": f"{done} full per-call steps of {l} tokens ({wk.name}); one-time chains + Init W "
-                      f"({init_s:.1f} s) excluded like the GPU value",
+            "sample": _oracle_sample_text(wk, plan, k, f" ({done} sampled steps, {init_s:.1f} s of setup)"),
             "init_w_s": round(init_s, 2)}
 
 
 def run_reference(args, rank, world):
+    """The reference arm: the oracle as it stands, on the host cores, on the
+    same workload, metric and config as the GPU arm; each step one sampled
+    oracle step (rank 0 only)."""
     if rank != 0:
         return
-    wk = wl.WORKLOADS[DEFAULT_WORKLOAD if args.workload not in (DEFAULT_WORKLOAD,) else args.workload]
-    O, key, p, P, C, ws, init_s = _oracle_setup(wk)
-    lin = wk.linears[0]
-    l = min(wk.l, 64)               # bounded sample of the workload's tokens per step
-    X = wl.activations(l, lin.n).T.copy()
-    b = wl.bias(lin.m)
+    wk = wl.WORKLOADS[args.workload]
+    if not wk.linears or wk.l < 1 or wk.name in ("decode_70b_sweep", "matvec_sweep", "sigma_sweep_7b",
+                                                  "kernels_hbm", "init_w_70b"):
+        print(json.dumps({"impl": "reference", "unavailable": f"no oracle step for workload {wk.name}"}))
+        return
+    O, OS, key, p, plan, init_s = _oracle_setup(wk, ORACLE_TOKENS)
+    k = ORACLE_TOKENS
     for i in range(args.warmup):
-        _oracle_step(O, key, p, P, C, ws, X, 900 + i, b)
-    times = []
-    for i in range(args.steps):
-        t0 = time.perf_counter()
-        _oracle_step(O, key, p, P, C, ws, X, 950 + i, b)
-        times.append(time.perf_counter() - t0)
-    sec = float(np.mean(times))
-    val = l / sec
-    out = {"impl": "reference", "metric": METRIC, "value": round(val, 2), "unit": "tokens/s",
+        _oracle_step(O, OS, key, p, plan, 900 + i)
+    secs = [_oracle_step(O, OS, key, p, plan, 950 + i) for i in range(args.steps)]
+    val = k / float(np.mean(secs))
+    out = {"impl": "reference", "metric": METRIC, "value": round(val, 3), "unit": "tokens/s",
            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-           "ms_per_step": round(sec * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+           "ms_per_step": round(wk.l / val * 1e3, 3), "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "u32", "data": "synthetic",
-           "config": {"workload": wk.name, "l": wk.l, "m": lin.m, "n": lin.n,
-                      "params": "Example 3.1"},
-           "cpu_baseline": {"value": round(val, 2), "unit": "tokens/s", "cores": O.num_threads(),
-                            "kind": "oracle",
-                            "sample": f"{l} of {wk.l} tokens per step; one-time chains + Init W "
-                                      f"({init_s:.1f} s) excluded"},
-           "e2e": {"value": round(val, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+           "config": _config(wk, world),
+           "cpu_baseline": {"value": round(val, 3), "unit": "tokens/s", "cores": O.num_threads(),
+                            "kind": "oracle", "sample": _oracle_sample_text(wk, plan, k,
+                                                                            f" ({init_s:.1f} s of setup)")},
+           "e2e": {"value": round(val, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
 

@@ -325,6 +325,62 @@ mosaic_status mosaic_mask_activation_ex(const mosaic_params *p, const mosaic_key
 /* *pass_dev += delta, enqueued on `stream` (one-thread kernel). */
 mosaic_status mosaic_advance_pass(uint64_t *pass_dev, uint64_t delta, void *stream);
 
+/* One entry point for the three mask-generation roles of the protocol box
+ * (Sec. 3.2, Pi_Sec-Approx-MatMul: Init W steps 1-3 and 5, Init X steps
+ * 1a-1c; eq. weight-mask and eq. activation-mask).  The roles take different
+ * operands -- the public chains are made once per input width, the weight
+ * mask consumes a float matrix and yields seven client/server outputs, the
+ * activation mask consumes the chains and J and yields U_x and K per pass --
+ * so the role-specific buffers travel in one struct and `kind` selects the
+ * role.  Each kind is exactly the role call named below (same validation,
+ * same results, same workspace size); fields a kind does not name are
+ * ignored.
+ *
+ *   kind                    stream_id    rows   l       fields used              same as
+ *   MOSAIC_MASK_CHAINS      chain id     --     --      P, C, CT (outputs)       mosaic_mask_chains
+ *   MOSAIC_MASK_WEIGHT      matrix id    m      --      W, ldw, n, P, CT (in);   mosaic_mask_weight
+ *                                                       sign_words, s_w, L, S_idx,
+ *                                                       S_val, Wp, Wp_planes
+ *                                                       (nullable), J (out)
+ *   MOSAIC_MASK_ACTIVATION  pass id      m      tokens  C, J, cj_planes          mosaic_mask_activation_ex
+ *                                                       (nullable), pass_dev
+ *                                                       (nullable) (in);
+ *                                                       Ux_tm, K_tm (out)
+ *
+ * `variant` is used by WEIGHT and ACTIVATION.  Returns MOSAIC_ERR_ARG for an
+ * unknown kind or a null `io`; otherwise the status of the role call.
+ * ws: mosaic_workspace_bytes(MOSAIC_OP_MASK_CHAINS / _WEIGHT / _ACTIVATION, ...). */
+typedef enum {
+    MOSAIC_MASK_CHAINS = 1,
+    MOSAIC_MASK_WEIGHT = 2,
+    MOSAIC_MASK_ACTIVATION = 3
+} mosaic_mask_kind;
+
+typedef struct {
+    const float *W;            /* WEIGHT: m x n float weights, leading dimension ldw */
+    int64_t ldw;
+    int64_t n;                 /* WEIGHT: columns of W (n <= n_pad)                  */
+    uint32_t *P;               /* Sr x n_pad: CHAINS out, WEIGHT in                  */
+    uint32_t *C;               /* n_pad x Sr: CHAINS out, ACTIVATION in              */
+    uint32_t *CT;              /* Sr x n_pad: CHAINS out, WEIGHT in                  */
+    uint32_t *sign_words;      /* WEIGHT out (n_pad / 32)                            */
+    float *s_w;                /* WEIGHT out (m)                                     */
+    uint32_t *L;               /* WEIGHT out (m x r_d)                               */
+    uint32_t *S_idx;           /* WEIGHT out                                         */
+    uint32_t *S_val;           /* WEIGHT out                                         */
+    uint32_t *Wp;              /* WEIGHT out ((m + Sr) x n_pad)                      */
+    uint16_t *Wp_planes;       /* WEIGHT out, nullable                               */
+    uint32_t *J;               /* m x Sr: WEIGHT out, ACTIVATION in                  */
+    const uint16_t *cj_planes; /* ACTIVATION in, nullable (mosaic_prepare_activation) */
+    const uint64_t *pass_dev;  /* ACTIVATION in, nullable (device pass counter)      */
+    uint32_t *Ux_tm;           /* ACTIVATION out (l x n_pad)                         */
+    uint32_t *K_tm;            /* ACTIVATION out (l x m)                             */
+} mosaic_mask_io;
+
+mosaic_status mosaic_mask(int kind, const mosaic_params *p, const mosaic_key *key, uint64_t stream_id,
+                          int64_t rows, int64_t n_pad, int64_t l, const mosaic_mask_io *io, int variant,
+                          void *ws, size_t ws_bytes, void *stream);
+
 /* ------------------------------------------------------------------------ */
 /* Unmask and decode (Approx-MatMul Online step 5; Pi_Sec-Linear Online      */
 /* step 3).                                                                  */

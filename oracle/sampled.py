@@ -106,9 +106,19 @@ def k_entries(p: Params, wr: WeightRows, tc: TokenCols) -> np.ndarray:
     return K
 
 
+def server_rows(wr: WeightRows, tc: TokenCols) -> np.ndarray:
+    """Online 3, the weight side: Y' = W' X' at rows x toks."""
+    return matmul(wr.W_masked, tc.X_masked)
+
+
+def server_q(tc: TokenCols, P) -> list:
+    """Online 3, the chain side: Q_i = P_i X' at all r_i x toks."""
+    return [matmul(Pi, tc.X_masked) for Pi in P]
+
+
 def server_entries(wr: WeightRows, tc: TokenCols, P):
     """Online 3: Y' = W' X' at rows x toks, and Q_i = P_i X' at all r_i x toks."""
-    return matmul(wr.W_masked, tc.X_masked), [matmul(Pi, tc.X_masked) for Pi in P]
+    return server_rows(wr, tc), server_q(tc, P)
 
 
 def unmask_entries(p: Params, wr: WeightRows, K, Y_masked, Q) -> np.ndarray:

@@ -644,6 +644,25 @@ mosaic_status mosaic_mask_activation_ex(const mosaic_params *p, const mosaic_key
                                 variant, ws, ws_bytes, stream);
 }
 
+mosaic_status mosaic_mask(int kind, const mosaic_params *p, const mosaic_key *key, uint64_t stream_id,
+                          int64_t rows, int64_t n_pad, int64_t l, const mosaic_mask_io *io, int variant,
+                          void *ws, size_t ws_bytes, void *stream) {
+    if (!io) return MOSAIC_ERR_ARG;
+    switch (kind) {
+    case MOSAIC_MASK_CHAINS:
+        return mosaic_mask_chains(p, key, stream_id, n_pad, io->P, io->C, io->CT, ws, ws_bytes, stream);
+    case MOSAIC_MASK_WEIGHT:
+        return mosaic_mask_weight(p, key, stream_id, io->W, io->ldw, rows, io->n, n_pad, io->P, io->CT,
+                                  io->sign_words, io->s_w, io->L, io->S_idx, io->S_val, io->Wp, io->Wp_planes,
+                                  io->J, variant, ws, ws_bytes, stream);
+    case MOSAIC_MASK_ACTIVATION:
+        return mosaic_mask_activation_ex(p, key, stream_id, io->pass_dev, rows, n_pad, l, io->C, io->J,
+                                         io->cj_planes, io->Ux_tm, io->K_tm, variant, ws, ws_bytes, stream);
+    default:
+        return MOSAIC_ERR_ARG;
+    }
+}
+
 mosaic_status mosaic_advance_pass(uint64_t *pass_dev, uint64_t delta, void *stream) {
     if (!pass_dev) return MOSAIC_ERR_ARG;
     return add_u64(pass_dev, delta, as_stream(stream));

@@ -5,9 +5,28 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/mosaic.h"
 
 namespace mosaic {
+
+// Raises `kern`'s dynamic shared-memory limit to `bytes` on the current device,
+// once per device ordinal (`done` holds one bit per ordinal).  Host threads may
+// race on a first call: each may set the attribute (an idempotent runtime call)
+// and the bit is published atomically.
+template <typename Kernel>
+inline bool ensure_smem_limit(std::atomic<unsigned long long> &done, Kernel kern, size_t bytes, int *dev_out = nullptr) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    if (dev_out) *dev_out = dev;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (done.load(std::memory_order_acquire) & bit) return true;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) != cudaSuccess)
+        return false;
+    done.fetch_or(bit, std::memory_order_acq_rel);
+    return true;
+}
 
 constexpr int kSparseWindow = 65536;   // stream words reserved per sparse row
 constexpr int kMaxGaussBound = 96;     // B = ceil(12 sigma) for sigma <= 8

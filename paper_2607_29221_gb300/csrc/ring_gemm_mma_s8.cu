@@ -191,15 +191,8 @@ mosaic_status ring_gemm_mma_s8(const uint32_t *A, int64_t lda, const uint32_t *B
     MOSAIC_TRY(launch_status());
     split_s8_kernel<<<grid_for(N * (ldp / 4), 256), 256, 0, st>>>(B, ldb, N, K, Bp, ldp, N * ldp);
     MOSAIC_TRY(launch_status());
-    static unsigned long long attr_set = 0;
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return MOSAIC_ERR_CUDA;
-    if (!(attr_set & (1ull << (dev & 63)))) {
-        if (cudaFuncSetAttribute(ring_gemm_s8_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * STAGE_B) !=
-            cudaSuccess)
-            return MOSAIC_ERR_CUDA;
-        attr_set |= 1ull << (dev & 63);
-    }
+    static std::atomic<unsigned long long> attr_set{0};   // one bit per device ordinal
+    if (!ensure_smem_limit(attr_set, ring_gemm_s8_kernel, 2 * STAGE_B)) return MOSAIC_ERR_CUDA;
     S8Args args{Ap, Bp, ldp, M * ldp, N * ldp, C, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)(ldp / TK)};
     const dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
     ring_gemm_s8_kernel<<<grid, THREADS, 2 * STAGE_B, st>>>(args);

@@ -208,16 +208,8 @@ mosaic_status launch_skinny(const uint32_t *A, int64_t lda, const uint32_t *B, i
     using C = SkCfg<MT, RW>;
     CUtensorMap ta, tb;
     if (!make_u32_map(&ta, A, K, M, lda, MT) || !make_u32_map(&tb, B, K, N, ldb, C::BR)) return MOSAIC_ERR_CUDA;
-    static unsigned long long attr_set = 0;   // one bit per device ordinal
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return MOSAIC_ERR_CUDA;
-    const unsigned long long bit = 1ull << (dev & 63);
-    if (!(attr_set & bit)) {
-        if (cudaFuncSetAttribute(ring_gemm_skinny_kernel<MT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 C::SMEM) != cudaSuccess)
-            return MOSAIC_ERR_CUDA;
-        attr_set |= bit;
-    }
+    static std::atomic<unsigned long long> attr_set{0};   // one bit per device ordinal
+    if (!ensure_smem_limit(attr_set, ring_gemm_skinny_kernel<MT, RW>, C::SMEM)) return MOSAIC_ERR_CUDA;
     const int64_t tiles = (N + C::BR - 1) / C::BR;
     const int64_t nk = (K + KC - 1) / KC;
     if (tiles > 0x7fffffff || nk > 0x7fffffff) return MOSAIC_ERR_SHAPE;

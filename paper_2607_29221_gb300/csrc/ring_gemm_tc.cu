@@ -535,16 +535,9 @@ mosaic_status launch_tc(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const
     CUtensorMap ta, tb;
     if (!make_plane_map(&ta, Ap, K, M, ldpa, a_plane, BM) || !make_plane_map(&tb, Bp, K, N, ldpb, b_plane, BN))
         return MOSAIC_ERR_CUDA;
-    static unsigned long long attr_set = 0;   // one bit per device ordinal
+    static std::atomic<unsigned long long> attr_set{0};   // one bit per device ordinal
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return MOSAIC_ERR_CUDA;
-    const unsigned long long bit = 1ull << (dev & 63);
-    if (!(attr_set & bit)) {
-        if (cudaFuncSetAttribute(ring_gemm_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 C::SMEM) != cudaSuccess)
-            return MOSAIC_ERR_CUDA;
-        attr_set |= bit;
-    }
+    if (!ensure_smem_limit(attr_set, ring_gemm_tc_kernel<BN>, C::SMEM, &dev)) return MOSAIC_ERR_CUDA;
     const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = (N + BN - 1) / BN, tiles = tiles_m * tiles_n;
     const int64_t nk = (K + BK - 1) / BK, nchunks = (nk + CHUNK - 1) / CHUNK;
     if (tiles * nchunks > (int64_t)INT32_MAX) return MOSAIC_ERR_SHAPE;   // 32-bit unit numbers

@@ -500,16 +500,9 @@ template <bool LIST_IS_COL, bool CLAMP>
 mosaic_status launch_pgather(const GatherArgs &a, cudaStream_t st) {
     const size_t smem = pgather_smem(a.r, pg_ring<LIST_IS_COL>());
     auto kern = pgather_kernel<LIST_IS_COL, CLAMP>;
-    static unsigned long long attr_set = 0;   // one bit per device ordinal
+    static std::atomic<unsigned long long> attr_set{0};   // one bit per device ordinal
     int dev = 0, sms = 0, per_sm = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return MOSAIC_ERR_CUDA;
-    const unsigned long long bit = 1ull << (dev & 63);
-    if (!(attr_set & bit)) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) !=
-            cudaSuccess)
-            return MOSAIC_ERR_CUDA;
-        attr_set |= bit;
-    }
+    if (!ensure_smem_limit(attr_set, kern, 227 * 1024, &dev)) return MOSAIC_ERR_CUDA;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kPgWarps * 32, smem) != cudaSuccess ||
         per_sm < 1)
@@ -602,16 +595,11 @@ template <bool LIST_IS_COL, bool CLAMP>
 mosaic_status launch_few(const GatherArgs &a, cudaStream_t st) {
     const size_t smem = (size_t)a.g_count * a.r * sizeof(uint32_t);
     auto kern = gather_few_kernel<LIST_IS_COL, CLAMP>;
-    static unsigned long long attr_set = 0;   // one bit per device ordinal
+    static std::atomic<unsigned long long> attr_set{0};   // one bit per device ordinal
     int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
+    if (!ensure_smem_limit(attr_set, kern, 192 * 1024, &dev) ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return MOSAIC_ERR_CUDA;
-    if (!(attr_set & (1ull << (dev & 63)))) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 192 * 1024) != cudaSuccess)
-            return MOSAIC_ERR_CUDA;
-        attr_set |= 1ull << (dev & 63);
-    }
     // Enough warps to stream the lists; every block stages the rows once.
     const int64_t need = (a.nlist + kFewWarps - 1) / kFewWarps;
     const int64_t cap = (int64_t)sms * 4;

@@ -6,18 +6,25 @@ projection and the down projection (the four per-layer calls of Sec. 4.1).
 The non-linear parts stay on the trusted side in plain fp32 on the device, as
 the paper keeps them on the client (attention is local, Sec. 3.2 "Local
 attention computation"): RMSNorm, causal grouped-query attention with a
-softmax, SiLU(gate) * up, and the residual adds.  Rotary position embeddings
-are not described by the paper and are left out.
+softmax (torch's fused scaled-dot-product attention in fp32, causal), SiLU(gate)
+* up, and the residual adds.  Rotary position embeddings are not described by
+the paper and are left out.
 
 Weights are seeded random N(0, 0.02) (the paper's checkpoints are not
 available); RMSNorm weights are 1.
+
+A pass can run with preallocated buffers (``alloc``) and a device pass
+counter, so that the whole layer is captured once as a CUDA graph whose every
+replay draws fresh masks.
 """
 from __future__ import annotations
 
 from dataclasses import dataclass
 
 import torch
+import torch.nn.functional as F
 
+from . import mosaic as M
 from . import protocol as PR
 from . import workloads as wl
 
@@ -41,19 +48,15 @@ def rmsnorm(x: torch.Tensor, eps: float) -> torch.Tensor:
 
 
 def attention(qkv: torch.Tensor, s: LayerShape) -> torch.Tensor:
-    """Causal grouped-query attention in fp32; qkv is l x (H + 2 KV) * d."""
+    """Causal grouped-query attention in fp32; qkv is l x (H + 2 KV) * d,
+    the output l x H d (token-major)."""
     l = qkv.shape[0]
-    q = qkv[:, : s.n_heads * s.head_dim].view(l, s.n_heads, s.head_dim).transpose(0, 1)
-    k = qkv[:, s.n_heads * s.head_dim: (s.n_heads + s.n_kv) * s.head_dim].view(l, s.n_kv, s.head_dim)
-    v = qkv[:, (s.n_heads + s.n_kv) * s.head_dim:].view(l, s.n_kv, s.head_dim)
-    rep = s.n_heads // s.n_kv
-    k = k.transpose(0, 1).repeat_interleave(rep, dim=0)
-    v = v.transpose(0, 1).repeat_interleave(rep, dim=0)
-    scores = torch.matmul(q, k.transpose(1, 2)) * (1.0 / float(s.head_dim) ** 0.5)
-    mask = torch.ones(l, l, dtype=torch.bool, device=qkv.device).triu(1)
-    scores = scores.masked_fill(mask, float("-inf"))
-    out = torch.matmul(torch.softmax(scores, dim=-1), v)            # H x l x d
-    return out.transpose(0, 1).reshape(l, s.n_heads * s.head_dim)
+    H, KV, d = s.n_heads, s.n_kv, s.head_dim
+    q = qkv[:, : H * d].view(l, H, d).transpose(0, 1)
+    k = qkv[:, H * d: (H + KV) * d].view(l, KV, d).transpose(0, 1).repeat_interleave(H // KV, dim=0)
+    v = qkv[:, (H + KV) * d:].view(l, KV, d).transpose(0, 1).repeat_interleave(H // KV, dim=0)
+    out = F.scaled_dot_product_attention(q.unsqueeze(0), k.unsqueeze(0), v.unsqueeze(0), is_causal=True)
+    return out[0].transpose(0, 1).reshape(l, H * d)
 
 
 class LayerWeights:
@@ -67,15 +70,8 @@ class LayerWeights:
         self.Wdown = torch.from_numpy(wl.weights(s.hidden, s.ffn, seed=seed + 3)).to(device)
 
 
-def reference_forward(w: LayerWeights, x: torch.Tensor) -> torch.Tensor:
-    """The same layer with plain fp32 matrix products (no masking, no quantisation)."""
-    s = w.s
-    h = rmsnorm(x, s.eps)
-    a = attention(h @ w.Wqkv.T, s)
-    x = x + a @ w.Wo.T
-    gu = rmsnorm(x, s.eps) @ w.Wgu.T
-    x = x + (torch.nn.functional.silu(gu[:, : s.ffn]) * gu[:, s.ffn:]) @ w.Wdown.T
-    return x
+def _no_mark(name: str) -> None:
+    return None
 
 
 class SecureDecoderLayer:
@@ -99,21 +95,61 @@ class SecureDecoderLayer:
         self.down = PR.SecureLinear(proto, w.Wdown, base + 4, chain(s.ffn))
         self.chains = chains
         self._pass = 0
+        self.bufs = None
 
     def linears(self):
         return [self.qkv, self.o, self.gu, self.down]
 
-    def init_x(self, l: int):
-        """Init X of all four calls of one pass (independent of the activations)."""
-        self._pass += 1
-        return [lin.init_x(l, 1_000_000 * (i + 1) + self._pass) for i, lin in enumerate(self.linears())]
+    def alloc(self, l: int) -> None:
+        """Preallocates every per-pass buffer of the four calls for l tokens."""
+        dev = self.proto.device
+        Sr = self.proto.sum_r
+        self.bufs = []
+        for lin in self.linears():
+            planes = lin.use_planes and l > M.SKINNY_MAX_M
+            self.bufs.append(dict(
+                Xp=torch.empty(l, lin.n_pad, dtype=torch.int32, device=dev),
+                s_x=torch.empty(l, dtype=torch.float32, device=dev),
+                Xpl=torch.empty(4, l, lin.n_pad, dtype=torch.int16, device=dev) if planes else None,
+                Z=torch.empty(l, lin.m + Sr, dtype=torch.int32, device=dev),
+                Y=torch.empty(l, lin.m, dtype=torch.float32, device=dev)))
 
-    def forward(self, x: torch.Tensor, masks=None) -> torch.Tensor:
+    def init_x(self, l: int, pass_base: int | None = None, pass_dev=None, out=None):
+        """Init X of all four calls of one pass (independent of the activations).
+        Call i draws pass pass_base + 1_000_000 i (+ *pass_dev on the device);
+        without pass_base a host counter advances per call."""
+        if pass_base is None:
+            self._pass += 1
+            pass_base = self._pass
+        outs = out if out is not None else [None] * 4
+        return [lin.init_x(l, 1_000_000 * (i + 1) + pass_base, pass_dev=pass_dev, out=outs[i])
+                for i, lin in enumerate(self.linears())]
+
+    def _linear(self, i: int, x: torch.Tensor, mp, mark) -> torch.Tensor:
+        lin = self.linears()[i]
+        b = self.bufs[i] if self.bufs is not None else {}
+        mark("encode")
+        Xp, s_x, Xpl = lin.mask_input(x, mp, b.get("Xp"), b.get("s_x"), b.get("Xpl"))
+        mark("server")
+        Z = lin.server(Xp, Xpl, b.get("Z"))
+        mark("unmask")
+        Y = lin.unmask(Z, mp, s_x, b.get("Y"))
+        mark("glue")
+        return Y
+
+    def forward(self, x: torch.Tensor, masks=None, mark=None) -> torch.Tensor:
+        """One pass over l tokens (x: l x hidden fp32).  `mark(part)`, if given,
+        is called where each part of the pass begins (init_x, encode, server,
+        unmask, glue), e.g. to record CUDA events."""
         s = self.s
-        masks = masks if masks is not None else self.init_x(x.shape[0])
+        mark = mark or _no_mark
+        if masks is None:
+            mark("init_x")
+            masks = self.init_x(x.shape[0])
+        mark("glue")
         h = rmsnorm(x, s.eps)
-        a = attention(self.qkv.forward(h.contiguous(), masks[0]), s)
-        x = x + self.o.forward(a.contiguous(), masks[1])
-        gu = self.gu.forward(rmsnorm(x, s.eps).contiguous(), masks[2])
-        act = torch.nn.functional.silu(gu[:, : s.ffn]) * gu[:, s.ffn:]
-        return x + self.down.forward(act.contiguous(), masks[3])
+        a = attention(self._linear(0, h, masks[0], mark), s)
+        x = x + self._linear(1, a, masks[1], mark)
+        gu = self._linear(2, rmsnorm(x, s.eps), masks[2], mark)
+        act = F.silu(gu[:, : s.ffn]) * gu[:, s.ffn:]
+        return x + self._linear(3, act, masks[3], mark)

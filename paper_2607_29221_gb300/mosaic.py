@@ -43,6 +43,18 @@ class mosaic_key(ctypes.Structure):
     _fields_ = [("key", ctypes.c_uint32 * 8)]
 
 
+MASK_CHAINS, MASK_WEIGHT, MASK_ACTIVATION = 1, 2, 3
+
+
+class mosaic_mask_io(ctypes.Structure):
+    _fields_ = [("W", ctypes.c_void_p), ("ldw", ctypes.c_int64), ("n", ctypes.c_int64),
+                ("P", ctypes.c_void_p), ("C", ctypes.c_void_p), ("CT", ctypes.c_void_p),
+                ("sign_words", ctypes.c_void_p), ("s_w", ctypes.c_void_p), ("L", ctypes.c_void_p),
+                ("S_idx", ctypes.c_void_p), ("S_val", ctypes.c_void_p), ("Wp", ctypes.c_void_p),
+                ("Wp_planes", ctypes.c_void_p), ("J", ctypes.c_void_p), ("cj_planes", ctypes.c_void_p),
+                ("pass_dev", ctypes.c_void_p), ("Ux_tm", ctypes.c_void_p), ("K_tm", ctypes.c_void_p)]
+
+
 _lib = None
 _P, _I64, _U32, _U64, _INT, _F32 = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_uint32,
                                     ctypes.c_uint64, ctypes.c_int, ctypes.c_float)
@@ -84,6 +96,8 @@ _SIGS = {
     "mosaic_mask_activation_ex": ([_PP, _PK, _U64, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _INT, _P, _SZ,
                                    _P], _INT),
     "mosaic_advance_pass": ([_P, _U64, _P], _INT),
+    "mosaic_mask": ([_INT, _PP, _PK, _U64, _I64, _I64, _I64, ctypes.POINTER(mosaic_mask_io), _INT, _P, _SZ,
+                     _P], _INT),
     "mosaic_prepare_unmask": ([_PP, _I64, _P, _P, _P], _INT),
     "mosaic_unmask_planes": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
                               _INT, _P, _SZ, _P], _INT),
@@ -317,6 +331,18 @@ def mosaic_mask_activation_ex(params, key, pass_id, pass_dev, m, n_pad, l, C, J,
     _call("mosaic_mask_activation_ex", ctypes.byref(params), ctypes.byref(key), pass_id, _ptr(pass_dev), m,
           n_pad, l, _ptr(C), _ptr(J), _ptr(cj_planes), _ptr(Ux_tm), _ptr(K_tm), variant, _ptr(ws),
           0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
+
+
+def mosaic_mask(kind, params, key, stream_id, rows, n_pad, l, io: dict, variant=GEMM_AUTO, ws=None,
+                stream=None):
+    """io: field name of mosaic_mask_io -> tensor (device buffers) or int (ldw, n)."""
+    s = mosaic_mask_io()
+    for name, _ in mosaic_mask_io._fields_:
+        v = io.get(name)
+        setattr(s, name, v if isinstance(v, int) or v is None else _ptr(v))
+    _call("mosaic_mask", kind, ctypes.byref(params), ctypes.byref(key), stream_id, rows, n_pad, l,
+          ctypes.byref(s), variant, _ptr(ws), 0 if ws is None else ws.numel() * ws.element_size(),
+          _stream(stream))
 
 
 def mosaic_advance_pass(pass_dev, delta=1, stream=None):

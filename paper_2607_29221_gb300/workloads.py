@@ -42,12 +42,37 @@ def gaussian_f32(seed: int, rows: int, cols: int, std: float) -> np.ndarray:
     return a
 
 
+def gaussian_f32_rows(seed: int, rows: int, cols: int, std: float, which) -> np.ndarray:
+    """Rows `which` (ascending) of gaussian_f32(seed, rows, cols, std), drawn in
+    chunks so that the whole matrix is never held at once."""
+    which = np.asarray(which, dtype=np.int64)
+    g = np.random.Generator(np.random.PCG64(seed))
+    out = np.empty((len(which), cols), np.float32)
+    chunk = max(1, (1 << 24) // max(cols, 1))
+    start, k = 0, 0
+    while start < rows and k < len(which):
+        n = min(chunk, rows - start)
+        a = g.standard_normal((n, cols), dtype=np.float32)
+        while k < len(which) and which[k] < start + n:
+            out[k] = a[which[k] - start]
+            k += 1
+        start += n
+    if std != 1.0:
+        out *= np.float32(std)
+    return out
+
+
 def activations(l: int, n: int, seed: int = SEED_X, std: float = 1.0) -> np.ndarray:
     return gaussian_f32(seed, l, n, std)
 
 
 def weights(m: int, n: int, seed: int = SEED_W, std: float = 0.02) -> np.ndarray:
     return gaussian_f32(seed, m, n, std)
+
+
+def weight_rows(m: int, n: int, which, seed: int = SEED_W, std: float = 0.02) -> np.ndarray:
+    """Rows `which` (ascending) of weights(m, n, seed, std)."""
+    return gaussian_f32_rows(seed, m, n, std, which)
 
 
 def bias(m: int, seed: int = SEED_B, std: float = 0.02) -> np.ndarray:

@@ -155,3 +155,26 @@ def test_validation_of_newer_entry_points(lib):
 def test_selftest_wait_validates_its_limit(lib):
     assert _status("mosaic_selftest_wait", 0, None) == 1
     assert _status("mosaic_selftest_wait", 1000001, None) == 1
+
+
+def test_mosaic_mask_dispatch_validation(lib):
+    """mosaic_mask: unknown kind or missing io struct is an argument error; each
+    kind reaches its role call's own validation (decided on the host)."""
+    key = M.make_key(range(8))
+    p = M.default_params()
+    fake = 1 << 40
+    io = M.mosaic_mask_io()
+    assert _status("mosaic_mask", 1, ctypes.byref(p), ctypes.byref(key), 0, 0, 64, 0, None, 0, None, 0,
+                   None) == 1
+    assert _status("mosaic_mask", 9, ctypes.byref(p), ctypes.byref(key), 0, 0, 64, 0, ctypes.byref(io), 0,
+                   None, 0, None) == 1
+    io.P = io.C = io.CT = fake
+    # chains with no workspace: the role call's own MOSAIC_ERR_WORKSPACE
+    assert _status("mosaic_mask", M.MASK_CHAINS, ctypes.byref(p), ctypes.byref(key), 0, 0, 64, 0,
+                   ctypes.byref(io), 0, None, 0, None) == 6
+    # chains with a width that is not a power of two
+    assert _status("mosaic_mask", M.MASK_CHAINS, ctypes.byref(p), ctypes.byref(key), 0, 0, 100, 0,
+                   ctypes.byref(io), 0, None, 0, None) == 2
+    bad = M.default_params(act_nested=2)
+    assert _status("mosaic_mask", M.MASK_ACTIVATION, ctypes.byref(bad), ctypes.byref(key), 0, 8, 32, 4,
+                   ctypes.byref(io), 0, None, 0, None) == 1
