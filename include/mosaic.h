@@ -446,7 +446,17 @@ mosaic_status mosaic_device_status(void *stream);
  *    process exits.
  *  - The first call on a device looks up the array's device address
  *    (cudaGetSymbolAddress) with that device current; make that first call
- *    before any stream capture.
+ *    before any stream capture.  The address is kept for the life of the
+ *    process: after cudaDeviceReset (or anything else that destroys the
+ *    device's primary context) it is stale, so do not call this entry point
+ *    on that device again in the same process.
+ *  - Speed: the array holds the l x m scratch first and then whichever
+ *    optional parts of mosaic_unmask still fit (digit planes of Q_d, tile
+ *    images of the Q_i, line-offset copies of the S lists).  Beyond small
+ *    l x m the digit planes do not fit (they need about 8 (l + m) r_d bytes),
+ *    so with MOSAIC_GEMM_TC / AUTO the Q_d L^T product runs on the CUDA cores
+ *    (IMAD), several times slower than with a caller workspace; the results
+ *    are the same.
  *  - All calls share the one array: calls whose GPU work overlaps (e.g. on two
  *    streams at once) race on it, so order them (same stream or events).
  *    Nothing in the array needs to start at zero: each call writes every

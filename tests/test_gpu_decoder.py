@@ -113,7 +113,13 @@ def test_masked_layer_close_to_float_layer(name, l):
         assert np.all(np.isfinite(y))
         errs.append(_rel(y - x, ref - x))      # relative error of the layer's update
         del layer
-    assert errs[0] < 2e-3, errs
+    # sigma = 0 leaves the quantisation error: a rotated row's absmax is about 4
+    # standard deviations, so rounding to q_max levels adds a relative RMS error of
+    # about (4 / q_max) / sqrt(12) = 1.15 / q_max per operand; bound the layer's
+    # update by 2.5 / q_max of its narrowest window.
+    from paper_2607_29221_gb300 import protocol as PR
+    qmin = min(M.mosaic_qmax(PR.pad_width(n)) for n in (s.hidden, s.ffn))
+    assert errs[0] < 2.5 / qmin, (errs, qmin)
     assert errs[1] < 2e-2, errs
     assert errs[0] <= errs[1] <= errs[2], errs
 

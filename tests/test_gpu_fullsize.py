@@ -5,7 +5,16 @@ parameters): the FFN up/down projections at 7B shape, every linear of one
 The GPU runs each secure linear call in full; the oracle recomputes the public
 chains in full and every other output at sampled weight rows and tokens
 (``oracle.sampled``), and they must agree bit-exactly; decoded floats within
-1e-6 x (|Y_hat s_w s_x| + |b|)."""
+1e-6 x (|Y_hat s_w s_x| + |b|).  The sampled rows include both sides of
+128-row tile edges spread over the whole matrix and the last tile; the sampled
+tokens both sides of 128-token tile edges.
+
+Every entry of the server output Z = X' [W'; P]^T is covered as well, by a
+host-side Freivalds check over Z_{2^32} (numpy uint32 arithmetic, nothing from
+the GPU's arithmetic): for four random vectors a, Z a = X' ([W'; P]^T a) on the
+GPU's own X' and [W'; P], which the sampled comparisons pin to the oracle.  A
+wrong entry e escapes one vector with probability at most 2^-(32 - v), v the
+trailing zero bits of e."""
 import numpy as np
 import pytest
 
@@ -55,6 +64,34 @@ def _u32(t):
     return t.cpu().numpy().view(np.uint32)
 
 
+def _sample_rows(m, edges=24):
+    """Rows 0, 1, m/3, m/2 + 7, m - 1, both sides of `edges` 128-row tile edges
+    spread evenly over the matrix, and the first row of the last tile."""
+    cuts = np.unique(np.linspace(1, max(1, (m - 1) // 128), edges).astype(np.int64)) * 128
+    rows = [0, 1, m // 3, m // 2 + 7, m - 1, (m - 1) // 128 * 128]
+    rows += [c - 1 for c in cuts] + [c for c in cuts]
+    return np.unique(np.clip(np.array(rows), 0, m - 1))
+
+
+def _sample_tokens(l):
+    """Tokens 0, l/2, l - 1 and both sides of every 128-token tile edge."""
+    toks = [0, l // 2, l - 1] + [c + d for c in range(128, l, 128) for d in (-1, 0)]
+    return np.unique(np.clip(np.array(toks), 0, l - 1))
+
+
+def _freivalds_host(Wp, Xp, Z, seed, k=4):
+    """Z a == X' (Wp^T a) over Z_{2^32} for k random a (numpy uint32, wraps)."""
+    N = Z.shape[1]
+    Wh, Xh, Zh = _u32(Wp[:N]), _u32(Xp), _u32(Z)
+    a = np.random.Generator(np.random.PCG64(seed)).integers(0, 1 << 32, size=(N, k), dtype=np.uint32)
+    v = np.zeros((Wh.shape[1], k), np.uint32)          # Wp^T a, accumulated row block by row block
+    for s0 in range(0, N, 4096):
+        blk = Wh[s0:s0 + 4096]
+        for i in range(k):
+            v[:, i] += (blk * a[s0:s0 + 4096, i:i + 1]).sum(axis=0, dtype=np.uint32)
+    assert np.array_equal(Zh @ a, Xh @ v)
+
+
 def _check_linear(proto, m, n, ls, matrix_id, w_std=0.02, seed_off=0):
     from paper_2607_29221_gb300 import protocol as PR
     p = O.Params()
@@ -63,7 +100,7 @@ def _check_linear(proto, m, n, ls, matrix_id, w_std=0.02, seed_off=0):
     W = wl.weights(m, n, seed=wl.SEED_W + seed_off, std=w_std)
     b = wl.bias(m, seed=wl.SEED_B + seed_off)
     layer = PR.SecureLinear(proto, torch.from_numpy(W).cuda(), matrix_id, ch, torch.from_numpy(b).cuda())
-    rows = np.unique(np.array([0, 1, m // 3, m // 2 + 7, m - 1]))
+    rows = _sample_rows(m)
     wr = OS.weight_rows(KEY, p, W[rows], rows, matrix_id, P, C, n_pad)
     rows_t = torch.from_numpy(rows).cuda()
     torch.cuda.synchronize()
@@ -87,7 +124,7 @@ def _check_linear(proto, m, n, ls, matrix_id, w_std=0.02, seed_off=0):
         Z = layer.server(Xp, Xpl)
         Yhat = torch.empty(l, m, dtype=torch.int32, device="cuda")
         Y = layer.unmask(Z, mp, s_x, Yhat=Yhat)
-        toks = np.unique(np.array([0, l // 2, l - 1]))
+        toks = _sample_tokens(l)
         tc = OS.token_cols(KEY, p, X_tm[toks], toks, pass_id, wr.sign_words, wr.qmax, C, n_pad)
         K = OS.k_entries(p, wr, tc)
         Ym, Q = OS.server_entries(wr, tc, P)
@@ -103,6 +140,7 @@ def _check_linear(proto, m, n, ls, matrix_id, w_std=0.02, seed_off=0):
         assert np.array_equal(Zs[:, rows], Ym.T), (m, n, l)
         assert np.array_equal(Zs[:, m:], np.hstack([q.T for q in Q])), (m, n, l)
         assert np.array_equal(_u32(Yhat[tk][:, rows_t]), Yh.T), (m, n, l)
+        _freivalds_host(layer.Wp, Xp, Z, seed=l + m)
         mag = np.abs(Yh.T.view(np.int32) * wr.s_w[None, :].astype(np.float64)
                      * tc.s_x[:, None].astype(np.float64)) + np.abs(b[rows].astype(np.float64))[None, :]
         err = np.abs(Y[tk][:, rows_t].cpu().numpy().astype(np.float64) - Yf.T)

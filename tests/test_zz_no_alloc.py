@@ -32,12 +32,18 @@ def _pass(layer, X_tm, pass_id):
     return mp, s_x, Z
 
 
-def test_noalloc_unmask_matches_workspace_unmask_twice():
+@pytest.mark.parametrize("variant_name,m,n,l", [("imad", 320, 500, 48), ("tc", 320, 500, 48),
+                                                ("tc", 4096, 256, 1024)])
+def test_noalloc_unmask_matches_workspace_unmask_twice(variant_name, m, n, l):
+    """Small shapes on both product variants, and l * m = 2^22 exactly: the l x m
+    scratch fills the whole array and every optional part is skipped."""
     from paper_2607_29221_gb300 import mosaic as M
     from paper_2607_29221_gb300 import protocol as PR
+    variant = {"imad": M.GEMM_IMAD, "tc": M.GEMM_TC}[variant_name]
+    if variant == M.GEMM_TC and not M.mosaic_gemm_variant_available(M.GEMM_TC):
+        pytest.skip("tensor-core variant not available")
     key = wl.mask_key()
-    proto = PR.Protocol(key, M.default_params(), variant=M.GEMM_IMAD)
-    m, n, l = 320, 500, 48
+    proto = PR.Protocol(key, M.default_params(), variant=variant)
     ch = PR.Chains(proto, PR.pad_width(n))
     W = torch.from_numpy(wl.weights(m, n)).cuda()
     b = torch.from_numpy(wl.bias(m)).cuda()
@@ -56,7 +62,7 @@ def test_noalloc_unmask_matches_workspace_unmask_twice():
         Y = torch.full((l, m), float("nan"), dtype=torch.float32, device="cuda")
         Yhat = torch.zeros(l, m, dtype=torch.int32, device="cuda")
         M.mosaic_unmask_noalloc(proto.params, l, m, Z, Z.stride(0), mp.K, layer.L, layer.S_idx,
-                                layer.S_val, layer.s_w, s_x, b, Y, Yhat, m, M.GEMM_IMAD)
+                                layer.S_val, layer.s_w, s_x, b, Y, Yhat, m, variant)
         outs.append((Y, Yhat))
     M.mosaic_device_status()
     for (mp, s_x, Z, Y_ref, Yhat_ref), (Y, Yhat) in zip(runs, outs):
