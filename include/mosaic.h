@@ -212,11 +212,16 @@ int mosaic_gemm_variant_available(int variant);
  * M, N, K >= 0, K <= 2^20.  The TC and MMA_S8 variants split A and B into
  * digit planes in `ws` (mosaic_workspace_bytes(MOSAIC_OP_RING_GEMM, ...));
  * IMAD needs no workspace.  TC requires lda, ldb multiples of 4 and 16-byte
- * aligned A, B (MOSAIC_ERR_ALIGN otherwise; AUTO then runs IMAD).  With 1 <= M <= MOSAIC_SKINNY_MAX_M (a few tokens, e.g. one
- * decode step) and K >= 1, TC and AUTO run a streaming CUDA-core kernel
- * instead, which reads each element of B once (4 bytes) and needs no
- * workspace; the result is the same ring product. */
+ * aligned A, B (MOSAIC_ERR_ALIGN otherwise; AUTO then runs IMAD).  With
+ * 1 <= M <= MOSAIC_SKINNY_MAX_M (a few tokens, e.g. one decode step) and
+ * K >= 1, TC and AUTO run a streaming CUDA-core kernel instead, which reads
+ * each element of B once (4 bytes) and needs no workspace.  With
+ * MOSAIC_SKINNY_MAX_M < M <= MOSAIC_STREAMW_MAX_M (a small decode batch) TC
+ * and AUTO run a tensor-core kernel that also reads each element of B once as
+ * uint32 and splits it into digits on the chip; it needs 8 M ceil8(K) bytes of
+ * `ws` for A's digit planes.  Every path gives the same ring product. */
 #define MOSAIC_SKINNY_MAX_M 16
+#define MOSAIC_STREAMW_MAX_M 64
 mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb,
                                uint32_t *C, int64_t ldc, int64_t M, int64_t N, int64_t K,
                                int variant, void *ws, size_t ws_bytes, void *stream);

@@ -356,10 +356,16 @@ mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B
     // A few tokens: the streaming kernel reads B once, no planes needed.
     if (skinny_ok(A, lda, B, ldb, M, K))
         return ring_gemm_skinny(A, lda, B, ldb, C, ldc, nullptr, 0, 1, M, N, K, st);
-    // Tensor-core variant: split both operands into digit planes in ws.
     const int64_t Kp = (K + 7) / 8 * 8;
     if (!aligned16(A) || !aligned16(B) || lda % 4 || ldb % 4) return MOSAIC_ERR_ALIGN;
     Carve cv = carve(ws, ws_bytes);
+    // Up to kTcwMaxM tokens: tensor cores, B read once as uint32 and split on the chip.
+    if (tcw_ok(A, lda, B, ldb, M, N, K)) {
+        uint16_t *Ap = cv.take<uint16_t>(tcw_ws_bytes(M, K) / 2);
+        if (!Ap) return MOSAIC_ERR_WORKSPACE;
+        return ring_gemm_tcw(A, lda, B, ldb, C, ldc, M, N, K, Ap, st);
+    }
+    // Tensor-core variant: split both operands into digit planes in ws.
     uint16_t *Ap = cv.take<uint16_t>((size_t)(4 * M * Kp));
     uint16_t *Bp = cv.take<uint16_t>((size_t)(4 * N * Kp));
     if (!Ap || !Bp) return MOSAIC_ERR_WORKSPACE;
@@ -395,9 +401,11 @@ mosaic_status mosaic_device_status(void *stream) {
     const mosaic_status s = device_status(as_stream(stream));
     const mosaic_status s2 = skinny_status();
     const mosaic_status s3 = gather_status();
+    const mosaic_status s4 = tcw_status();
     if (s != MOSAIC_OK) return s;
     if (s2 != MOSAIC_OK) return s2;
     if (s3 != MOSAIC_OK) return s3;
+    if (s4 != MOSAIC_OK) return s4;
     return cudaGetLastError() == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
 }
 

@@ -196,6 +196,20 @@ mosaic_status ring_gemm_skinny(const uint32_t *A, int64_t lda, const uint32_t *B
 // Reads and clears the streaming kernel's timeout word (after a stream sync).
 mosaic_status skinny_status();
 
+// Tensor-core ring GEMM for kSkinnyMaxM < M <= kTcwMaxM token rows that
+// streams B as uint32 (4 bytes an element) and splits it into digits on the
+// chip: C = A B^T (NT, uint32, K-contiguous).  Ap: tcw_ws_bytes(M, K) bytes of
+// 16-byte aligned scratch for A's fp16 digit planes.  tcw_ok() tells whether
+// the operands qualify (16-byte aligned bases, row strides multiples of 4
+// words, a Blackwell device).
+constexpr int64_t kTcwMaxM = 64;
+size_t tcw_ws_bytes(int64_t M, int64_t K);
+bool tcw_ok(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb, int64_t M, int64_t N, int64_t K);
+mosaic_status ring_gemm_tcw(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb, uint32_t *C,
+                            int64_t ldc, int64_t M, int64_t N, int64_t K, uint16_t *Ap, cudaStream_t st);
+// Reads and clears that kernel's timeout word (after a stream sync).
+mosaic_status tcw_status();
+
 // Freivalds check: Y (k x ncols) = a (k x m) W (m x ncols, ldw), and the
 // per-token comparison a^T Y' vs Ychk X' (lhs, rhs: k x l scratch each).
 mosaic_status freivalds_colsum(const uint32_t *a, int k, const uint32_t *W, int64_t ldw, int64_t m,

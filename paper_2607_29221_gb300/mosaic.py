@@ -22,6 +22,7 @@ STATUS = {0: "ok", 1: "invalid argument", 2: "invalid shape", 3: "misaligned", 4
 
 GEMM_AUTO, GEMM_TC, GEMM_MMA_S8, GEMM_IMAD = 0, 1, 2, 3
 SKINNY_MAX_M = 16   # MOSAIC_SKINNY_MAX_M: token counts the streaming product serves
+STREAMW_MAX_M = 64  # MOSAIC_STREAMW_MAX_M: up to here the tensor-core product streams B as uint32
 OP_RING_GEMM, OP_MASK_CHAINS, OP_MASK_WEIGHT, OP_MASK_ACTIVATION, OP_UNMASK = 1, 2, 3, 4, 5
 OP_FREIVALDS_CHECK, OP_ACTIVATION_PLANES, OP_UNMASK_PLANES = 6, 7, 8
 TAG_M, TAG_N, TAG_L, TAG_S, TAG_EW, TAG_R, TAG_T, TAG_EX, TAG_SIGN, TAG_CHECK = range(1, 11)

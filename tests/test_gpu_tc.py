@@ -188,6 +188,42 @@ def test_few_tokens_edges():
     assert np.all(got[:, :2] == 0) and np.all(got[:, 2:] == 0xFFFFFFFF)
 
 
+# --------------------------------------------------------------------------
+# 17..64 tokens: the TC variant streams uint32 B by TMA, splits it into fp16
+# digits in tensor memory on the chip and runs 4 MMAs per 16 K (one per digit
+# of B, N = (4 - i) x token tile); stream-K over (128-row tile, 256-K chunk)
+# units, partial tiles added with red.add.
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Mm", [17, 24, 32, 33, 48, 49, 64])
+@pytest.mark.parametrize("N,K", [(1, 1), (61, 128), (129, 33), (300, 652), (1000, 4100), (121, 8192),
+                                 (257, 257)])
+def test_streamw_tokens_random(Mm, N, K):
+    A = wl.uniform_u32(131 + Mm, Mm, K)
+    B = wl.uniform_u32(137, N, K)
+    assert np.array_equal(ring_gemm_u32(A, B), ref(A, B))
+
+
+@pytest.mark.parametrize("Mm", [20, 40, 64])
+@pytest.mark.parametrize("va,vb", [(ALL_M128, ALL_M128), (ALL_P127, ALL_M128), (0xFFFFFFFF, 0x80000000),
+                                   (0xFFFFFFFF, 0xFFFFFFFF)])
+def test_streamw_tokens_adversarial(Mm, va, vb):
+    """Constant digits over K = 3000: shift group 3 reaches 2^24 at every drain
+    with all digits -128; every entry is K va vb mod 2^32."""
+    Mm, N, K = Mm, 300, 3000
+    A = np.full((Mm, K), va, np.uint32)
+    B = np.full((N, K), vb, np.uint32)
+    want = np.uint32((K * va * vb) % (1 << 32))
+    assert np.all(ring_gemm_u32(A, B) == want)
+
+
+def test_streamw_tokens_many_tiles_and_units():
+    """More (tile, chunk) units than SMs with a ragged last tile and K chunk:
+    CTAs start and end inside tiles."""
+    A = wl.uniform_u32(141, 40, 5000)
+    B = wl.uniform_u32(142, 20000 + 77, 5000)
+    assert np.array_equal(ring_gemm_u32(A, B), ref(A, B))
+
+
 @pytest.mark.parametrize("N", [5000, 9984])
 def test_tc_whole_waves_then_stream_k(N):
     """160 (312) tiles on 152 SMs with 8 K chunks: the first one (two) waves of
