@@ -340,7 +340,8 @@ def mosaic_mask(kind, params, key, stream_id, rows, n_pad, l, io: dict, variant=
     s = mosaic_mask_io()
     for name, _ in mosaic_mask_io._fields_:
         v = io.get(name)
-        setattr(s, name, v if isinstance(v, int) or v is None else _ptr(v))
+        if v is not None:                 # fields left out stay 0 / NULL
+            setattr(s, name, v if isinstance(v, int) else _ptr(v))
     _call("mosaic_mask", kind, ctypes.byref(params), ctypes.byref(key), stream_id, rows, n_pad, l,
           ctypes.byref(s), variant, _ptr(ws), 0 if ws is None else ws.numel() * ws.element_size(),
           _stream(stream))
