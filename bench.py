@@ -533,7 +533,7 @@ def run_mine(args, rank, world):
                    if len(runner.layers) > 1 else "one server-product launch")
     if variant == M.GEMM_TC:
         roof["frac_of_sustained"] = round(roof["achieved"] / bf16_sus, 4)
-    enc_bytes = sum(l * (4 * ly.n + (16 if ly.use_planes and l > M.SKINNY_MAX_M else 8) * ly.n_pad)
+    enc_bytes = sum(l * (4 * ly.n + (16 if ly.use_planes and l > M.STREAMW_MAX_M else 8) * ly.n_pad)
                     for ly in runner.layers)
     enc_gbs = enc_bytes / (enc_ms / 1e3) / 1e9 if enc_ms > 0 else 0.0
     rooflines = [dict(roof, kernel=roof["kernel"]),
@@ -609,7 +609,7 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
         bufs = [dict(Xp=torch.empty(l, ly.n_pad, dtype=torch.int32, device=dev),
                      s_x=torch.empty(l, dtype=torch.float32, device=dev),
                      Xpl=(torch.empty(4, l, ly.n_pad, dtype=torch.int16, device=dev)
-                          if ly.use_planes and l > M.SKINNY_MAX_M else None),
+                          if ly.use_planes and l > M.STREAMW_MAX_M else None),
                      Z=torch.empty(l, ly.m + proto.sum_r, dtype=torch.int32, device=dev),
                      Y=torch.empty(l, ly.m, dtype=torch.float32, device=dev)) for ly in layers]
         xs = [torch.from_numpy(wl.activations(l, ly.n, seed=wl.SEED_X + l)).to(dev) for ly in layers]
@@ -658,16 +658,18 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
         step_ms = online_ms + initx_ms
         del masks
         w_bytes = sum((ly.m + proto.sum_r) * ly.n_pad * 4 for ly in layers)
-        # up to SKINNY_MAX_M tokens the server streams uint32 W' (4 B an element),
-        # beyond that the tensor cores read its bf16 digit planes (8 B an element)
+        # up to STREAMW_MAX_M tokens the server streams uint32 W' (4 B an element:
+        # CUDA cores up to SKINNY_MAX_M tokens, tensor cores above), beyond that
+        # the tensor cores read its bf16 digit planes (8 B an element)
         skinny = variant != M.GEMM_IMAD and l <= M.SKINNY_MAX_M
-        read_bytes = w_bytes if skinny or variant == M.GEMM_IMAD else 2 * w_bytes
+        streamw = variant != M.GEMM_IMAD and M.SKINNY_MAX_M < l <= M.STREAMW_MAX_M
+        read_bytes = w_bytes if skinny or streamw or variant == M.GEMM_IMAD else 2 * w_bytes
         sweep.append({"l": l, "ms_per_step": round(step_ms, 4), "tokens_s": round(world * l / (step_ms / 1e3), 1),
                       "online_ms": round(online_ms, 4), "online_ms_eager": round(eager_ms, 4),
                       "init_x_ms_per_step": round(initx_ms, 4),
                       "gpu_launches_per_step": int(round(launches / args.steps)),
                       "gemm_ms": round(gemm_ms, 4), "ring_tops": round(2 * runner.ring_macs / (gemm_ms / 1e3) / 1e12, 2),
-                      "server_kernel": "ring_gemm_skinny" if skinny else
+                      "server_kernel": "ring_gemm_skinny" if skinny else "ring_gemm_tcw" if streamw else
                                        ("ring_gemm_imad" if variant == M.GEMM_IMAD else "ring_gemm_tc"),
                       "w_prime_bytes": w_bytes, "server_read_bytes": read_bytes,
                       "server_read_gbs": round(read_bytes / (gemm_ms / 1e3) / 1e9, 1),

@@ -106,7 +106,7 @@ class SecureDecoderLayer:
         Sr = self.proto.sum_r
         self.bufs = []
         for lin in self.linears():
-            planes = lin.use_planes and l > M.SKINNY_MAX_M
+            planes = lin.use_planes and l > M.STREAMW_MAX_M
             self.bufs.append(dict(
                 Xp=torch.empty(l, lin.n_pad, dtype=torch.int32, device=dev),
                 s_x=torch.empty(l, dtype=torch.float32, device=dev),

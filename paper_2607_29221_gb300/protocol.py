@@ -149,7 +149,7 @@ class SecureLinear:
         dev = self.proto.device
         Xp = _u32(l, self.n_pad, device=dev) if Xp is None else Xp
         s_x = torch.empty(l, dtype=torch.float32, device=dev) if s_x is None else s_x
-        planes = self.use_planes and l > M.SKINNY_MAX_M
+        planes = self.use_planes and l > M.STREAMW_MAX_M
         if planes and Xplanes is None:
             Xplanes = torch.empty(4, l, self.n_pad, dtype=torch.int16, device=dev)
         M.mosaic_encode(X_tm, X_tm.stride(0), l, self.n, self.n_pad, self.qmax, 1, self.sign_words,
@@ -159,12 +159,14 @@ class SecureLinear:
     def server(self, Xp, Xplanes, Z=None):
         """Untrusted accelerator: Z = X'_tm [W'; P]^T = [Y' | Q_1 .. Q_d] (token-major).
 
-        Up to SKINNY_MAX_M tokens the product streams the uint32 W' (4 bytes an
-        element); more tokens run on the tensor cores from the digit planes."""
+        Up to STREAMW_MAX_M tokens the product streams the uint32 W' (4 bytes an
+        element: CUDA cores up to SKINNY_MAX_M tokens, tensor cores with an
+        on-chip digit split above); more tokens run on the tensor cores from the
+        digit planes of W' and X'."""
         l = Xp.shape[0]
         N = self.m + self.proto.sum_r
         Z = _u32(l, N, device=self.proto.device) if Z is None else Z
-        if self.use_planes and l > M.SKINNY_MAX_M:
+        if self.use_planes and l > M.STREAMW_MAX_M:
             M.mosaic_ring_gemm_planes(Xplanes, self.n_pad, l * self.n_pad, self.Wp_planes,
                                       self.n_pad, N * self.n_pad, Z, N, l, N, self.n_pad,
                                       M.GEMM_TC)
