@@ -7,16 +7,20 @@
 // batch is memory-bound).  The digit-plane product (ring_gemm_tc.cu) reads B
 // as four bf16 planes, 8 bytes an element; this kernel reads the uint32 B,
 // 4 bytes an element, and splits it into digits on the chip:
-//   * 128 rows x 32 K of B land in shared memory by TMA (128-byte swizzle);
+//   * a stage is 64 K: two boxes of 128 rows x 32 K of B land in shared
+//     memory by TMA (128-byte swizzle), in a ring of their own that the
+//     converters release as soon as they have read them;
 //   * converter warps split each element into its four signed base-2^8
 //     digits d_i = byte_i(b + 0x80808080) - 128 as fp16 (exact for
 //     |d| <= 128) and store them with tcgen05.st into a ring of tensor-memory
 //     slots, from where the MMA reads its A operand: shared memory carries
 //     only the TMA traffic and the small token operand;
 //   * the tokens' digit planes (fp16 [4][M][Kp], split once per call) come by
-//     TMA as one 3-D box {32 K, NT rows, 4 planes} per stage (64-byte swizzle);
+//     TMA as two 3-D boxes {32 K, NT rows, 4 planes} per stage (64-byte
+//     swizzle) into a second ring; one barrier per stage, armed by a single
+//     MMA commit, releases both the token boxes and the stage's digit slot;
 //   * the product D (128 weight rows x tokens) = W_i [X_0; ...; X_{3-i}]^T
-//     runs as ONE tcgen05.mma per weight digit i with N = (4 - i) NT, written
+//     runs as ONE tcgen05.mma per weight digit i and 16 K with N = (4 - i) NT, written
 //     at column i NT of an accumulator set whose shift group s occupies
 //     columns [s NT, (s + 1) NT): column block j of MMA i lands in group i + j,
 //     so the 10 digit pairs with i + j <= 3 take 4 MMAs per 16 K;
@@ -24,12 +28,14 @@
 //     fp32 integer) the epilogue folds all four groups into int32 registers,
 //     acc += g0 + 2^8 g1 + 2^16 g2 + 2^24 g3 mod 2^32, while the MMAs go on in
 //     the other accumulator set (two sets when 8 NT columns leave room for
-//     the digit slots);
+//     four digit slots);
 //   * (weight tile, 256-K chunk) units are split evenly over a persistent
 //     grid (stream-K); each CTA adds its partial tiles into C with red.add
 //     (C is zeroed first), exact and order-free in Z_{2^32}.
-// Warps: 0 TMA producer, 1 TMEM allocation + MMA issuer, 2..5 converters,
-// 6..9 epilogue (warp w reaches TMEM lanes 32 (w % 4) .. + 31).  Every wait is
+// Warps: 0 TMA producer, 1 TMEM allocation + MMA issuer, 2..9 converters
+// (two groups of four, one warp per TMEM lane quarter; group j converts the
+// j-th 32-K box of every stage), 10..13 epilogue (warp w reaches TMEM lanes
+// 32 (w % 4) .. + 31).  Every wait is
 // bounded (about 2 s of %globaltimer): on expiry the kernel raises its device
 // error word (read by tcw_status), stops, lets its own copies and products
 // land (bounded), frees TMEM and returns.
@@ -48,27 +54,29 @@ __device__ uint32_t g_tcw_error = 0;
 namespace {
 
 constexpr int WR = 128;          // weight rows per tile (MMA M)
-constexpr int KB = 32;           // K per stage
-constexpr int CHUNK = 8;         // stages per drain: 256 K
+constexpr int KB = 32;           // K per TMA box
+constexpr int KS = 64;           // K per stage: two boxes
+constexpr int CHUNK = 4;         // stages per drain: 256 K
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int THREADS = 320;
-constexpr int CONV_WARPS = 4;
+constexpr int CONV_WARPS = 8;    // two groups of four (one warp per TMEM lane quarter)
 constexpr int EPI_WARPS = 4;
+constexpr int THREADS = 32 * (2 + CONV_WARPS + EPI_WARPS);
 constexpr int W_BOX = WR * KB * 4;          // 16 KB of uint32
+constexpr int SLOT_COLS = 4 * (KS / 2);     // a stage's digits: 4 planes x 32 columns (64 K of fp16 pairs)
+constexpr int SLOTS = 2;                    // digit slots (stages) in TMEM
 
 template <int NT>
 struct WCfg {
-    static constexpr int X_PLANE = NT * KB * 2;            // one fp16 digit plane of the token box
+    static constexpr int X_PLANE = NT * KB * 2;            // one fp16 digit plane of a token box
     static constexpr int X_BOX = 4 * X_PLANE;
-    static constexpr int STAGE = W_BOX + X_BOX;
-    static constexpr int STAGES = NT <= 48 ? 6 : 5;
-    static constexpr int NSETS = 8 * NT <= 384 ? 2 : 1;    // accumulator sets of 4 NT columns
+    static constexpr int WST = NT == 64 ? 3 : 4;           // weight stages (2 boxes each) in the ring
+    static constexpr int XST = NT == 64 ? 3 : 4;           // token stages (2 boxes each) in the ring
+    static constexpr int NSETS = 8 * NT + SLOTS * SLOT_COLS <= (int)TMEM_COLS ? 2 : 1;   // accumulator sets
     static constexpr int ACC_COLS = NSETS * 4 * NT;
-    static constexpr int SLOTS_FIT = ((int)TMEM_COLS - ACC_COLS) / 64;
-    static constexpr int SLOTS = SLOTS_FIT > 4 ? 4 : SLOTS_FIT;   // digit slots of 64 columns (4 planes x 32 K)
-    static constexpr int SMEM = STAGES * STAGE + 1024 + 512;
+    static constexpr int SMEM = WST * 2 * W_BOX + XST * 2 * X_BOX + 1024 + 512;
+    static_assert(SMEM <= 227 * 1024, "");
+    static_assert(ACC_COLS + SLOTS * SLOT_COLS <= (int)TMEM_COLS, "");
     static_assert(NT % 16 == 0 && NT >= 16 && NT <= 64, "");
-    static_assert(SLOTS >= 2, "at least two digit slots");
     static_assert(X_PLANE % 512 == 0, "token planes keep the 64-byte swizzle phase");
     // kind::f16 descriptor: D f32, A and B fp16, both K-major, N >> 3, M >> 4.
     __host__ __device__ static constexpr uint32_t idesc(int n) {
@@ -114,24 +122,18 @@ __device__ __forceinline__ void umma_commit(uint64_t *bar) {
                      smem_u32(bar))
                  : "memory");
 }
-// 16 columns of the warp's 32 lanes; the caller waits (tcgen05.wait::ld).
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t *v) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
-        : "r"(taddr));
+// 8 columns of the warp's 32 lanes; the caller waits (tcgen05.wait::ld).
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t *v) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7])
+                 : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-// 16 columns of the warp's 32 lanes from registers.
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *v) {
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
-        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
-        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
-        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
-        : "memory");
+// 8 columns of the warp's 32 lanes from registers.
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t *v) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
+                 "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+                 : "memory");
 }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
@@ -171,36 +173,39 @@ __global__ void __launch_bounds__(THREADS, 1)
     ring_gemm_tcw_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                          WArgs a) {
     using C = WCfg<NT>;
-    constexpr int S = C::STAGES, SL = C::SLOTS, NS = C::NSETS;
+    constexpr int SW = C::WST, SX = C::XST, NS = C::NSETS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + S * C::STAGE);
-    uint64_t *empty = full + S;
-    uint64_t *a_full = empty + S;
-    uint64_t *a_empty = a_full + SL;
-    uint64_t *acc_full = a_empty + SL;
+    uint8_t *xring = smem + SW * 2 * W_BOX;
+    uint64_t *w_full = reinterpret_cast<uint64_t *>(xring + SX * 2 * C::X_BOX);
+    uint64_t *w_empty = w_full + SW;
+    uint64_t *x_full = w_empty + SW;
+    uint64_t *done = x_full + SX;       // stage s's MMAs complete: its token boxes and digit slot are free
+    uint64_t *a_full = done + SX;
+    uint64_t *acc_full = a_full + SLOTS;
     uint64_t *acc_empty = acc_full + NS;
     uint64_t *drain = acc_empty + NS;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nk = (a.K + KB - 1) / KB;
-    // This CTA's units [u0, u1) of (tile, chunk), numbered tile-major.
+    const int nst = (a.K + KS - 1) / KS;   // stages of a tile
+    // This CTA's units [u0, u1) of (tile, 256-K chunk), numbered tile-major.
     const int64_t U = (int64_t)a.tiles * a.nchunks;
     const int u0 = (int)(U * blockIdx.x / gridDim.x), u1 = (int)(U * (blockIdx.x + 1) / gridDim.x);
     const int tile0 = u0 / a.nchunks, c0 = u0 - tile0 * a.nchunks;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < S; ++s) {
-            mbar_init(&full[s], 1);
-            mbar_init(&empty[s], CONV_WARPS + 1);
+        for (int s = 0; s < SW; ++s) {
+            mbar_init(&w_full[s], 1);
+            mbar_init(&w_empty[s], CONV_WARPS);
         }
-        for (int b = 0; b < SL; ++b) {
-            mbar_init(&a_full[b], CONV_WARPS);
-            mbar_init(&a_empty[b], 1);
+        for (int s = 0; s < SX; ++s) {
+            mbar_init(&x_full[s], 1);
+            mbar_init(&done[s], 1);
         }
+        for (int b = 0; b < SLOTS; ++b) mbar_init(&a_full[b], CONV_WARPS);
         for (int s = 0; s < NS; ++s) {
             mbar_init(&acc_full[s], 1);
             mbar_init(&acc_empty[s], EPI_WARPS);
@@ -222,24 +227,29 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t slot_col = (uint32_t)C::ACC_COLS;   // first digit slot
 
     if (warp == 0) {
-        // ---- TMA producer ----
+        // ---- TMA producer: stage g = two W boxes and two token boxes of 32 K ----
         if (lane == 0) {
             int g = 0;   // stages issued
             int tile = tile0, c = c0;
             for (int u = u0; u < u1 && !*abort_flag; ++u) {
-                const int kb1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
+                const int ks1 = (c + 1) * CHUNK < nst ? (c + 1) * CHUNK : nst;
                 bool ok = true;
-                for (int kb = c * CHUNK; kb < kb1; ++kb, ++g) {
-                    const int s = g % S, round = g / S;
-                    if (round > 0 && !mbar_wait(&empty[s], (uint32_t)(round - 1) & 1u, abort_flag)) {
+                for (int ks = c * CHUNK; ks < ks1; ++ks, ++g) {
+                    const int sw = g % SW, sx = g % SX;
+                    if ((g >= SW && !mbar_wait(&w_empty[sw], (uint32_t)(g / SW - 1) & 1u, abort_flag)) ||
+                        (g >= SX && !mbar_wait(&done[sx], (uint32_t)(g / SX - 1) & 1u, abort_flag))) {
                         raise_abort(abort_flag);
                         ok = false;
                         break;
                     }
-                    uint8_t *st = smem + s * C::STAGE;
-                    mbar_expect_tx(&full[s], C::STAGE);
-                    tma_load_2d(st, &tmW, &full[s], kb * KB, tile * WR);
-                    tma_load_3d(st + W_BOX, &tmX, &full[s], kb * KB, 0, 0);
+                    uint8_t *ws = smem + sw * 2 * W_BOX;
+                    mbar_expect_tx(&w_full[sw], 2 * W_BOX);
+                    tma_load_2d(ws, &tmW, &w_full[sw], ks * KS, tile * WR);
+                    tma_load_2d(ws + W_BOX, &tmW, &w_full[sw], ks * KS + KB, tile * WR);
+                    uint8_t *xs = xring + sx * 2 * C::X_BOX;
+                    mbar_expect_tx(&x_full[sx], 2 * C::X_BOX);
+                    tma_load_3d(xs, &tmX, &x_full[sx], ks * KS, 0, 0);
+                    tma_load_3d(xs + C::X_BOX, &tmX, &x_full[sx], ks * KS + KB, 0, 0);
                 }
                 if (!ok) break;
                 if (++c == a.nchunks) {
@@ -249,7 +259,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             if (*abort_flag) {
                 // Let the copies this thread started land before the CTA exits.
-                for (int q = g > S ? g - S : 0; q < g; ++q) mbar_drain(&full[q % S], (uint32_t)(q / S) & 1u);
+                for (int q = g > SW ? g - SW : 0; q < g; ++q) mbar_drain(&w_full[q % SW], (uint32_t)(q / SW) & 1u);
+                for (int q = g > SX ? g - SX : 0; q < g; ++q) mbar_drain(&x_full[q % SX], (uint32_t)(q / SX) & 1u);
             }
         }
     } else if (warp == 1) {
@@ -267,33 +278,35 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
                 fence_after();
                 const uint32_t dset = tmem + (uint32_t)(set * 4 * NT);
-                const int kb1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
+                const int ks1 = (c + 1) * CHUNK < nst ? (c + 1) * CHUNK : nst;
                 bool ok = true;
-                for (int kb = c * CHUNK; kb < kb1; ++kb, ++g) {
-                    const int s = g % S, b = g % SL;
-                    if (!mbar_wait(&full[s], (uint32_t)(g / S) & 1u, abort_flag) ||
-                        !mbar_wait(&a_full[b], (uint32_t)(g / SL) & 1u, abort_flag)) {
+                for (int ks = c * CHUNK; ks < ks1; ++ks, ++g) {
+                    const int sx = g % SX, b = g % SLOTS;
+                    if (!mbar_wait(&x_full[sx], (uint32_t)(g / SX) & 1u, abort_flag) ||
+                        !mbar_wait(&a_full[b], (uint32_t)(g / SLOTS) & 1u, abort_flag)) {
                         raise_abort(abort_flag);
                         ok = false;
                         break;
                     }
                     fence_after();
-                    const uint64_t dx = desc0 + (uint64_t)((s * C::STAGE + W_BOX) >> 4);
-                    const uint32_t aslot = tmem + slot_col + (uint32_t)(b * 64);
-                    const bool first = kb == c * CHUNK;
+                    const uint64_t dx = desc0 + (uint64_t)((SW * 2 * W_BOX + sx * 2 * C::X_BOX) >> 4);
+                    const uint32_t aslot = tmem + slot_col + (uint32_t)(b * SLOT_COLS);
+                    const bool first = ks == c * CHUNK;
 #pragma unroll
-                    for (int kk = 0; kk < KB / 16; ++kk) {
+                    for (int j = 0; j < 2; ++j) {
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            // Weight digit i against token digits 0 .. 3 - i: groups i .. 3.
-                            umma_tmem_a(dset + (uint32_t)(i * NT), aslot + (uint32_t)(16 * i + 8 * kk),
-                                        dx + (uint64_t)(2 * kk), C::idesc((4 - i) * NT),
-                                        (first && kk == 0 && i == 0) ? 0u : 1u);
+                        for (int kk = 0; kk < KB / 16; ++kk) {
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                // Weight digit i against token digits 0 .. 3 - i: groups i .. 3.
+                                umma_tmem_a(dset + (uint32_t)(i * NT), aslot + (uint32_t)(32 * i + 16 * j + 8 * kk),
+                                            dx + (uint64_t)((j * C::X_BOX) >> 4) + (uint64_t)(2 * kk),
+                                            C::idesc((4 - i) * NT), (first && j == 0 && kk == 0 && i == 0) ? 0u : 1u);
+                            }
                         }
                     }
                     issued_any = true;
-                    umma_commit(&empty[s]);
-                    umma_commit(&a_empty[b]);
+                    umma_commit(&done[sx]);
                 }
                 if (!ok) break;
                 umma_commit(&acc_full[set]);
@@ -306,38 +319,40 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
         }
     } else if (warp < 2 + CONV_WARPS) {
-        // ---- converters: row r of each weight box -> four fp16 digit columns in a TMEM slot ----
-        const int q = warp & 3;
+        // ---- converters: group j, row r of box j of each stage -> four fp16
+        // digit planes of 16 words (32 K) in the stage's TMEM slot ----
+        const int q = warp & 3, j = (warp - 2) >> 2;
         const int r = q * 32 + lane;
-        const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + slot_col;
+        const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + slot_col + (uint32_t)(16 * j);
         int g = 0;
         int c = c0;
         bool ok = true;
         for (int u = u0; u < u1 && ok; ++u) {
-            const int kb1 = (c + 1) * CHUNK < nk ? (c + 1) * CHUNK : nk;
-            for (int kb = c * CHUNK; kb < kb1; ++kb, ++g) {
-                const int s = g % S, b = g % SL;
-                if (!mbar_wait(&full[s], (uint32_t)(g / S) & 1u, abort_flag)) {
+            const int ks1 = (c + 1) * CHUNK < nst ? (c + 1) * CHUNK : nst;
+            for (int ks = c * CHUNK; ks < ks1; ++ks, ++g) {
+                const int sw = g % SW, b = g % SLOTS;
+                if (!mbar_wait(&w_full[sw], (uint32_t)(g / SW) & 1u, abort_flag)) {
                     raise_abort(abort_flag);
                     ok = false;
                     break;
                 }
-                // Row r of the box: 8 chunks of 16 bytes, chunk j stored at j ^ (r & 7).
-                const uint32_t row_addr = smem_u32(smem + s * C::STAGE) + (uint32_t)r * 128u;
+                // Row r of box j: 8 chunks of 16 bytes, chunk i stored at i ^ (r & 7).
+                const uint32_t row_addr = smem_u32(smem + (sw * 2 + j) * W_BOX) + (uint32_t)r * 128u;
                 uint32_t w[32];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    const uint32_t addr = row_addr + (uint32_t)((j ^ (r & 7)) * 16);
+                for (int i = 0; i < 8; ++i) {
+                    const uint32_t addr = row_addr + (uint32_t)((i ^ (r & 7)) * 16);
                     asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
-                                 : "=r"(w[4 * j]), "=r"(w[4 * j + 1]), "=r"(w[4 * j + 2]), "=r"(w[4 * j + 3])
+                                 : "=r"(w[4 * i]), "=r"(w[4 * i + 1]), "=r"(w[4 * i + 2]), "=r"(w[4 * i + 3])
                                  : "r"(addr)
                                  : "memory");
                 }
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&empty[s]);
+                if (lane == 0) mbar_arrive(&w_empty[sw]);
 #pragma unroll
                 for (int k = 0; k < 32; ++k) w[k] += 0x80808080u;
-                if (g >= SL && !mbar_wait(&a_empty[b], (uint32_t)(g / SL - 1) & 1u, abort_flag)) {
+                // The stage two back used this slot: its MMAs must be complete.
+                if (g >= SLOTS && !mbar_wait(&done[(g - SLOTS) % SX], (uint32_t)((g - SLOTS) / SX) & 1u, abort_flag)) {
                     raise_abort(abort_flag);
                     ok = false;
                     break;
@@ -348,7 +363,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                     uint32_t d[16];
 #pragma unroll
                     for (int p = 0; p < 16; ++p) d[p] = digit_pair_f16(w[2 * p], w[2 * p + 1], i);
-                    tmem_st16(lane_base + (uint32_t)(b * 64 + 16 * i), d);
+                    tmem_st8(lane_base + (uint32_t)(b * SLOT_COLS + 32 * i), d);
+                    tmem_st8(lane_base + (uint32_t)(b * SLOT_COLS + 32 * i + 8), d + 8);
                 }
                 tmem_st_wait();
                 fence_before();
@@ -377,15 +393,15 @@ __global__ void __launch_bounds__(THREADS, 1)
             fence_after();
             const uint32_t sa = lane_addr + (uint32_t)(set * 4 * NT);
 #pragma unroll
-            for (int p = 0; p < NT; p += 16) {
-                uint32_t g0[16], g1[16], g2[16], g3[16];
-                tmem_ld16(sa + 0 * NT + p, g0);
-                tmem_ld16(sa + 1 * NT + p, g1);
-                tmem_ld16(sa + 2 * NT + p, g2);
-                tmem_ld16(sa + 3 * NT + p, g3);
+            for (int p = 0; p < NT; p += 8) {
+                uint32_t g0[8], g1[8], g2[8], g3[8];
+                tmem_ld8(sa + 0 * NT + p, g0);
+                tmem_ld8(sa + 1 * NT + p, g1);
+                tmem_ld8(sa + 2 * NT + p, g2);
+                tmem_ld8(sa + 3 * NT + p, g3);
                 tmem_ld_wait();
 #pragma unroll
-                for (int j = 0; j < 16; ++j)
+                for (int j = 0; j < 8; ++j)
                     acc[p + j] += fold4(__uint_as_float(g0[j]), __uint_as_float(g1[j]), __uint_as_float(g2[j]),
                                         __uint_as_float(g3[j]));
             }
@@ -508,7 +524,7 @@ mosaic_status ring_gemm_tcw(const uint32_t *A, int64_t lda, const uint32_t *B, i
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
         return MOSAIC_ERR_CUDA;
-    const int64_t tiles = (N + WR - 1) / WR, nk = (K + KB - 1) / KB, nchunks = (nk + CHUNK - 1) / CHUNK;
+    const int64_t tiles = (N + WR - 1) / WR, nst = (K + KS - 1) / KS, nchunks = (nst + CHUNK - 1) / CHUNK;
     if (tiles * nchunks > (int64_t)INT32_MAX) return MOSAIC_ERR_SHAPE;
     const WArgs args{Cm, ldc, (int)M, (int)N, (int)K, (int)tiles, (int)nchunks};
     if (nt == 32) return launch_tcw<32>(tw, tx, args, sms, st);
