@@ -437,18 +437,24 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
 }
 
-// Digit planes of the token operand as fp16 bits: planes[d][r][c] = byte_d(a + 0x80808080) - 128.
-__global__ void digit_split_f16_kernel(const uint32_t *a, int64_t lda, int64_t rows, int64_t cols,
-                                       uint16_t *planes, int64_t ldp, int64_t plane_stride) {
-    const int64_t total = rows * cols;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * blockDim.x) {
+// Digit planes of the token operand as fp16 bits, planes[d][r][c] =
+// byte_d(a + 0x80808080) - 128, and C (rows x n, leading dimension ldc)
+// zeroed for the red.add reduction, in one launch.
+__global__ void split_f16_zero_kernel(const uint32_t *a, int64_t lda, int64_t rows, int64_t cols, uint16_t *planes,
+                                      int64_t ldp, int64_t plane_stride, uint32_t *C, int64_t ldc, int64_t n) {
+    const int64_t total = rows * cols, ctotal = rows * n;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += stride) {
         const int64_t r = i / cols, c = i - r * cols;
         const uint32_t b = a[r * lda + c] + 0x80808080u;
 #pragma unroll
         for (int d = 0; d < 4; ++d)
             planes[d * plane_stride + r * ldp + c] =
                 __half_as_ushort(__int2half_rn((int)((b >> (8 * d)) & 0xffu) - 128));
+    }
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < ctotal; i += stride) {
+        const int64_t r = i / n, c = i - r * n;
+        C[r * ldc + c] = 0u;
     }
 }
 
@@ -513,10 +519,9 @@ mosaic_status ring_gemm_tcw(const uint32_t *A, int64_t lda, const uint32_t *B, i
         return MOSAIC_ERR_SHAPE;
     if (!aligned16(Ap)) return MOSAIC_ERR_ALIGN;
     const int64_t Kp = (K + 7) / 8 * 8;
-    digit_split_f16_kernel<<<grid_for(M * K, 256), 256, 0, st>>>(A, lda, M, K, Ap, Kp, M * Kp);
+    split_f16_zero_kernel<<<grid_for(M * (K > N ? K : N), 256), 256, 0, st>>>(A, lda, M, K, Ap, Kp, M * Kp, Cm, ldc,
+                                                                               N);
     MOSAIC_TRY(launch_status());
-    if (cudaMemset2DAsync(Cm, (size_t)ldc * 4, 0, (size_t)N * 4, (size_t)M, st) != cudaSuccess)
-        return MOSAIC_ERR_CUDA;
     const int nt = M <= 32 ? 32 : M <= 48 ? 48 : 64;
     CUtensorMap tw, tx;
     if (!make_w_map(&tw, B, K, N, ldb) || !make_x_map(&tx, Ap, K, M, Kp, nt)) return MOSAIC_ERR_CUDA;
