@@ -402,10 +402,12 @@ mosaic_status mosaic_device_status(void *stream) {
     const mosaic_status s2 = skinny_status();
     const mosaic_status s3 = gather_status();
     const mosaic_status s4 = tcw_status();
+    const mosaic_status s5 = fwht_status();
     if (s != MOSAIC_OK) return s;
     if (s2 != MOSAIC_OK) return s2;
     if (s3 != MOSAIC_OK) return s3;
     if (s4 != MOSAIC_OK) return s4;
+    if (s5 != MOSAIC_OK) return s5;
     return cudaGetLastError() == cudaSuccess ? MOSAIC_OK : MOSAIC_ERR_CUDA;
 }
 

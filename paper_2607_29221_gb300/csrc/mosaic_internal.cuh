@@ -143,6 +143,9 @@ mosaic_status fwht_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, 
                           float *y, int32_t qmax, const uint32_t *mask, int64_t ldm, uint32_t *out,
                           int64_t ldo, float *scale, uint16_t *planes, cudaStream_t st);
 
+// Reads and clears the streamed rotation's timeout word (after a stream sync).
+mosaic_status fwht_status();
+
 // Generic strided ring GEMM on CUDA cores:
 // C[i*ldc + j] = (Cin ? Cin[i*ldcin + j] : 0) + sgn * sum_k A[i*sai + k*sak] * B[j*sbj + k*sbk]
 mosaic_status ring_gemm_imad(const uint32_t *A, int64_t sai, int64_t sak, const uint32_t *B,

@@ -479,3 +479,50 @@ def test_mask_activation_entry_points_and_device_pass_id():
         assert np.array_equal(host_u32(U), want[40 + r][0]) and np.array_equal(host_u32(K), want[40 + r][1])
     assert int(ctr.item()) == 3
     M.mosaic_device_status()
+
+
+@pytest.mark.parametrize("n_pad", [16384, 32768])
+def test_rotation_and_encode_streamed_rows(n_pad):
+    """Rows of 16384 and 32768 whose length is a multiple of 32 run on the
+    persistent kernel that fetches each block's next row by TMA: more rows than
+    SMs (each block loops over several rows), a row stride above the length,
+    and a length below n_pad; rotation alone, and encode with and without the
+    mask, digit planes and rotation, all bit-exact."""
+    M = M_()
+    rows = 330 if n_pad == 16384 else 170
+    for n, ldx in ((n_pad, n_pad), (n_pad - 4096, n_pad - 4096 + 64)):
+        x = wl.spike_activations(rows, ldx, seed=n + 1)
+        x[3, :] = 0.0
+        x[5, 17] = np.nan
+        words = O.sample_signs(KEY, 13, n_pad)
+        y = torch.empty(rows, n_pad, dtype=torch.float32, device="cuda")
+        M.mosaic_hadamard(dev(x), ldx, y, rows, n, n_pad, dev(words))
+        want = O.fwht_rows(x[:, :n], n_pad, words)
+        got = host_f32(y)
+        # the NaN row: same NaN positions (payload bits may differ), every other value bit-exact
+        assert np.array_equal(np.isnan(got), np.isnan(want)), n
+        fin = ~np.isnan(want)
+        assert np.array_equal(got.view(np.uint32)[fin], want.view(np.uint32)[fin]), n
+        qmax = O.qmax_for(n_pad)
+        mask = wl.uniform_u32(17, rows, n_pad)
+        for rotate, use_mask, use_planes in ((1, True, True), (1, False, False), (0, True, False)):
+            out = torch.empty(rows, n_pad, dtype=torch.int32, device="cuda")
+            sc = torch.empty(rows, dtype=torch.float32, device="cuda")
+            planes = torch.empty(4, rows, n_pad, dtype=torch.int16, device="cuda") if use_planes else None
+            M.mosaic_encode(dev(x), ldx, rows, n, n_pad, qmax, rotate, dev(words),
+                            dev(mask) if use_mask else None, n_pad, out, n_pad, sc, planes)
+            if rotate:
+                v = want
+            else:
+                v = np.zeros((rows, n_pad), np.float32); v[:, :n] = x[:, :n]
+            code, scale = O.encode_rows(v, qmax)
+            got = host_u32(out)
+            assert np.array_equal(got, code + mask if use_mask else code), (n, rotate, use_mask)
+            gs = host_f32(sc)
+            assert np.array_equal(np.isnan(gs), np.isnan(scale))
+            assert np.array_equal(gs[~np.isnan(gs)], scale[~np.isnan(scale)])
+            if use_planes:
+                pl = host_f32(planes.view(torch.bfloat16).float()).astype(np.int64)
+                rebuilt = sum(pl[i] << (8 * i) for i in range(4)) % (1 << 32)
+                assert np.array_equal(rebuilt.astype(np.uint32), got)
+    M.mosaic_device_status()
