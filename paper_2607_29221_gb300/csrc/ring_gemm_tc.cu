@@ -451,19 +451,26 @@ __global__ void __launch_bounds__(THREADS, 1)
                         if (n0 + cc < nout) atomicAdd(crow + n0 + cc, acc[cc]);
                 } else if (vec) {
                     // Plain mode: C = Cin + acc.  Stream-K mode: C (prepared) += acc.
+                    // C may be Cin (in place), so the compiler keeps every load
+                    // behind the stores before it: the loads of 16 columns are
+                    // issued together, then their stores, so that a thread waits
+                    // for four round trips per tile instead of one per 4 columns.
                     const uint32_t *base = a.split ? crow : cin;
 #pragma unroll
-                    for (int cc = 0; cc < HB; cc += 4) {
-                        uint4 o = make_uint4(acc[cc], acc[cc + 1], acc[cc + 2], acc[cc + 3]);
-                        if (base) {
-                            const uint4 i4 = *reinterpret_cast<const uint4 *>(base + n0 + cc);
-                            o.x += i4.x; o.y += i4.y; o.z += i4.z; o.w += i4.w;
+                    for (int cb = 0; cb < HB; cb += 16) {
+                        uint4 ib[4], sb[4];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            ib[q] = base ? *reinterpret_cast<const uint4 *>(base + n0 + cb + 4 * q) : make_uint4(0, 0, 0, 0);
+                            sb[q] = sub ? *reinterpret_cast<const uint4 *>(sub + n0 + cb + 4 * q) : make_uint4(0, 0, 0, 0);
                         }
-                        if (sub) {
-                            const uint4 s4 = *reinterpret_cast<const uint4 *>(sub + n0 + cc);
-                            o.x -= s4.x; o.y -= s4.y; o.z -= s4.z; o.w -= s4.w;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const int cc = cb + 4 * q;
+                            const uint4 o = make_uint4(acc[cc] + ib[q].x - sb[q].x, acc[cc + 1] + ib[q].y - sb[q].y,
+                                                       acc[cc + 2] + ib[q].z - sb[q].z, acc[cc + 3] + ib[q].w - sb[q].w);
+                            *reinterpret_cast<uint4 *>(crow + n0 + cc) = o;
                         }
-                        *reinterpret_cast<uint4 *>(crow + n0 + cc) = o;
                     }
                 } else {
                     const uint32_t *base = a.split ? crow : cin;
