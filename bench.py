@@ -485,6 +485,17 @@ def run_mine(args, rank, world):
         parts("end")
     torch.cuda.synchronize()
     part_ms = {k: round(v / part_steps, 4) for k, v in parts.totals().items()}
+    # Per-kernel device time of eager steps (the library's own event pair
+    # around each launch, so not inside the timed steps above): the client
+    # kernels' rooflines.
+    M.mosaic_kernel_times(reset=True)
+    M.mosaic_kernel_timing(True)
+    for i in range(part_steps):
+        flush.fill_(i & 0xFF)
+        runner.step(X, 30_000 + i)
+    torch.cuda.synchronize()
+    M.mosaic_kernel_timing(False)
+    ktimes = M.mosaic_kernel_times(reset=True)
 
     # End to end through the public API with host buffers: the copy of X in
     # and of Y out inside the timed region, every step.
@@ -541,6 +552,8 @@ def run_mine(args, rank, world):
                   "achieved": round(enc_gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(enc_gbs / hbm, 4),
                   "traffic": None, "bytes_per_step": enc_bytes, "ms_per_step": round(enc_ms, 4),
                   "peak_source": f"{peak_src} copy bandwidth"}]
+    rooflines += _client_rooflines(ktimes, part_steps, runner.layers, proto, l, bf16, peak_src,
+                                   float(clocks.get("sm_mhz") or clocks.get("sm_max_mhz") or 2070.0))
     out = {
         "metric": METRIC, "value": round(tokens_s, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms_max, 4),
@@ -562,11 +575,74 @@ def run_mine(args, rank, world):
                 "launch": "one CUDA graph per step, the copy of X overlapping Init X",
                 "value_eager": round(world * l / (e2e_eager_ms_max / 1e3), 1)},
         "gpu_launches": int(launches_timed),
+        "kernel_ms_per_step": {k: round(v[1] / part_steps, 4) for k, v in sorted(ktimes.items())},
         "clocks": clocks,
     }
     if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(wk, args.cpu_budget_s)
     print(json.dumps(out), flush=True)
+
+
+# Derived peaks of the client kernels that neither copy bandwidth nor the
+# tensor cores bound (152 SMs at the median SM clock seen under load):
+# ChaCha20 draws against 64 32-bit integer ops per clock per SM (four
+# partitions of 16 INT32 lanes), the tiled gathers against one 128-byte
+# shared-memory wavefront per clock per SM.
+GB300_SMS = 152
+INT_OPS_PER_CLK_SM = 64
+SMEM_BYTES_PER_CLK_SM = 128
+CHACHA_OPS_PER_BLOCK = 20 * 4 * 12 + 16   # 80 quarter rounds of 12 add/xor/rotate, 16 final adds
+
+
+def _client_rooflines(kt, steps, layers, proto, l, bf16, peak_src, sm_mhz):
+    """Rooflines of the client kernels from the library's per-kernel event
+    times (`kt`: {"<role>:<kernel>": (launches, ms)} over `steps` eager steps).
+    Algorithmic work per step, summed over the step's secure linears:
+      draws   ChaCha20 blocks: R (l r_d words, 16 a block), the T lists (one
+              round of 32 blocks per token and level), E_x (l n_pad samples,
+              8 a block);
+      gathers one 4-byte shared-memory word per gathered MAC: Init X
+              l (n_pad + m) t_i per level, the unmask m l t_i per level;
+      K = r_d products 20 flops (10 bf16 digit pairs) per ring MAC: Init X
+              l (n_pad + m) r_d, the unmask l m r_d."""
+    p = proto.params
+    d = int(p.d)
+    r = [int(p.r[i]) for i in range(d)]
+    t = [int(p.t[i]) for i in range(d)]
+    nested = int(p.act_nested) != 0
+    r_act = r[d - 1] if nested else r[0]
+    act_lv = list(range(1, d)) if nested else []
+    w_lv = list(range(1, d))
+    clk = sm_mhz * 1e6
+    alu_peak = GB300_SMS * INT_OPS_PER_CLK_SM * clk / 1e12
+    smem_peak = GB300_SMS * SMEM_BYTES_PER_CLK_SM * clk / 1e9
+    blocks = sum(-(-l * r_act // 16) + len(act_lv) * l * 32 + -(-l * ly.n_pad // 8) for ly in layers)
+    gx = sum(l * (ly.n_pad + ly.m) * t[i] for ly in layers for i in act_lv)
+    gu = sum(ly.m * l * t[i] for ly in layers for i in w_lv)
+    fx = sum(20 * l * (ly.n_pad + ly.m) * r_act for ly in layers)
+    fu = sum(20 * l * ly.m * r[d - 1] for ly in layers)
+    rows = [("init_x:initx_draw", "initx_draw_kernel (Init X draws: R, T lists, E_x; ChaCha20)", "alu",
+             blocks * CHACHA_OPS_PER_BLOCK / 1e12, alu_peak, "Tops/s", "derived int32 ALU peak"),
+            ("init_x:pgather", "pgather_kernel (Init X LPN terms of U_x and K)", "smem",
+             gx * 4 / 1e9, smem_peak, "GB/s", "derived shared-memory wavefront peak"),
+            ("unmask:pgather", "pgather_kernel (unmask LPN terms + decode)", "smem",
+             gu * 4 / 1e9, smem_peak, "GB/s", "derived shared-memory wavefront peak"),
+            ("init_x:ring_gemm_tc", "ring_gemm_tc_kernel (Init X: R [C_d; J_d]^T, K = r_d)", "tensor",
+             fx / 1e12, bf16, "TFLOP/s", f"{peak_src} bf16 dense burst"),
+            ("unmask:ring_gemm_tc", "ring_gemm_tc_kernel (unmask: Y' - K - Q_d L^T, K = r_d)", "tensor",
+             fu / 1e12, bf16, "TFLOP/s", f"{peak_src} bf16 dense burst")]
+    out = []
+    for key, name, bound, work, peak, unit, src in rows:
+        n, ms = kt.get(key, (0, 0.0))
+        if n == 0 or ms <= 0.0 or work <= 0.0:
+            continue
+        ms_step = ms / steps
+        achieved = work / (ms_step / 1e3)
+        out.append({"kernel": name, "bound": bound, "achieved": round(achieved, 2), "peak": round(peak, 3),
+                    "unit": unit, "frac": round(achieved / peak, 4), "traffic": None,
+                    "ms_per_step": round(ms_step, 4), "launches_per_step": round(n / steps, 2),
+                    "peak_source": src})
+    return out
 
 
 def _roofline(variant, M, ring_macs, gemm_ms, bf16, peak_src, traffic):
@@ -580,7 +656,7 @@ def _roofline(variant, M, ring_macs, gemm_ms, bf16, peak_src, traffic):
     if variant == M.GEMM_MMA_S8:
         achieved = 10 * 2 * ring_macs / (gemm_ms / 1e3) / 1e12      # int8 digit-pair ops
         peak = 2 * bf16                                            # nominal int8 : bf16 = 2 : 1
-        return {"bound": "tensor", "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TOPS",
+        return {"bound": "tensor", "achieved": round(achieved, 2), "peak": round(peak, 3), "unit": "TOPS",
                 "frac": round(achieved / peak, 4), "traffic": traffic,
                 "kernel": "ring_gemm_s8 (mma.sync m16n8k32, 10 int8 digit-pair products per ring MAC)",
                 "peak_source": f"{peak_src} bf16 dense burst x 2 (nominal int8 ratio)"}

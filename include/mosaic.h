@@ -89,6 +89,27 @@ void mosaic_default_params(mosaic_params *p);
  * all threads; host-side counter, for benchmarking). */
 uint64_t mosaic_kernel_launches(void);
 
+/* Per-kernel device time, for measurement (not part of the method).
+ * mosaic_kernel_timing(1) makes every later launch of this library on a
+ * stream that is not being captured into a CUDA graph record a pair of CUDA
+ * events around itself, on that stream; mosaic_kernel_timing(0) stops it.
+ * Returns the previous setting.  Off by default (a launch then pays one atomic
+ * load).  Timing adds two event records per launch, so time whole steps with
+ * it off.
+ * mosaic_kernel_times waits for every recorded pair, adds the durations to
+ * per-key totals and writes up to `cap` of them to `out` (cap may be 0); the
+ * key is "<role>:<kernel>", role naming the entry point that launched the
+ * kernel (init_x, encode, server, unmask, init_w, ...).  With `reset` the
+ * totals start again from zero after being written.  Returns the number of
+ * keys, or -1 if an event could not be read (the records are dropped). */
+typedef struct {
+    char name[64];
+    uint64_t launches;
+    double ms;
+} mosaic_kernel_time;
+int mosaic_kernel_timing(int enable);
+int mosaic_kernel_times(mosaic_kernel_time *out, int cap, int reset);
+
 /* Human-readable name of a status code (static string). */
 const char *mosaic_status_string(mosaic_status s);
 

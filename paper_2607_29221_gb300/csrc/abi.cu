@@ -255,6 +255,7 @@ int mosaic_gaussian_table(float sigma, uint64_t *table, int capacity) {
 mosaic_status mosaic_prg_uniform(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
                                  uint32_t rounds, int64_t rows, int64_t cols, uint32_t *out,
                                  int64_t ldo, void *stream) {
+    RoleScope role("prg");
     if (!key || !rounds_ok(rounds)) return MOSAIC_ERR_ARG;
     if (rows < 0 || cols < 0 || ldo < cols) return MOSAIC_ERR_SHAPE;
     if (rows * cols >= ((int64_t)1 << 36)) return MOSAIC_ERR_SHAPE;
@@ -267,6 +268,7 @@ mosaic_status mosaic_prg_uniform(const mosaic_key *key, uint32_t tag, uint64_t s
 mosaic_status mosaic_prg_gaussian(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
                                   uint32_t rounds, float sigma, int64_t count, uint32_t *out,
                                   void *stream) {
+    RoleScope role("prg");
     if (!key || !rounds_ok(rounds)) return MOSAIC_ERR_ARG;
     if (!(sigma >= 0.0f && sigma <= 8.0f)) return MOSAIC_ERR_ARG;
     if (count < 0 || count >= ((int64_t)1 << 35)) return MOSAIC_ERR_SHAPE;
@@ -279,6 +281,7 @@ mosaic_status mosaic_prg_gaussian(const mosaic_key *key, uint32_t tag, uint64_t 
 mosaic_status mosaic_prg_sparse(const mosaic_key *key, uint32_t tag, uint64_t stream_id,
                                 uint32_t rounds, int64_t rows, uint32_t r, uint32_t t,
                                 uint32_t *idx, uint32_t *val, uint32_t *fail, void *stream) {
+    RoleScope role("prg");
     if (!key || !rounds_ok(rounds)) return MOSAIC_ERR_ARG;
     if (rows < 0 || rows >= ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
     if (t < 1 || t > 1024 || r < 2 || t > r / 2) return MOSAIC_ERR_ARG;
@@ -290,6 +293,7 @@ mosaic_status mosaic_prg_sparse(const mosaic_key *key, uint32_t tag, uint64_t st
 
 mosaic_status mosaic_hadamard(const float *x, int64_t ldx, float *y, int64_t rows, int64_t n,
                               int64_t n_pad, const uint32_t *sign_words, void *stream) {
+    RoleScope role("hadamard");
     if (!npad_ok(n_pad) || n < 1 || n > n_pad || rows < 0 || ldx < n) return MOSAIC_ERR_SHAPE;
     if (rows == 0) return MOSAIC_OK;
     if (!x || !y) return MOSAIC_ERR_ARG;
@@ -302,6 +306,7 @@ mosaic_status mosaic_encode(const float *x, int64_t ldx, int64_t rows, int64_t n
                             int32_t qmax, int rotate, const uint32_t *sign_words,
                             const uint32_t *mask, int64_t ldm, uint32_t *out, int64_t ldo,
                             float *scale, uint16_t *planes, void *stream) {
+    RoleScope role("encode");
     if (!npad_ok(n_pad) || n < 1 || n > n_pad || rows < 0 || ldx < n || ldo < n_pad)
         return MOSAIC_ERR_SHAPE;
     if (mask && ldm < n_pad) return MOSAIC_ERR_SHAPE;
@@ -317,6 +322,7 @@ mosaic_status mosaic_encode(const float *x, int64_t ldx, int64_t rows, int64_t n
 
 mosaic_status mosaic_digit_split(const uint32_t *a, int64_t lda, int64_t rows, int64_t cols,
                                  uint16_t *planes, void *stream) {
+    RoleScope role("digit_split");
     if (rows < 0 || cols < 0 || cols % 8 || lda < cols) return MOSAIC_ERR_SHAPE;
     if (rows == 0 || cols == 0) return MOSAIC_OK;
     if (!a || !planes) return MOSAIC_ERR_ARG;
@@ -337,6 +343,7 @@ int mosaic_gemm_variant_available(int variant) {
 mosaic_status mosaic_ring_gemm(const uint32_t *A, int64_t lda, const uint32_t *B, int64_t ldb,
                                uint32_t *C, int64_t ldc, int64_t M, int64_t N, int64_t K,
                                int variant, void *ws, size_t ws_bytes, void *stream) {
+    RoleScope role("ring_gemm");
     if (M < 0 || N < 0 || K < 0 || K > ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
     if (lda < K || ldb < K || ldc < N) return MOSAIC_ERR_SHAPE;
     if (variant < MOSAIC_GEMM_AUTO || variant > MOSAIC_GEMM_IMAD) return MOSAIC_ERR_ARG;
@@ -378,6 +385,7 @@ mosaic_status mosaic_ring_gemm_planes(const uint16_t *A_planes, int64_t ldpa, in
                                       const uint16_t *B_planes, int64_t ldpb, int64_t b_plane,
                                       uint32_t *C, int64_t ldc, int64_t M, int64_t N, int64_t K,
                                       int variant, void *stream) {
+    RoleScope role("ring_gemm");
     if (M < 0 || N < 0 || K < 0 || K > ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
     if (ldpa < K || ldpb < K || ldc < N || a_plane < M * ldpa || b_plane < N * ldpb)
         return MOSAIC_ERR_SHAPE;
@@ -431,6 +439,7 @@ size_t mosaic_workspace_bytes(int op, int64_t m, int64_t n_pad, int64_t l, const
 mosaic_status mosaic_mask_chains(const mosaic_params *p, const mosaic_key *key, uint64_t chain_id,
                                  int64_t n_pad, uint32_t *P, uint32_t *C, uint32_t *CT, void *ws,
                                  size_t ws_bytes, void *stream) {
+    RoleScope role("init_w");
     MOSAIC_TRY(check_params(p));
     if (!key) return MOSAIC_ERR_ARG;
     if (!npad_ok(n_pad)) return MOSAIC_ERR_SHAPE;
@@ -468,6 +477,7 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, 
                                  float *s_w, uint32_t *L, uint32_t *S_idx, uint32_t *S_val,
                                  uint32_t *Wp, uint16_t *Wp_planes, uint32_t *J, int variant,
                                  void *ws, size_t ws_bytes, void *stream) {
+    RoleScope role("init_w");
     MOSAIC_TRY(check_params(p));
     if (!key) return MOSAIC_ERR_ARG;
     if (!npad_ok(n_pad) || n < 1 || n > n_pad || m < 1 || ldw < n || m >= ((int64_t)1 << 20))
@@ -534,6 +544,7 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
                                    const uint32_t *C, const uint32_t *J, const uint16_t *cj,
                                    uint32_t *Ux_tm, uint32_t *K_tm, int variant, void *ws,
                                    size_t ws_bytes, void *stream) {
+    RoleScope role("init_x");
     MOSAIC_TRY(check_params(p));
     if (!key) return MOSAIC_ERR_ARG;
     if (!npad_ok(n_pad) || m < 1 || l < 0 || l >= ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
@@ -681,6 +692,7 @@ mosaic_status mosaic_advance_pass(uint64_t *pass_dev, uint64_t delta, void *stre
 mosaic_status mosaic_prepare_activation(const mosaic_params *p, int64_t m, int64_t n_pad,
                                         const uint32_t *C, const uint32_t *J, uint16_t *cj_planes,
                                         void *stream) {
+    RoleScope role("prepare");
     MOSAIC_TRY(check_params(p));
     if (!npad_ok(n_pad) || m < 1) return MOSAIC_ERR_SHAPE;
     if (!C || !J || !cj_planes) return MOSAIC_ERR_ARG;
@@ -713,6 +725,7 @@ mosaic_status unmask_impl(const mosaic_params *p, int64_t l, int64_t m, const ui
                           const uint32_t *S_val, const float *s_w, const float *s_x, const float *bias,
                           float *Y, uint32_t *Yhat, int64_t ldy, int variant, void *ws, size_t ws_bytes,
                           void *stream) {
+    RoleScope role("unmask");
     MOSAIC_TRY(check_params(p));
     const uint32_t d = p->d;
     const int64_t Sr = sum_r(p), rd = p->r[d - 1], od = off_r(p, d);
@@ -811,6 +824,7 @@ mosaic_status mosaic_unmask_planes(const mosaic_params *p, int64_t l, int64_t m,
 
 mosaic_status mosaic_prepare_unmask(const mosaic_params *p, int64_t m, const uint32_t *L, uint16_t *L_planes,
                                     void *stream) {
+    RoleScope role("prepare");
     MOSAIC_TRY(check_params(p));
     if (m < 1) return MOSAIC_ERR_SHAPE;
     if (!L || !L_planes) return MOSAIC_ERR_ARG;
@@ -822,6 +836,7 @@ mosaic_status mosaic_prepare_unmask(const mosaic_params *p, int64_t m, const uin
 mosaic_status mosaic_freivalds_setup(const mosaic_params *p, const mosaic_key *key, uint64_t matrix_id,
                                      int k, const uint32_t *Wm, int64_t ldw, int64_t m, int64_t n_pad,
                                      uint32_t *a, uint32_t *Ychk, void *stream) {
+    RoleScope role("freivalds");
     MOSAIC_TRY(check_params(p));
     if (!key) return MOSAIC_ERR_ARG;
     if (k < 1 || k > 16) return MOSAIC_ERR_ARG;
@@ -836,6 +851,7 @@ mosaic_status mosaic_freivalds_check(int k, const uint32_t *a, const uint32_t *Y
                                      int64_t n_pad, int64_t l, const uint32_t *Z, int64_t ldz,
                                      const uint32_t *Xp, int64_t ldx, uint32_t *bad, uint32_t *n_bad,
                                      void *ws, size_t ws_bytes, void *stream) {
+    RoleScope role("freivalds");
     if (k < 1 || k > 16) return MOSAIC_ERR_ARG;
     if (m < 1 || n_pad < 1 || l < 0 || ldz < m || ldx < n_pad) return MOSAIC_ERR_SHAPE;
     if (l == 0) return MOSAIC_OK;

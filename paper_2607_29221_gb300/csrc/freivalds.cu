@@ -70,7 +70,10 @@ mosaic_status freivalds_colsum(const uint32_t *a, int k, const uint32_t *W, int6
     if (rows < 64) rows = 64;
     yblocks = (m + rows - 1) / rows;
     if (xblocks > 0x7fffffff || yblocks > 65535) return MOSAIC_ERR_SHAPE;
-    colsum_kernel<<<dim3((unsigned)xblocks, (unsigned)yblocks), 256, 0, st>>>(a, k, W, ldw, m, ncols, rows, Y);
+    {
+        KernelSpan span("freivalds_colsum", st);
+        colsum_kernel<<<dim3((unsigned)xblocks, (unsigned)yblocks), 256, 0, st>>>(a, k, W, ldw, m, ncols, rows, Y);
+    }
     return launch_status();
 }
 
@@ -79,7 +82,10 @@ mosaic_status freivalds_check(int k, const uint32_t *a, const uint32_t *Ychk, in
                               uint32_t *bad, uint32_t *n_bad, uint32_t *lhs, uint32_t *rhs, cudaStream_t st) {
     MOSAIC_TRY(skinny_or_imad(a, m, Z, ldz, lhs, k, l, m, st));
     MOSAIC_TRY(skinny_or_imad(Ychk, n_pad, Xp, ldx, rhs, k, l, n_pad, st));
-    compare_kernel<<<(unsigned)((l + 255) / 256), 256, 0, st>>>(lhs, rhs, k, l, bad, n_bad);
+    {
+        KernelSpan span("freivalds_compare", st);
+        compare_kernel<<<(unsigned)((l + 255) / 256), 256, 0, st>>>(lhs, rhs, k, l, bad, n_bad);
+    }
     return launch_status();
 }
 

@@ -362,7 +362,10 @@ mosaic_status launch(const FwhtArgs &a, cudaStream_t st) {
             return MOSAIC_ERR_CUDA;
     }
     const int64_t blocks = (a.rows + C::RPB - 1) / C::RPB;
-    fwht_kernel<E, T><<<(unsigned)blocks, T * C::RPB, C::SMEM, st>>>(a);
+    {
+        KernelSpan span("fwht", st);
+        fwht_kernel<E, T><<<(unsigned)blocks, T * C::RPB, C::SMEM, st>>>(a);
+    }
     return launch_status();
 }
 
@@ -665,7 +668,10 @@ mosaic_status launch_stream(const FwhtArgs &a, cudaStream_t st) {
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
         return MOSAIC_ERR_CUDA;
     const int64_t grid = a.rows < sms ? a.rows : sms;
-    fwht_stream_kernel<T><<<(unsigned)grid, T, C::SMEM, st>>>(tmx, tmm, a, has_m);
+    {
+        KernelSpan span("fwht_stream", st);
+        fwht_stream_kernel<T><<<(unsigned)grid, T, C::SMEM, st>>>(tmx, tmm, a, has_m);
+    }
     return launch_status();
 }
 
@@ -773,17 +779,29 @@ mosaic_status fwht65536(FwhtArgs a, cudaStream_t st) {
     const dim3 grid((unsigned)(kHalf / (256 * 4)), (unsigned)rows);
     if (rows > 65535) return MOSAIC_ERR_SHAPE;
     if (a.mode == 0) {
-        combine_kernel<<<grid, 256, 0, st>>>(y, ldy, rows, a.rotate, nullptr);
+        {
+            KernelSpan span("fwht_combine", st);
+            combine_kernel<<<grid, 256, 0, st>>>(y, ldy, rows, a.rotate, nullptr);
+        }
         return launch_status();
     }
     uint32_t *amax = reinterpret_cast<uint32_t *>(a.scale);
     if (cudaMemsetAsync(amax, 0, sizeof(uint32_t) * (size_t)rows, st) != cudaSuccess) return MOSAIC_ERR_CUDA;
-    combine_kernel<<<grid, 256, 0, st>>>(y, ldy, rows, a.rotate, amax);
+    {
+        KernelSpan span("fwht_combine", st);
+        combine_kernel<<<grid, 256, 0, st>>>(y, ldy, rows, a.rotate, amax);
+    }
     MOSAIC_TRY(launch_status());
-    scale_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(a.scale, rows, a.qmax);
+    {
+        KernelSpan span("fwht_scale", st);
+        scale_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(a.scale, rows, a.qmax);
+    }
     MOSAIC_TRY(launch_status());
     const dim3 g2((unsigned)(65536 / (256 * 4)), (unsigned)rows);
-    quantize_kernel<<<g2, 256, 0, st>>>(a.out, a.ldo, a.scale, a.qmax, a.mask, a.ldm, a.planes, rows);
+    {
+        KernelSpan span("fwht_quantize", st);
+        quantize_kernel<<<g2, 256, 0, st>>>(a.out, a.ldo, a.scale, a.qmax, a.mask, a.ldm, a.planes, rows);
+    }
     return launch_status();
 }
 

@@ -92,6 +92,27 @@ inline mosaic_status launch_status() {
     return MOSAIC_OK;
 }
 
+// Optional per-kernel device timing (mosaic_kernel_timing).  A launcher opens
+// a KernelSpan right before its launch and lets it close after; while timing
+// is on and `st` is not being captured, the span brackets the launch with a
+// CUDA event pair keyed by "<role>:<kernel>", the role being the entry point
+// that made the call (set by a RoleScope there).
+struct KernelSpan {
+    KernelSpan(const char *kernel, cudaStream_t st);
+    ~KernelSpan();
+    KernelSpan(const KernelSpan &) = delete;
+    KernelSpan &operator=(const KernelSpan &) = delete;
+    void *slot_ = nullptr;
+    cudaStream_t st_;
+};
+struct RoleScope {
+    explicit RoleScope(const char *role);
+    ~RoleScope();
+    RoleScope(const RoleScope &) = delete;
+    RoleScope &operator=(const RoleScope &) = delete;
+    const char *prev_;
+};
+
 #define MOSAIC_TRY(expr)                        \
     do {                                        \
         mosaic_status _s = (expr);              \

@@ -299,8 +299,11 @@ mosaic_status prg_uniform(const Key &key, uint32_t tag, uint64_t sid, int rounds
     const int64_t total = rows * cols;
     if (total == 0) return MOSAIC_OK;
     const int64_t nblk = (total + 15) / 16;
-    uniform_kernel<<<prg_blocks(nblk, kThreads), kThreads, 0, st>>>(
-        key, tag, sid, sid_dev, rounds, cols, total, out, ldo);
+    {
+        KernelSpan span("prg_uniform", st);
+        uniform_kernel<<<prg_blocks(nblk, kThreads), kThreads, 0, st>>>(
+            key, tag, sid, sid_dev, rounds, cols, total, out, ldo);
+    }
     return launch_status();
 }
 
@@ -315,8 +318,11 @@ mosaic_status prg_gaussian(const Key &key, uint32_t tag, uint64_t sid, int round
     tab.bound = gaussian_table_host(sigma, tab.t);
     tab.n = 2 * tab.bound + 1;
     const int64_t nblk = (count + 7) / 8;
-    gaussian_kernel<<<prg_blocks(nblk, kThreads), kThreads, 0, st>>>(
-        key, tag, sid, sid_dev, rounds, tab, count, out);
+    {
+        KernelSpan span("prg_gaussian", st);
+        gaussian_kernel<<<prg_blocks(nblk, kThreads), kThreads, 0, st>>>(
+            key, tag, sid, sid_dev, rounds, tab, count, out);
+    }
     return launch_status();
 }
 
@@ -378,7 +384,10 @@ mosaic_status prg_initx(const Key &key, int rounds, uint64_t sid, const uint64_t
         cudaFuncSetAttribute(initx_draw_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
             cudaSuccess)
         return MOSAIC_ERR_CUDA;
-    initx_draw_kernel<<<(unsigned)grid, kDrawThreads, smem, st>>>(a);
+    {
+        KernelSpan span("initx_draw", st);
+        initx_draw_kernel<<<(unsigned)grid, kDrawThreads, smem, st>>>(a);
+    }
     return launch_status();
 }
 
@@ -392,8 +401,11 @@ mosaic_status prg_sparse(const Key &key, uint32_t tag, uint64_t sid, int rounds,
         cudaFuncSetAttribute(sparse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
             cudaSuccess)
         return MOSAIC_ERR_CUDA;
-    sparse_kernel<<<(unsigned)((rows + kSparseWarps - 1) / kSparseWarps), kSparseWarps * 32, smem, st>>>(
-        key, tag, sid, sid_dev, rounds, rows, r, (int)t, idx, val, fail, bitmap_words);
+    {
+        KernelSpan span("prg_sparse", st);
+        sparse_kernel<<<(unsigned)((rows + kSparseWarps - 1) / kSparseWarps), kSparseWarps * 32, smem, st>>>(
+            key, tag, sid, sid_dev, rounds, rows, r, (int)t, idx, val, fail, bitmap_words);
+    }
     return launch_status();
 }
 

@@ -104,7 +104,10 @@ mosaic_status ring_gemm_imad(const uint32_t *A, int64_t sai, int64_t sak, const 
     GemmArgs a{A, sai, sak, B, sbj, sbk, C, ldc, Cin, ldcin, sgn, M, N, K};
     const int64_t gx = (N + BN - 1) / BN, gy = (M + BM - 1) / BM;
     if (gy > 65535) return MOSAIC_ERR_SHAPE;
-    ring_gemm_imad_kernel<<<dim3((unsigned)gx, (unsigned)gy), NT, 0, st>>>(a);
+    {
+        KernelSpan span("ring_gemm_imad", st);
+        ring_gemm_imad_kernel<<<dim3((unsigned)gx, (unsigned)gy), NT, 0, st>>>(a);
+    }
     return launch_status();
 }
 

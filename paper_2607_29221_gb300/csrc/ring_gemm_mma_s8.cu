@@ -187,15 +187,24 @@ mosaic_status ring_gemm_mma_s8(const uint32_t *A, int64_t lda, const uint32_t *B
     if (!ws || ws_bytes < ws_mma_s8(M, N, K)) return MOSAIC_ERR_WORKSPACE;
     int8_t *Ap = reinterpret_cast<int8_t *>((reinterpret_cast<uintptr_t>(ws) + 255) & ~static_cast<uintptr_t>(255));
     int8_t *Bp = Ap + ((4 * M * ldp + 255) / 256) * 256;
-    split_s8_kernel<<<grid_for(M * (ldp / 4), 256), 256, 0, st>>>(A, lda, M, K, Ap, ldp, M * ldp);
+    {
+        KernelSpan span("split_s8", st);
+        split_s8_kernel<<<grid_for(M * (ldp / 4), 256), 256, 0, st>>>(A, lda, M, K, Ap, ldp, M * ldp);
+    }
     MOSAIC_TRY(launch_status());
-    split_s8_kernel<<<grid_for(N * (ldp / 4), 256), 256, 0, st>>>(B, ldb, N, K, Bp, ldp, N * ldp);
+    {
+        KernelSpan span("split_s8", st);
+        split_s8_kernel<<<grid_for(N * (ldp / 4), 256), 256, 0, st>>>(B, ldb, N, K, Bp, ldp, N * ldp);
+    }
     MOSAIC_TRY(launch_status());
     static std::atomic<unsigned long long> attr_set{0};   // one bit per device ordinal
     if (!ensure_smem_limit(attr_set, ring_gemm_s8_kernel, 2 * STAGE_B)) return MOSAIC_ERR_CUDA;
     S8Args args{Ap, Bp, ldp, M * ldp, N * ldp, C, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)(ldp / TK)};
     const dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
-    ring_gemm_s8_kernel<<<grid, THREADS, 2 * STAGE_B, st>>>(args);
+    {
+        KernelSpan span("ring_gemm_s8", st);
+        ring_gemm_s8_kernel<<<grid, THREADS, 2 * STAGE_B, st>>>(args);
+    }
     return launch_status();
 }
 

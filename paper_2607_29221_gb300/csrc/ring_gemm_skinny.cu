@@ -215,7 +215,10 @@ mosaic_status launch_skinny(const uint32_t *A, int64_t lda, const uint32_t *B, i
     if (tiles > 0x7fffffff || nk > 0x7fffffff) return MOSAIC_ERR_SHAPE;
     SkArgs args{Cm, ldc, Cin, ldcin, sgn, (int)M, (int)N, (int)nk, (int)tiles};
     const int grid = tiles < sms ? (int)tiles : sms;
-    ring_gemm_skinny_kernel<MT, RW><<<grid, THREADS, C::SMEM, st>>>(ta, tb, args);
+    {
+        KernelSpan span("ring_gemm_skinny", st);
+        ring_gemm_skinny_kernel<MT, RW><<<grid, THREADS, C::SMEM, st>>>(ta, tb, args);
+    }
     return launch_status();
 }
 

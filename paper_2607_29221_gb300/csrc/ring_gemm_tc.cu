@@ -571,7 +571,10 @@ mosaic_status launch_tc(const uint16_t *Ap, int64_t ldpa, int64_t a_plane, const
         args.dp_tiles = (int)((tiles / grid) * grid);   // whole waves run as whole tiles
     }
     if (grid > 0x7fffffff) return MOSAIC_ERR_SHAPE;
-    ring_gemm_tc_kernel<BN><<<(unsigned)grid, THREADS, C::SMEM, st>>>(ta, tb, args);
+    {
+        KernelSpan span("ring_gemm_tc", st);
+        ring_gemm_tc_kernel<BN><<<(unsigned)grid, THREADS, C::SMEM, st>>>(ta, tb, args);
+    }
     return launch_status();
 }
 

@@ -490,7 +490,10 @@ mosaic_status launch_tcw(const CUtensorMap &tw, const CUtensorMap &tx, const WAr
     if (!ensure_smem_limit(attr_set, ring_gemm_tcw_kernel<NT>, C::SMEM)) return MOSAIC_ERR_CUDA;
     const int64_t units = (int64_t)args.tiles * args.nchunks;
     const int64_t grid = units < sms ? units : sms;
-    ring_gemm_tcw_kernel<NT><<<(unsigned)grid, THREADS, C::SMEM, st>>>(tw, tx, args);
+    {
+        KernelSpan span("ring_gemm_tcw", st);
+        ring_gemm_tcw_kernel<NT><<<(unsigned)grid, THREADS, C::SMEM, st>>>(tw, tx, args);
+    }
     return launch_status();
 }
 
@@ -519,8 +522,11 @@ mosaic_status ring_gemm_tcw(const uint32_t *A, int64_t lda, const uint32_t *B, i
         return MOSAIC_ERR_SHAPE;
     if (!aligned16(Ap)) return MOSAIC_ERR_ALIGN;
     const int64_t Kp = (K + 7) / 8 * 8;
-    split_f16_zero_kernel<<<grid_for(M * (K > N ? K : N), 256), 256, 0, st>>>(A, lda, M, K, Ap, Kp, M * Kp, Cm, ldc,
-                                                                               N);
+    {
+        KernelSpan span("split_f16_zero", st);
+        split_f16_zero_kernel<<<grid_for(M * (K > N ? K : N), 256), 256, 0, st>>>(A, lda, M, K, Ap, Kp, M * Kp, Cm, ldc,
+                                                                                   N);
+    }
     MOSAIC_TRY(launch_status());
     const int nt = M <= 32 ? 32 : M <= 48 ? 48 : 64;
     CUtensorMap tw, tx;

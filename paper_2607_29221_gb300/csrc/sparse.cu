@@ -523,7 +523,10 @@ mosaic_status launch_pgather(const GatherArgs &a, cudaStream_t st) {
         vec_ab = vec_ab && (!a.a2 || (aligned16(a.a2) && a.lda2 % 4 == 0)) &&
                  (!a.out2 || (aligned16(a.out2) && a.ldo2 % 4 == 0));
     }
-    kern<<<(unsigned)grid, kPgWarps * 32, smem, st>>>(a, (int)units, (int)units0, (int)chunks, vec_src, vec_ab);
+    {
+        KernelSpan span("pgather", st);
+        kern<<<(unsigned)grid, kPgWarps * 32, smem, st>>>(a, (int)units, (int)units0, (int)chunks, vec_src, vec_ab);
+    }
     return launch_status();
 }
 
@@ -603,7 +606,10 @@ mosaic_status launch_few(const GatherArgs &a, cudaStream_t st) {
     // Enough warps to stream the lists; every block stages the rows once.
     const int64_t need = (a.nlist + kFewWarps - 1) / kFewWarps;
     const int64_t cap = (int64_t)sms * 4;
-    kern<<<(unsigned)(need < cap ? need : cap), kFewWarps * 32, smem, st>>>(a);
+    {
+        KernelSpan span("gather_few", st);
+        kern<<<(unsigned)(need < cap ? need : cap), kFewWarps * 32, smem, st>>>(a);
+    }
     return launch_status();
 }
 
@@ -616,7 +622,10 @@ mosaic_status launch_gather(const GatherArgs &a, cudaStream_t st) {
         return MOSAIC_ERR_CUDA;
     dim3 grid((unsigned)((a.nlist + G_ENTS - 1) / G_ENTS), (unsigned)((a.g_count + TG - 1) / TG));
     if (grid.y > 65535) return MOSAIC_ERR_SHAPE;
-    gather_kernel<TG, LIST_IS_COL, CLAMP><<<grid, GW * 32, smem, st>>>(a);
+    {
+        KernelSpan span("gather", st);
+        gather_kernel<TG, LIST_IS_COL, CLAMP><<<grid, GW * 32, smem, st>>>(a);
+    }
     return launch_status();
 }
 
@@ -885,8 +894,11 @@ mosaic_status build_tile_image(const uint32_t *src, int64_t lds, int64_t col0, u
     const int rp = (int)((r + 31) / 32 * 32);
     const int64_t tiles = (g_count + kPgRows - 1) / kPgRows;
     if (tiles > 65535) return MOSAIC_ERR_SHAPE;
-    tile_image_kernel<<<dim3((unsigned)(rp / 32), (unsigned)tiles), 256, 0, st>>>(src, lds, col0, (int)r, g_count,
-                                                                                  rp, img);
+    {
+        KernelSpan span("tile_image", st);
+        tile_image_kernel<<<dim3((unsigned)(rp / 32), (unsigned)tiles), 256, 0, st>>>(src, lds, col0, (int)r, g_count,
+                                                                                      rp, img);
+    }
     return launch_status();
 }
 
@@ -937,7 +949,10 @@ mosaic_status unmask_prep(const uint32_t *Z, int64_t ldz, int64_t l, int64_t qco
     }
     if (grid == 0) return MOSAIC_OK;
     if (grid > 0x7fffffff) return MOSAIC_ERR_SHAPE;
-    unmask_prep_kernel<<<(unsigned)grid, 256, 0, st>>>(a);
+    {
+        KernelSpan span("unmask_prep", st);
+        unmask_prep_kernel<<<(unsigned)grid, 256, 0, st>>>(a);
+    }
     return launch_status();
 }
 
@@ -1070,14 +1085,20 @@ mosaic_status sparse_rowgather(const uint32_t *P, int64_t ldp, const SparseLevel
     SparseLevel l0 = nlev > 0 ? lev[0] : SparseLevel{nullptr, nullptr, 0, 0, 0};
     SparseLevel l1 = nlev > 1 ? lev[1] : SparseLevel{nullptr, nullptr, 0, 0, 0};
     dim3 grid((unsigned)((ncols + 255) / 256), (unsigned)m);
-    rowgather_kernel<<<grid, 256, 0, st>>>(P, ldp, l0, l1, nlev, ncols, a, lda, out, ldo);
+    {
+        KernelSpan span("rowgather", st);
+        rowgather_kernel<<<grid, 256, 0, st>>>(P, ldp, l0, l1, nlev, ncols, a, lda, out, ldo);
+    }
     return launch_status();
 }
 
 mosaic_status add_u32(const uint32_t *a, int64_t lda, const uint32_t *b, int64_t ldb, uint32_t *out,
                       int64_t ldo, int64_t rows, int64_t cols, cudaStream_t st) {
     if (rows == 0 || cols == 0) return MOSAIC_OK;
-    add_kernel<<<grid_for(rows * cols, 256), 256, 0, st>>>(a, lda, b, ldb, out, ldo, rows, cols);
+    {
+        KernelSpan span("ring_add", st);
+        add_kernel<<<grid_for(rows * cols, 256), 256, 0, st>>>(a, lda, b, ldb, out, ldo, rows, cols);
+    }
     return launch_status();
 }
 
@@ -1086,7 +1107,10 @@ mosaic_status transpose_u32(const uint32_t *a, int64_t lda, int64_t rows, int64_
     if (rows == 0 || cols == 0) return MOSAIC_OK;
     dim3 grid((unsigned)((cols + 31) / 32), (unsigned)((rows + 31) / 32));
     if (grid.y > 65535) return MOSAIC_ERR_SHAPE;
-    transpose_kernel<<<grid, dim3(32, 8), 0, st>>>(a, lda, rows, cols, out, ldo);
+    {
+        KernelSpan span("transpose", st);
+        transpose_kernel<<<grid, dim3(32, 8), 0, st>>>(a, lda, rows, cols, out, ldo);
+    }
     return launch_status();
 }
 
@@ -1096,8 +1120,11 @@ mosaic_status digit_split(const uint32_t *a, int64_t lda, int64_t rows, int64_t 
     const int vec = (lda % 4 == 0) && (ldp % 4 == 0) && (plane_stride % 4 == 0) &&
                     (reinterpret_cast<uintptr_t>(a) & 15u) == 0 &&
                     (reinterpret_cast<uintptr_t>(planes) & 7u) == 0;
-    digit_split_kernel<<<grid_for(rows * ((cols + 3) / 4), 256), 256, 0, st>>>(
-        a, lda, rows, cols, planes, ldp, plane_stride, vec);
+    {
+        KernelSpan span("digit_split", st);
+        digit_split_kernel<<<grid_for(rows * ((cols + 3) / 4), 256), 256, 0, st>>>(
+            a, lda, rows, cols, planes, ldp, plane_stride, vec);
+    }
     return launch_status();
 }
 

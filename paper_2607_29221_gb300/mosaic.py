@@ -56,6 +56,10 @@ class mosaic_mask_io(ctypes.Structure):
                 ("pass_dev", ctypes.c_void_p), ("Ux_tm", ctypes.c_void_p), ("K_tm", ctypes.c_void_p)]
 
 
+class mosaic_kernel_time(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 64), ("launches", ctypes.c_uint64), ("ms", ctypes.c_double)]
+
+
 _lib = None
 _P, _I64, _U32, _U64, _INT, _F32 = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_uint32,
                                     ctypes.c_uint64, ctypes.c_int, ctypes.c_float)
@@ -66,6 +70,8 @@ _PK = ctypes.POINTER(mosaic_key)
 _SIGS = {
     "mosaic_default_params": ([_PP], None),
     "mosaic_kernel_launches": ([], ctypes.c_uint64),
+    "mosaic_kernel_timing": ([_INT], _INT),
+    "mosaic_kernel_times": ([ctypes.POINTER(mosaic_kernel_time), _INT, _INT], _INT),
     "mosaic_status_string": ([_INT], ctypes.c_char_p),
     "mosaic_qmax": ([_I64, _U32], ctypes.c_int32),
     "mosaic_gaussian_table": ([_F32, _P, _INT], _INT),
@@ -177,6 +183,23 @@ def _call(name, *args):
 # ---------------------------------------------------------------------------
 def mosaic_kernel_launches() -> int:
     return int(lib().mosaic_kernel_launches())
+
+
+def mosaic_kernel_timing(enable: bool) -> bool:
+    """Turns per-kernel event timing on or off; returns the previous setting."""
+    return bool(lib().mosaic_kernel_timing(1 if enable else 0))
+
+
+def mosaic_kernel_times(reset: bool = True) -> dict:
+    """{"<role>:<kernel>": (launches, total ms)} of the launches timed so far."""
+    n = int(lib().mosaic_kernel_times(None, 0, 0))
+    if n < 0:
+        raise MosaicError("mosaic_kernel_times", -1)
+    buf = (mosaic_kernel_time * max(n, 1))()
+    n = int(lib().mosaic_kernel_times(buf, n, 1 if reset else 0))
+    if n < 0:
+        raise MosaicError("mosaic_kernel_times", -1)
+    return {buf[i].name.decode(): (int(buf[i].launches), float(buf[i].ms)) for i in range(min(n, len(buf)))}
 
 
 def mosaic_qmax(n_pad: int, qbits: int = 16) -> int:

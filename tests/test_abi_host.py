@@ -178,3 +178,12 @@ def test_mosaic_mask_dispatch_validation(lib):
     bad = M.default_params(act_nested=2)
     assert _status("mosaic_mask", M.MASK_ACTIVATION, ctypes.byref(bad), ctypes.byref(key), 0, 8, 32, 4,
                    ctypes.byref(io), 0, None, 0, None) == 1
+
+
+def test_kernel_timing_toggle_without_gpu(lib):
+    """Per-kernel timing is off by default, toggles, and reports no records
+    when nothing was launched."""
+    from paper_2607_29221_gb300 import mosaic as M
+    assert M.mosaic_kernel_timing(True) is False
+    assert M.mosaic_kernel_timing(False) is True
+    assert M.mosaic_kernel_times(reset=True) == {}

@@ -37,3 +37,38 @@ def test_default_workload_is_the_decoder_layer():
     cfg = bench._config(__import__("paper_2607_29221_gb300.workloads", fromlist=["x"]).WORKLOADS[
         bench.DEFAULT_WORKLOAD], 1)
     assert cfg["l"] == 2048 and [x["m"] for x in cfg["linears"]] == [10240, 8192, 57344, 8192]
+
+
+def test_client_rooflines_count_the_work_of_the_7b_step():
+    """Algorithmic work of the client kernels on the 7B attention projection
+    (l = 512, n = m = 4096, Example 3.1 parameters): 315,776 ChaCha20 blocks,
+    2 x 512 x 8192 x 80 gathered MACs in Init X and 2 x 4096 x 512 x 80 in the
+    unmask, 20 x 512 x 8192 x 652 and 20 x 512 x 4096 x 652 product flops."""
+    sys.path.insert(0, ROOT)
+    import types
+    import bench
+    from paper_2607_29221_gb300 import mosaic as M
+    proto = types.SimpleNamespace(params=M.default_params())
+    layer = types.SimpleNamespace(m=4096, n_pad=4096)
+    kt = {"init_x:initx_draw": (2, 2e-3 * 2), "init_x:pgather": (4, 4e-3 * 2),
+          "unmask:pgather": (4, 4e-3 * 2), "init_x:ring_gemm_tc": (2, 2e-3 * 2),
+          "unmask:ring_gemm_tc": (2, 2e-3 * 2)}
+    rows = bench._client_rooflines(kt, 2, [layer], proto, 512, 1910.6, "measured", 2070.0)
+    assert len(rows) == 5
+
+    def row(text):
+        return [r for r in rows if text in r["kernel"]][0]
+    clk = 2070e6
+    draw = row("initx_draw_kernel")
+    assert abs(draw["achieved"] - 315_776 * 976 / 2e-6 / 1e12) < 0.01
+    assert abs(draw["peak"] - round(152 * 64 * clk / 1e12, 3)) < 1e-9
+    gx = row("Init X LPN")
+    assert abs(gx["achieved"] - 2 * 512 * 8192 * 80 * 4 / 4e-6 / 1e9) < 0.01
+    assert abs(gx["peak"] - round(152 * 128 * clk / 1e9, 3)) < 1e-9
+    gu = row("unmask LPN")
+    assert abs(gu["achieved"] - 2 * 4096 * 512 * 80 * 4 / 4e-6 / 1e9) < 0.01
+    tcx = row("Init X: R")
+    assert abs(tcx["achieved"] - 20 * 512 * 8192 * 652 / 2e-6 / 1e12) < 0.01
+    tcu = row("unmask: Y'")
+    assert abs(tcu["achieved"] - 20 * 512 * 4096 * 652 / 2e-6 / 1e12) < 0.01
+    assert all(abs(r["frac"] / (r["achieved"] / r["peak"]) - 1) < 1e-3 for r in rows)

@@ -77,3 +77,54 @@ def test_graph_step_matches_eager_passes(l):
     assert int(ctr.item()) == 2
     assert not np.array_equal(eager[0][0], eager[1][0])   # fresh masks per pass
     M.mosaic_device_status()
+
+
+def test_kernel_timing_records_eager_launches_only():
+    """Per-kernel timing: an eager step with timing on records every launch
+    of the library (Init X draws, product and gathers, the server product, the
+    unmask) under the entry point that made it, as many as the launch counter
+    saw, with the outputs unchanged; a launch captured into a CUDA graph is
+    not recorded."""
+    from paper_2607_29221_gb300 import mosaic as M
+    from paper_2607_29221_gb300 import protocol as PR
+    gp = M.default_params(d=3, r=[96, 64, 40], t=[0, 8, 4])
+    proto = PR.Protocol(KEY, gp, variant=M.GEMM_TC)
+    m, n, l = 256, 256, 64
+    ch = PR.Chains(proto, PR.pad_width(n))
+    layer = PR.SecureLinear(proto, torch.from_numpy(wl.weights(m, n, std=1.0)).cuda(), 3, ch)
+    X = torch.from_numpy(wl.activations(l, n)).cuda()
+    Y0 = layer.forward(X, layer.init_x(l, 77)).clone()
+    mp = layer.init_x(l, 78)
+    Xp = torch.empty(l, layer.n_pad, dtype=torch.int32, device="cuda")
+    s_x = torch.empty(l, dtype=torch.float32, device="cuda")
+    Xpl = torch.empty(4, l, layer.n_pad, dtype=torch.int16, device="cuda")
+    Z = torch.empty(l, m + proto.sum_r, dtype=torch.int32, device="cuda")
+    layer.mask_input(X, mp, Xp, s_x, Xpl)
+    torch.cuda.synchronize()
+    M.mosaic_kernel_times(reset=True)
+    M.mosaic_kernel_timing(True)
+    try:
+        n0 = M.mosaic_kernel_launches()
+        Y1 = layer.forward(X, layer.init_x(l, 77))
+        torch.cuda.synchronize()
+        launched = M.mosaic_kernel_launches() - n0
+        kt = M.mosaic_kernel_times(reset=True)
+        side = torch.cuda.Stream()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            layer.server(Xp, Xpl, Z)
+        torch.cuda.synchronize()
+        captured = M.mosaic_kernel_times(reset=True)
+    finally:
+        M.mosaic_kernel_timing(False)
+    assert torch.equal(Y0, Y1)
+    assert sum(v[0] for v in kt.values()) == launched
+    for key in ("init_x:initx_draw", "init_x:ring_gemm_tc", "unmask:ring_gemm_tc"):
+        assert key in kt and kt[key][0] >= 1 and kt[key][1] > 0.0, (key, kt)
+    for role in ("init_x:", "unmask:"):
+        assert any(k.startswith(role) and "gather" in k for k in kt), kt
+    assert any(k.startswith("encode:") for k in kt) and any(k.startswith("ring_gemm:") for k in kt), kt
+    assert captured == {}
+    g.replay()
+    torch.cuda.synchronize()
+    del g
