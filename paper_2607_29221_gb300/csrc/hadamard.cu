@@ -370,9 +370,9 @@ mosaic_status launch(const FwhtArgs &a, cudaStream_t st) {
 }
 
 // ---------------------------------------------------------------------------
-// Rows of 16384 and 32768 whose length n is a multiple of 32: a persistent
-// grid (one block per SM) that fetches each block's NEXT input row by TMA
-// while the current row is transformed and stored.  In the kernel above an SM
+// Rows of 32768 whose length n is a multiple of 32: a persistent grid (one
+// block per SM) that fetches each block's NEXT input row by TMA while the
+// current row is transformed and stored.  In the kernel above an SM
 // holds a single row at a time (32 values per thread in registers, a 512- or
 // 1024-thread block), so its loads, butterflies and stores never overlap.
 // The row arrives as a 3-D tensor {32 values, chunks, rows} with the 128-byte
@@ -380,11 +380,9 @@ mosaic_status launch(const FwhtArgs &a, cudaStream_t st) {
 // [128 c, 128 c + 128) with its 16-byte pieces XOR-permuted by c & 7, so each
 // thread reads its own run with 8 conflict-free 16-byte loads.  The
 // arithmetic (stage order, roundings) is that of fwht_kernel, line for line,
-// so the results are identical.  Rows of 16384 also prefetch the mask row of
-// the encode the same way (its own buffer; the transpose has a third one);
-// rows of 32768 run the transpose in the input buffer and read the mask from
-// global memory.  Every wait is bounded; on expiry the block raises
-// g_fwht_error and stops.
+// so the results are identical.  The transpose runs in the input buffer
+// (132 KB) and the encode reads the mask from global memory.  Every wait is
+// bounded; on expiry the block raises g_fwht_error and stops.
 // ---------------------------------------------------------------------------
 template <int T>
 struct StreamCfg {
@@ -393,38 +391,29 @@ struct StreamCfg {
     static constexpr int WN = T / 32;
     static constexpr int CS = E / WN;
     static constexpr int RUNS = E / CS;
-    static constexpr bool OWN_T = N <= 16384;                        // separate transpose buffer
-    static constexpr size_t XBUF = OWN_T ? (size_t)N * 4 : (size_t)(N + N / 32) * 4;
-    static constexpr size_t MBUF = OWN_T ? (size_t)N * 4 : 0;       // mask row (encode)
-    static constexpr size_t TBUF = OWN_T ? (size_t)(N + N / 32) * 4 : 0;
-    static constexpr size_t SMEM = 1024 + XBUF + MBUF + TBUF + 64;
+    static constexpr size_t XBUF = (size_t)(N + N / 32) * 4;        // input row, then its transpose
+    static constexpr size_t SMEM = 1024 + XBUF + 64;
     static constexpr int BOX_CHUNKS = 256;                           // 32 KB per copy
     static constexpr int COPIES = N / 32 / BOX_CHUNKS;
 };
 
 template <int T>
-__global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant__ CUtensorMap tmx,
-                                                           const __grid_constant__ CUtensorMap tmm, FwhtArgs a,
-                                                           int has_mask_map) {
+__global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant__ CUtensorMap tmx, FwhtArgs a) {
     using C = StreamCfg<T>;
     constexpr int E = C::E, N = C::N, WN = C::WN, CS = C::CS, RUNS = C::RUNS;
     extern __shared__ uint8_t raw[];
     uint8_t *base_ptr = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~(uintptr_t)1023);
     float *xbuf = reinterpret_cast<float *>(base_ptr);
-    uint32_t *mbuf = reinterpret_cast<uint32_t *>(base_ptr + C::XBUF);
-    float *tbuf = C::OWN_T ? reinterpret_cast<float *>(base_ptr + C::XBUF + C::MBUF) : xbuf;
-    uint64_t *bar_x = reinterpret_cast<uint64_t *>(base_ptr + C::XBUF + C::MBUF + C::TBUF);
-    uint64_t *bar_m = bar_x + 1;
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_m + 1);
+    float *tbuf = xbuf;
+    uint64_t *bar_x = reinterpret_cast<uint64_t *>(base_ptr + C::XBUF);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_x + 1);
     __shared__ float red_max[WN];
     __shared__ int red_ok[WN];
 
     const int lt = threadIdx.x, lane = lt & 31;
     const int base = lt * E;
-    const bool use_mmap = C::OWN_T && a.mode == 1 && a.mask && has_mask_map;
     if (lt == 0) {
         mbar_init(bar_x, 1);
-        mbar_init(bar_m, 1);
         *abort_flag = 0;
         mbar_init_fence();
     }
@@ -437,18 +426,8 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
             tma_load_3d(reinterpret_cast<uint8_t *>(xbuf) + (size_t)c * C::BOX_CHUNKS * 128, &tmx, bar_x, 0,
                         c * C::BOX_CHUNKS, (int)row);
     };
-    auto issue_m = [&](int64_t row) {
-        mbar_expect_tx(bar_m, (uint32_t)(N * 4));
-#pragma unroll
-        for (int c = 0; c < C::COPIES; ++c)
-            tma_load_3d(reinterpret_cast<uint8_t *>(mbuf) + (size_t)c * C::BOX_CHUNKS * 128, &tmm, bar_m, 0,
-                        c * C::BOX_CHUNKS, (int)row);
-    };
     int64_t row = blockIdx.x;
-    if (lt == 0 && row < a.rows) {
-        issue_x(row);
-        if (use_mmap) issue_m(row);
-    }
+    if (lt == 0 && row < a.rows) issue_x(row);
     uint32_t ph = 0;
     for (; row < a.rows; row += gridDim.x, ph ^= 1u) {
         const int64_t next = row + gridDim.x;
@@ -469,14 +448,6 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
                              : "=f"(v[4 * q]), "=f"(v[4 * q + 1]), "=f"(v[4 * q + 2]), "=f"(v[4 * q + 3])
                              : "r"(addr)
                              : "memory");
-            }
-        }
-        if constexpr (C::OWN_T) {
-            // The input buffer is free: fetch the next row while this one runs.
-            __syncthreads();
-            if (lt == 0 && next < a.rows && !*abort_flag) {
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                issue_x(next);
             }
         }
         if (a.rotate) {
@@ -508,7 +479,7 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
                 }
             }
         }
-        if constexpr (!C::OWN_T) __syncthreads();   // every thread has read the input buffer
+        __syncthreads();   // every thread has read the input buffer
 #pragma unroll
         for (int e = 0; e < E; e++) tbuf[pad_idx(base + e)] = v[e];
         __syncthreads();
@@ -516,13 +487,11 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
         for (int j = 0; j < WN; j++)
 #pragma unroll
             for (int u = 0; u < CS; u++) v[j * CS + u] = tbuf[pad_idx(j * 32 * E + lt * CS + u)];
-        if constexpr (!C::OWN_T) {
-            // The transpose was done in the input buffer: fetch the next row now.
-            __syncthreads();
-            if (lt == 0 && next < a.rows && !*abort_flag) {
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                issue_x(next);
-            }
+        // The transpose was done in the input buffer: fetch the next row now.
+        __syncthreads();
+        if (lt == 0 && next < a.rows && !*abort_flag) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            issue_x(next);
         }
         if (a.rotate) {
 #pragma unroll
@@ -584,36 +553,13 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
             code[e] = quant ? (uint32_t)c : 0u;
         }
         if (a.mask) {
-            if (use_mmap) {
-                if (!mbar_wait(bar_m, ph, abort_flag)) {
-                    *abort_flag = 1;
-                    atomicExch(&g_fwht_error, 1u);
-                }
-                // Mask word k of the row: chunk k / 32, 16-byte piece ((k / 4) % 8) ^ (chunk % 8), word k % 4.
+            const uint32_t *mr = a.mask + row * a.ldm;
 #pragma unroll
-                for (int run = 0; run < RUNS; run++) {
+            for (int run = 0; run < RUNS; run++) {
+                uint32_t mk[CS];
+                load_u32<CS>(mr + elem(run), mk);
 #pragma unroll
-                    for (int u = 0; u < CS; u++) {
-                        const int k = elem(run) + u, ch = k >> 5;
-                        code[run * CS + u] += *reinterpret_cast<const uint32_t *>(
-                            reinterpret_cast<const uint8_t *>(mbuf) + (size_t)ch * 128 +
-                            ((((k >> 2) & 7) ^ (ch & 7)) * 16) + (k & 3) * 4);
-                    }
-                }
-                __syncthreads();   // every thread has read the mask buffer
-                if (lt == 0 && next < a.rows && !*abort_flag) {
-                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                    issue_m(next);
-                }
-            } else {
-                const uint32_t *mr = a.mask + row * a.ldm;
-#pragma unroll
-                for (int run = 0; run < RUNS; run++) {
-                    uint32_t mk[CS];
-                    load_u32<CS>(mr + elem(run), mk);
-#pragma unroll
-                    for (int u = 0; u < CS; u++) code[run * CS + u] += mk[u];
-                }
+                for (int u = 0; u < CS; u++) code[run * CS + u] += mk[u];
             }
         }
         uint32_t *orow = a.out + row * a.ldo;
@@ -628,10 +574,7 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
     }
     // After a normal exit every issued copy has been waited for; after an
     // expired wait, let the copies still in flight land (bounded) first.
-    if (lt == 0 && *abort_flag) {
-        mbar_drain(bar_x, ph);
-        if (use_mmap) mbar_drain(bar_m, ph);
-    }
+    if (lt == 0 && *abort_flag) mbar_drain(bar_x, ph);
     __syncthreads();
 }
 
@@ -653,15 +596,8 @@ bool make_chunk_map(CUtensorMap *map, const void *base, int64_t len, int64_t row
 template <int T>
 mosaic_status launch_stream(const FwhtArgs &a, cudaStream_t st) {
     using C = StreamCfg<T>;
-    CUtensorMap tmx, tmm;
+    CUtensorMap tmx;
     if (!make_chunk_map(&tmx, a.x, a.n, a.rows, a.ldx, true)) return MOSAIC_ERR_CUDA;
-    int has_m = 0;
-    if (C::OWN_T && a.mode == 1 && a.mask) {
-        if (!make_chunk_map(&tmm, a.mask, a.n_pad, a.rows, a.ldm, false)) return MOSAIC_ERR_CUDA;
-        has_m = 1;
-    } else {
-        tmm = tmx;
-    }
     static std::atomic<unsigned long long> attr_set{0};
     int dev = 0, sms = 0;
     if (!ensure_smem_limit(attr_set, fwht_stream_kernel<T>, C::SMEM, &dev) ||
@@ -670,12 +606,12 @@ mosaic_status launch_stream(const FwhtArgs &a, cudaStream_t st) {
     const int64_t grid = a.rows < sms ? a.rows : sms;
     {
         KernelSpan span("fwht_stream", st);
-        fwht_stream_kernel<T><<<(unsigned)grid, T, C::SMEM, st>>>(tmx, tmm, a, has_m);
+        fwht_stream_kernel<T><<<(unsigned)grid, T, C::SMEM, st>>>(tmx, a);
     }
     return launch_status();
 }
 
-// The streamed kernel takes rows whose length is a multiple of 32 words with
+// The streamed kernels take rows whose length is a multiple of 32 words with
 // 16-byte aligned rows (x, and the mask when there is one); rows of 2^31 or
 // more are left to the per-row kernel (32-bit row coordinates).
 bool stream_ok(const FwhtArgs &a) {
@@ -683,6 +619,228 @@ bool stream_ok(const FwhtArgs &a) {
     if (a.n % 32 != 0 || !aligned16(a.x) || a.ldx % 4 != 0) return false;
     if (a.mode == 1 && a.mask && (!aligned16(a.mask) || a.ldm % 4 != 0)) return false;
     return encode_fn() != nullptr;
+}
+
+// ---------------------------------------------------------------------------
+// Rows of 16384 (length n a multiple of 32), two rows in flight per SM.  Each
+// CTA (512 threads, 32 values a thread, at most 64 registers so that two CTAs
+// share an SM) transforms one row at a time with the stage order and roundings
+// of fwht_kernel, so the results are identical.  The row arrives by TMA in the
+// CTA's input buffer (the 3-D {32 values, chunks, rows} view with the 128-byte
+// swizzle: chunk c, thread c's 32 consecutive values, lies at bytes
+// [128 c, 128 c + 128) with its 16-byte pieces XOR-permuted by c & 7, so each
+// thread reads its run with 8 conflict-free 16-byte loads); the transpose
+// reuses the buffer, and the next row's copy is issued as soon as the
+// transpose has been read back.  One CTA cannot overlap its own butterflies
+// with its stores, but the other CTA on the SM can.  The TMA wait is bounded
+// (abort flag + g_fwht_error).
+// ---------------------------------------------------------------------------
+constexpr int kPairT = 512;                     // threads per CTA
+constexpr int kPairE = 32;                      // values per thread
+constexpr int kPairN = kPairT * kPairE;         // values per CTA: 16384
+constexpr int kPairWN = kPairT / 32;            // warps: 16
+constexpr int kPairCS = kPairE / kPairWN;       // run length after the transpose: 2
+constexpr int kPairRuns = kPairE / kPairCS;     // runs: 16
+constexpr size_t kPairXBUF = (size_t)(kPairN + kPairN / 32) * 4;   // padded transpose fits
+constexpr size_t kPairSMEM = 1024 + kPairXBUF + 64;
+constexpr int kPairBox = 256;                   // chunks of 32 values per TMA box (32 KB)
+
+__global__ void __launch_bounds__(kPairT, 2) fwht_pair_kernel(const __grid_constant__ CUtensorMap tmx, FwhtArgs a) {
+    constexpr int E = kPairE, N = kPairN, WN = kPairWN, CS = kPairCS, RUNS = kPairRuns;
+    extern __shared__ uint8_t raw[];
+    uint8_t *base_ptr = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~(uintptr_t)1023);
+    float *xbuf = reinterpret_cast<float *>(base_ptr);
+    uint64_t *bar_x = reinterpret_cast<uint64_t *>(base_ptr + kPairXBUF);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_x + 1);
+    __shared__ float red_max[WN];
+    __shared__ int red_ok[WN];
+
+    const int lt = threadIdx.x, lane = lt & 31;
+    const int base = lt * E;
+    if (lt == 0) {
+        mbar_init(bar_x, 1);
+        *abort_flag = 0;
+        mbar_init_fence();
+    }
+    __syncthreads();
+    auto issue_x = [&](int64_t row) {
+        mbar_expect_tx(bar_x, (uint32_t)(N * 4));
+#pragma unroll
+        for (int c = 0; c < N / 32 / kPairBox; ++c)
+            tma_load_3d(reinterpret_cast<uint8_t *>(xbuf) + (size_t)c * kPairBox * 128, &tmx, bar_x, 0,
+                        c * kPairBox, (int)row);
+    };
+    int64_t row = blockIdx.x;
+    if (lt == 0 && row < a.rows) issue_x(row);
+    uint32_t ph = 0;
+    for (; row < a.rows; row += gridDim.x, ph ^= 1u) {
+        const int64_t next = row + gridDim.x;
+        if (!mbar_wait(bar_x, ph, abort_flag)) {
+            *abort_flag = 1;
+            atomicExch(&g_fwht_error, 1u);
+        }
+        __syncthreads();
+        if (*abort_flag) break;
+        float v[E];
+        {
+            const uint32_t rb = smem_u32(xbuf) + (uint32_t)lt * 128u;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const uint32_t addr = rb + (uint32_t)((q ^ (lt & 7)) * 16);
+                asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                             : "=f"(v[4 * q]), "=f"(v[4 * q + 1]), "=f"(v[4 * q + 2]), "=f"(v[4 * q + 3])
+                             : "r"(addr)
+                             : "memory");
+            }
+        }
+        if (a.rotate) {
+            if (a.signs) {
+                const uint32_t w = a.signs[base >> 5] >> (base & 31);
+#pragma unroll
+                for (int e = 0; e < E; e++)
+                    if ((w >> e) & 1u) v[e] = -v[e];
+            }
+#pragma unroll
+            for (int h = 1; h < E; h <<= 1) {
+#pragma unroll
+                for (int i = 0; i < E; i += 2 * h) {
+#pragma unroll
+                    for (int j = i; j < i + h; j++) {
+                        const float p = v[j], q = v[j + h];
+                        v[j] = __fadd_rn(p, q);
+                        v[j + h] = __fsub_rn(p, q);
+                    }
+                }
+            }
+#pragma unroll
+            for (int hl = 1; hl < 32; hl <<= 1) {
+                const float sgn = (lane & hl) ? -1.0f : 1.0f;
+#pragma unroll
+                for (int e = 0; e < E; e++) {
+                    const float o = __shfl_xor_sync(0xffffffffu, v[e], hl);
+                    v[e] = __fmaf_rn(v[e], sgn, o);
+                }
+            }
+        }
+        __syncthreads();   // every thread has read the input buffer
+#pragma unroll
+        for (int e = 0; e < E; e++) xbuf[pad_idx(base + e)] = v[e];
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < WN; j++)
+#pragma unroll
+            for (int u = 0; u < CS; u++) v[j * CS + u] = xbuf[pad_idx(j * 32 * E + lt * CS + u)];
+        __syncthreads();   // every thread has read the transpose
+        if (lt == 0 && next < a.rows) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            issue_x(next);
+        }
+        if (a.rotate) {
+#pragma unroll
+            for (int hj = 1; hj < WN; hj <<= 1) {
+#pragma unroll
+                for (int i = 0; i < WN; i += 2 * hj) {
+#pragma unroll
+                    for (int j = i; j < i + hj; j++) {
+#pragma unroll
+                        for (int u = 0; u < CS; u++) {
+                            const float p = v[j * CS + u], q = v[(j + hj) * CS + u];
+                            v[j * CS + u] = __fadd_rn(p, q);
+                            v[(j + hj) * CS + u] = __fsub_rn(p, q);
+                        }
+                    }
+                }
+            }
+        }
+        auto elem = [&](int run) -> int { return run * 32 * E + lt * CS; };
+        if (a.rotate) {
+#pragma unroll
+            for (int e = 0; e < E; e++) v[e] = __fmul_rn(v[e], a.inv_sqrt);
+        }
+        if (a.mode == 0) {
+            float *yr = a.y + row * a.ldy;
+#pragma unroll
+            for (int run = 0; run < RUNS; run++) store_f32<CS>(yr + elem(run), v + run * CS);
+            continue;
+        }
+        float mx = 0.0f;
+        int ok = 1;
+#pragma unroll
+        for (int e = 0; e < E; e++) {
+            ok &= isfinite(v[e]) ? 1 : 0;
+            mx = fmaxf(mx, fabsf(v[e]));
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            ok &= __shfl_xor_sync(0xffffffffu, ok, o);
+        }
+        if (lane == 0) {
+            red_max[lt >> 5] = mx;
+            red_ok[lt >> 5] = ok;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int w = 0; w < WN; w++) {
+            mx = fmaxf(mx, red_max[w]);
+            ok &= red_ok[w];
+        }
+        const float s = ok ? __fdiv_rn(mx, (float)a.qmax) : __int_as_float(0x7fc00000);
+        if (lt == 0) a.scale[row] = s;
+        const bool quant = ok && s != 0.0f;
+        uint32_t code[E];
+#pragma unroll
+        for (int e = 0; e < E; e++) {
+            const float t = __fadd_rn(__fdiv_rn(v[e], s), 12582912.0f);
+            int32_t c = __float_as_int(t) - 0x4B400000;
+            c = min(max(c, -a.qmax), a.qmax);
+            code[e] = quant ? (uint32_t)c : 0u;
+        }
+        if (a.mask) {
+            const uint32_t *mr = a.mask + row * a.ldm;
+#pragma unroll
+            for (int run = 0; run < RUNS; run++) {
+                uint32_t mk[CS];
+                load_u32<CS>(mr + elem(run), mk);
+#pragma unroll
+                for (int u = 0; u < CS; u++) code[run * CS + u] += mk[u];
+            }
+        }
+        uint32_t *orow = a.out + row * a.ldo;
+#pragma unroll
+        for (int run = 0; run < RUNS; run++) store_u32<CS>(orow + elem(run), code + run * CS);
+        if (a.planes) {
+            const int64_t ps = a.rows * a.n_pad;
+            uint16_t *prow = a.planes + row * a.n_pad;
+#pragma unroll
+            for (int run = 0; run < RUNS; run++) store_planes<CS>(prow + elem(run), ps, code + run * CS);
+        }
+    }
+    // After a normal exit every issued copy has been waited for; after an
+    // expired wait, let the copy still in flight land (bounded) first.
+    if (lt == 0 && *abort_flag) mbar_drain(bar_x, ph);
+    __syncthreads();
+}
+
+mosaic_status launch_pair(const FwhtArgs &a, cudaStream_t st) {
+    CUtensorMap tmx;
+    if (!make_chunk_map(&tmx, a.x, a.n, a.rows, a.ldx, true)) return MOSAIC_ERR_CUDA;
+    static std::atomic<unsigned long long> attr_set{0};
+    int dev = 0, sms = 0, per_sm = 0;
+    if (!ensure_smem_limit(attr_set, fwht_pair_kernel, kPairSMEM, &dev) ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1 ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fwht_pair_kernel, kPairT, kPairSMEM) != cudaSuccess ||
+        per_sm < 1)
+        return MOSAIC_ERR_CUDA;
+    // As many rows in flight as the GPU holds at once (two CTAs per SM), each
+    // CTA walking rows with a stride of the grid.
+    const int64_t slots = (int64_t)sms * per_sm;
+    const int64_t grid = a.rows < slots ? a.rows : slots;
+    {
+        KernelSpan span("fwht_pair", st);
+        fwht_pair_kernel<<<(unsigned)grid, kPairT, kPairSMEM, st>>>(tmx, a);
+    }
+    return launch_status();
 }
 
 // ---------------------------------------------------------------------------
@@ -832,7 +990,7 @@ mosaic_status fwht_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, 
         case 2048: return launch<16, 128>(a, st);
         case 4096: return launch<16, 256>(a, st);
         case 8192: return launch<32, 256>(a, st);
-        case 16384: return stream_ok(a) ? launch_stream<512>(a, st) : launch<32, 512>(a, st);
+        case 16384: return stream_ok(a) ? launch_pair(a, st) : launch<32, 512>(a, st);
         case 32768: return stream_ok(a) ? launch_stream<1024>(a, st) : launch<32, 1024>(a, st);
         default: return MOSAIC_ERR_SHAPE;
     }
