@@ -748,6 +748,17 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
         torch.cuda.synchronize()
         server_ms = float(np.mean([a.elapsed_time(b) for a, b in srv]))
         del gsrv
+        # Per-kernel device time of a few eager online steps (the library's own
+        # event pair around each launch): the server kernel's time alone.
+        kt_steps = 3
+        M.mosaic_kernel_times(reset=True)
+        M.mosaic_kernel_timing(True)
+        for i in range(kt_steps):
+            flush.fill_(i & 0xFF)
+            runner.step(None, i)
+        torch.cuda.synchronize()
+        M.mosaic_kernel_timing(False)
+        kt = M.mosaic_kernel_times(reset=True)
         step_ms = online_ms + initx_ms
         del masks
         w_bytes = sum((ly.m + proto.sum_r) * ly.n_pad * 4 for ly in layers)
@@ -767,7 +778,13 @@ def run_decode_sweep(args, rank, world, torch, M, PR, proto, dev, stream, timed,
                                        ("ring_gemm_imad" if variant == M.GEMM_IMAD else "ring_gemm_tc"),
                       "w_prime_bytes": w_bytes, "server_read_bytes": read_bytes,
                       "server_read_gbs": round(read_bytes / (server_ms / 1e3) / 1e9, 1),
-                      "server_hbm_frac": round(read_bytes / (server_ms / 1e3) / 1e9 / hbm, 4)})
+                      "server_hbm_frac": round(read_bytes / (server_ms / 1e3) / 1e9 / hbm, 4),
+                      "kernel_ms_per_step": {k: round(v[1] / kt_steps, 4) for k, v in sorted(kt.items())}})
+        skey = "ring_gemm:" + sweep[-1]["server_kernel"]
+        if skey in kt and kt[skey][1] > 0:
+            kms = kt[skey][1] / kt_steps
+            sweep[-1]["server_kernel_ms"] = round(kms, 4)
+            sweep[-1]["server_kernel_hbm_frac"] = round(read_bytes / (kms / 1e3) / 1e9 / hbm, 4)
     clocks = sampler.stop()
     M.mosaic_device_status()
     if rank != 0:

@@ -439,22 +439,43 @@ __global__ void __launch_bounds__(THREADS, 1)
 
 // Digit planes of the token operand as fp16 bits, planes[d][r][c] =
 // byte_d(a + 0x80808080) - 128, and C (rows x n, leading dimension ldc)
-// zeroed for the red.add reduction, in one launch.
-__global__ void split_f16_zero_kernel(const uint32_t *a, int64_t lda, int64_t rows, int64_t cols, uint16_t *planes,
-                                      int64_t ldp, int64_t plane_stride, uint32_t *C, int64_t ldc, int64_t n) {
-    const int64_t total = rows * cols, ctotal = rows * n;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += stride) {
-        const int64_t r = i / cols, c = i - r * cols;
-        const uint32_t b = a[r * lda + c] + 0x80808080u;
+// zeroed for the red.add reduction, in one launch: block (x, r) covers
+// columns [1024 x, 1024 x + 1024) of row r, four consecutive columns a
+// thread (16-byte loads and stores where the row allows).
+__device__ __forceinline__ uint16_t digit_f16(uint32_t b, int d) {
+    return __half_as_ushort(__int2half_rn((int)((b >> (8 * d)) & 0xffu) - 128));
+}
+__global__ void split_f16_zero_kernel(const uint32_t *a, int64_t lda, int64_t cols, uint16_t *planes, int64_t ldp,
+                                      int64_t plane_stride, uint32_t *C, int64_t ldc, int64_t n, int vec_a,
+                                      int vec_c) {
+    const int64_t r = blockIdx.y;
+    const int64_t c = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+    if (c < cols) {
+        const uint32_t *ar = a + r * lda + c;
+        uint16_t *pr = planes + r * ldp + c;
+        if (vec_a && c + 4 <= cols) {
+            const uint4 v = *reinterpret_cast<const uint4 *>(ar);
+            const uint32_t b[4] = {v.x + 0x80808080u, v.y + 0x80808080u, v.z + 0x80808080u, v.w + 0x80808080u};
 #pragma unroll
-        for (int d = 0; d < 4; ++d)
-            planes[d * plane_stride + r * ldp + c] =
-                __half_as_ushort(__int2half_rn((int)((b >> (8 * d)) & 0xffu) - 128));
+            for (int d = 0; d < 4; ++d)
+                *reinterpret_cast<uint2 *>(pr + d * plane_stride) =
+                    make_uint2((uint32_t)digit_f16(b[0], d) | ((uint32_t)digit_f16(b[1], d) << 16),
+                               (uint32_t)digit_f16(b[2], d) | ((uint32_t)digit_f16(b[3], d) << 16));
+        } else {
+            for (int k = 0; k < 4 && c + k < cols; ++k) {
+                const uint32_t b = ar[k] + 0x80808080u;
+#pragma unroll
+                for (int d = 0; d < 4; ++d) pr[d * plane_stride + k] = digit_f16(b, d);
+            }
+        }
     }
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < ctotal; i += stride) {
-        const int64_t r = i / n, c = i - r * n;
-        C[r * ldc + c] = 0u;
+    if (c < n) {
+        uint32_t *cr = C + r * ldc + c;
+        if (vec_c && c + 4 <= n) {
+            *reinterpret_cast<uint4 *>(cr) = make_uint4(0u, 0u, 0u, 0u);
+        } else {
+            for (int k = 0; k < 4 && c + k < n; ++k) cr[k] = 0u;
+        }
     }
 }
 
@@ -524,8 +545,12 @@ mosaic_status ring_gemm_tcw(const uint32_t *A, int64_t lda, const uint32_t *B, i
     const int64_t Kp = (K + 7) / 8 * 8;
     {
         KernelSpan span("split_f16_zero", st);
-        split_f16_zero_kernel<<<grid_for(M * (K > N ? K : N), 256), 256, 0, st>>>(A, lda, M, K, Ap, Kp, M * Kp, Cm, ldc,
-                                                                                   N);
+        // Planes rows are Kp (a multiple of 8) fp16 apart, so their 8-byte stores are aligned.
+        const int vec_a = aligned16(A) && lda % 4 == 0;
+        const int vec_c = aligned16(Cm) && ldc % 4 == 0;
+        const int64_t wide = K > N ? K : N;
+        split_f16_zero_kernel<<<dim3((unsigned)((wide + 1023) / 1024), (unsigned)M), 256, 0, st>>>(
+            A, lda, K, Ap, Kp, M * Kp, Cm, ldc, N, vec_a, vec_c);
     }
     MOSAIC_TRY(launch_status());
     const int nt = M <= 32 ? 32 : M <= 48 ? 48 : 64;
