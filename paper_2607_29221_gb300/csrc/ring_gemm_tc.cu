@@ -47,6 +47,12 @@ constexpr int CHUNK = 8;        // stages between drains: 256 K
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int THREADS = 320;   // warp 0 TMA, warp 1 MMA, warps 2..9 epilogue
 constexpr int EPI_WARPS = 8;
+// Write-out slices: each epilogue warp moves its 32 rows 16 columns at a time
+// through a [32][EPI_PITCH] block of shared memory (pitch 20 words: the
+// row-per-lane 16-byte writes and the 8-rows-per-access 16-byte reads are
+// both conflict-free).
+constexpr int EPI_PITCH = 20;
+constexpr int EPI_BYTES = EPI_WARPS * 32 * EPI_PITCH * 4;
 
 // Drain conversions.  The fp32 group sums are integers with |x| <= 2^24 and
 // the F2I unit converts 16 values per clock per SM while the tensor pipe
@@ -91,7 +97,7 @@ struct Cfg {
     static constexpr int A_BYTES = 4 * A_PLANE;
     static constexpr int B_BYTES = 4 * B_PLANE;
     static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+    static constexpr int SMEM = STAGES * STAGE + 1024 + 256 + EPI_BYTES;
     // kind::f16 instruction descriptors: D f32, A/B bf16, K-major, N >> 3, M >> 4;
     // IDESC2 has N = 2 BN (two consecutive B digit planes as one operand).
     static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
@@ -189,6 +195,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint64_t *drain = acc_empty + 1;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+    const uint32_t epi_base = smem_u32(smem + STAGES * C::STAGE + 256);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nk = (a.K + BK - 1) / BK;
@@ -429,49 +436,73 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int n0 = tn0 - (second ? a.N1 : 0) + h * HB;
             const int nout = second ? a.N - a.N1 : a.N1;
             const int gm = m0 + row;
-            if (gm < a.M) {
-                uint32_t *crow = second ? a.C2 + (int64_t)gm * a.ldc2 : a.C + (int64_t)gm * a.ldc;
-                const uint32_t *cin0 = second ? a.Cin2 : a.Cin;
-                const uint32_t *cin = cin0 ? cin0 + (int64_t)gm * (second ? a.ldcin2 : a.ldcin) : nullptr;
-                const int64_t ldc_o = second ? a.ldc2 : a.ldc;
-                const int64_t ldcin_o = second ? a.ldcin2 : a.ldcin;
-                const uint32_t *sub = (!second && a.Csub) ? a.Csub + (int64_t)gm * a.ldcsub : nullptr;
-                if (a.sgn < 0) {
+            uint32_t *const cbase = second ? a.C2 : a.C;
+            const int64_t ldc_o = second ? a.ldc2 : a.ldc;
+            const uint32_t *const cin0 = second ? a.Cin2 : a.Cin;
+            const int64_t ldcin_o = second ? a.ldcin2 : a.ldcin;
+            const uint32_t *const sub0 = second ? nullptr : a.Csub;
+            if (a.sgn < 0) {
 #pragma unroll
-                    for (int cc = 0; cc < HB; ++cc) acc[cc] = 0u - acc[cc];
+                for (int cc = 0; cc < HB; ++cc) acc[cc] = 0u - acc[cc];
+            }
+            // Other CTAs add into a split tile too: exact and order-free in Z_{2^32}.
+            const bool atomic = a.split && !whole;
+            // Plain mode: C = Cin - Csub + acc.  Stream-K mode, whole tile: C (prepared) += acc.
+            const bool vecw = !atomic && (n0 + HB <= nout) && ((ldc_o & 3) == 0) &&
+                              ((reinterpret_cast<uintptr_t>(cbase) & 15u) == 0) &&
+                              (a.split || !cin0 || (((ldcin_o & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin0) & 15u) == 0))) &&
+                              (!sub0 || (((a.ldcsub & 3) == 0) && ((reinterpret_cast<uintptr_t>(sub0) & 15u) == 0)));
+            if (vecw) {
+                // Coalesced write-out: 16 columns of the warp's 32 rows go to its
+                // slice block (one row per lane) and come back as 8 rows x 64
+                // bytes per access, so C, Cin and Csub move in half lines
+                // instead of 16 bytes of 32 rows per access.
+                const uint32_t wb = epi_base + (uint32_t)((warp - 2) * 32 * EPI_PITCH * 4);
+                const int pc = (lane >> 3) * 4;
+#pragma unroll
+                for (int s0 = 0; s0 < HB; s0 += 16) {
+#pragma unroll
+                    for (int cc = 0; cc < 16; cc += 4)
+                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                         wb + 4u * (uint32_t)(lane * EPI_PITCH + cc)),
+                                     "r"(acc[s0 + cc]), "r"(acc[s0 + cc + 1]), "r"(acc[s0 + cc + 2]), "r"(acc[s0 + cc + 3])
+                                     : "memory");
+                    __syncwarp();
+                    uint4 v[4], ib[4], sb[4];
+#pragma unroll
+                    for (int it = 0; it < 4; ++it) {
+                        const int rl = it * 8 + (lane & 7);
+                        const int gr = m0 + q * 32 + rl;
+                        const int64_t col = n0 + s0 + pc;
+                        asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                                     : "=r"(v[it].x), "=r"(v[it].y), "=r"(v[it].z), "=r"(v[it].w)
+                                     : "r"(wb + 4u * (uint32_t)(rl * EPI_PITCH + pc))
+                                     : "memory");
+                        const uint32_t *bp = a.split ? cbase + (int64_t)gr * ldc_o + col
+                                                     : (cin0 ? cin0 + (int64_t)gr * ldcin_o + col : nullptr);
+                        const uint32_t *sp = sub0 ? sub0 + (int64_t)gr * a.ldcsub + col : nullptr;
+                        ib[it] = (gr < a.M && bp) ? *reinterpret_cast<const uint4 *>(bp) : make_uint4(0, 0, 0, 0);
+                        sb[it] = (gr < a.M && sp) ? *reinterpret_cast<const uint4 *>(sp) : make_uint4(0, 0, 0, 0);
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int it = 0; it < 4; ++it) {
+                        const int rl = it * 8 + (lane & 7);
+                        const int gr = m0 + q * 32 + rl;
+                        if (gr < a.M)
+                            *reinterpret_cast<uint4 *>(cbase + (int64_t)gr * ldc_o + n0 + s0 + pc) =
+                                make_uint4(v[it].x + ib[it].x - sb[it].x, v[it].y + ib[it].y - sb[it].y,
+                                           v[it].z + ib[it].z - sb[it].z, v[it].w + ib[it].w - sb[it].w);
+                    }
                 }
-                const bool vec = (n0 + HB <= nout) && ((ldc_o & 3) == 0) &&
-                                 ((reinterpret_cast<uintptr_t>(crow) & 15u) == 0) &&
-                                 (!cin || (((ldcin_o & 3) == 0) && ((reinterpret_cast<uintptr_t>(cin) & 15u) == 0))) &&
-                                 (!sub || (((a.ldcsub & 3) == 0) && ((reinterpret_cast<uintptr_t>(sub) & 15u) == 0)));
-                if (a.split && !whole) {
-                    // Other CTAs add into this tile too: exact and order-free in Z_{2^32}.
+            } else if (gm < a.M) {
+                uint32_t *crow = cbase + (int64_t)gm * ldc_o;
+                const uint32_t *cin = cin0 ? cin0 + (int64_t)gm * ldcin_o : nullptr;
+                const uint32_t *sub = sub0 ? sub0 + (int64_t)gm * a.ldcsub : nullptr;
+                if (atomic) {
 #pragma unroll
                     for (int cc = 0; cc < HB; ++cc)
                         if (n0 + cc < nout) atomicAdd(crow + n0 + cc, acc[cc]);
-                } else if (vec) {
-                    // Plain mode: C = Cin + acc.  Stream-K mode: C (prepared) += acc.
-                    // C may be Cin (in place), so the compiler keeps every load
-                    // behind the stores before it: the loads of 16 columns are
-                    // issued together, then their stores, so that a thread waits
-                    // for four round trips per tile instead of one per 4 columns.
-                    const uint32_t *base = a.split ? crow : cin;
-#pragma unroll
-                    for (int cb = 0; cb < HB; cb += 16) {
-                        uint4 ib[4], sb[4];
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            ib[q] = base ? *reinterpret_cast<const uint4 *>(base + n0 + cb + 4 * q) : make_uint4(0, 0, 0, 0);
-                            sb[q] = sub ? *reinterpret_cast<const uint4 *>(sub + n0 + cb + 4 * q) : make_uint4(0, 0, 0, 0);
-                        }
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const int cc = cb + 4 * q;
-                            const uint4 o = make_uint4(acc[cc] + ib[q].x - sb[q].x, acc[cc + 1] + ib[q].y - sb[q].y,
-                                                       acc[cc + 2] + ib[q].z - sb[q].z, acc[cc + 3] + ib[q].w - sb[q].w);
-                            *reinterpret_cast<uint4 *>(crow + n0 + cc) = o;
-                        }
-                    }
                 } else {
                     const uint32_t *base = a.split ? crow : cin;
 #pragma unroll
