@@ -496,6 +496,24 @@ mosaic_status mosaic_unmask_noalloc(const mosaic_params *p, int64_t l, int64_t m
                                     int variant, void *stream);
 
 /* ------------------------------------------------------------------------ */
+/* Float glue of a decoder layer (Sec. 4.1: the non-linear parts run on the   */
+/* trusted side in plain arithmetic).  Model operations between the secure    */
+/* linear calls, not part of the masked product; one pass over HBM each.     */
+/* ------------------------------------------------------------------------ */
+/* RMSNorm without a gain: y[r][c] = x[r][c] / sqrt(mean_c x[r][c]^2 + eps),
+ * fp32, row-major (leading dimensions ldx, ldy >= n); y may equal x.  One
+ * block per row, the sum of squares in fp32.  rows < 2^31. */
+mosaic_status mosaic_rmsnorm(const float *x, int64_t ldx, int64_t rows, int64_t n, float eps, float *y,
+                             int64_t ldy, void *stream);
+
+/* SwiGLU gate: out[r][c] = silu(gu[r][c]) * gu[r][ffn + c] with
+ * silu(g) = g / (1 + exp(-g)), fp32; gu is rows x 2 ffn (gate columns first,
+ * leading dimension ldg >= 2 ffn), out rows x ffn (ldo >= ffn; must not
+ * overlap gu).  rows <= 65535. */
+mosaic_status mosaic_swiglu(const float *gu, int64_t ldg, int64_t rows, int64_t ffn, float *out, int64_t ldo,
+                            void *stream);
+
+/* ------------------------------------------------------------------------ */
 /* Integrity check (Sec. 3.2 box, Init W step 4 and Online step 4; appendix  */
 /* "Computational integrity": Freivalds' check).                             */
 /* ------------------------------------------------------------------------ */

@@ -20,7 +20,7 @@ LIB = os.path.join(BUILD, "libmosaic.so")
 
 SOURCES = ["abi.cu", "prg.cu", "hadamard.cu", "ring_gemm_imad.cu", "ring_gemm_tc.cu", "sparse.cu",
            "noalloc.cu", "ring_gemm_skinny.cu", "freivalds.cu",
-           "ring_gemm_mma_s8.cu", "ring_gemm_tcw.cu", "timing.cu"]
+           "ring_gemm_mma_s8.cu", "ring_gemm_tcw.cu", "timing.cu", "glue.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          f"-I{ROOT}/include"]

@@ -5,9 +5,9 @@ the fused QKV projection, the attention output projection, the fused gate+up
 projection and the down projection (the four per-layer calls of Sec. 4.1).
 The non-linear parts stay on the trusted side in plain fp32 on the device, as
 the paper keeps them on the client (attention is local, Sec. 3.2 "Local
-attention computation"): RMSNorm, causal grouped-query attention with a
-softmax (torch's fused scaled-dot-product attention in fp32, causal), SiLU(gate)
-* up, and the residual adds.  Rotary position embeddings are not described by
+attention computation"): RMSNorm and SiLU(gate) * up (one-pass kernels of this
+library), causal grouped-query attention with a softmax (torch's fused
+scaled-dot-product attention in fp32, causal), and the residual adds.  Rotary position embeddings are not described by
 the paper and are left out.
 
 Weights are seeded random N(0, 0.02) (the paper's checkpoints are not
@@ -43,8 +43,18 @@ class LayerShape:
         return (self.n_heads + 2 * self.n_kv) * self.head_dim
 
 
-def rmsnorm(x: torch.Tensor, eps: float) -> torch.Tensor:
-    return x * torch.rsqrt(x.pow(2).mean(dim=-1, keepdim=True) + eps)
+def rmsnorm(x: torch.Tensor, eps: float, out: torch.Tensor | None = None) -> torch.Tensor:
+    """x / sqrt(mean(x^2) + eps) per row, one pass (mosaic_rmsnorm)."""
+    y = torch.empty_like(x) if out is None else out
+    M.mosaic_rmsnorm(x, x.stride(0), x.shape[0], x.shape[1], eps, y, y.stride(0))
+    return y
+
+
+def swiglu(gu: torch.Tensor, ffn: int, out: torch.Tensor | None = None) -> torch.Tensor:
+    """SiLU(gate) * up with gate = columns [0, ffn), up = [ffn, 2 ffn), one pass (mosaic_swiglu)."""
+    act = torch.empty(gu.shape[0], ffn, dtype=gu.dtype, device=gu.device) if out is None else out
+    M.mosaic_swiglu(gu, gu.stride(0), gu.shape[0], ffn, act, act.stride(0))
+    return act
 
 
 def attention(qkv: torch.Tensor, s: LayerShape) -> torch.Tensor:
@@ -151,5 +161,5 @@ class SecureDecoderLayer:
         a = attention(self._linear(0, h, masks[0], mark), s)
         x = x + self._linear(1, a, masks[1], mark)
         gu = self._linear(2, rmsnorm(x, s.eps), masks[2], mark)
-        act = F.silu(gu[:, : s.ffn]) * gu[:, s.ffn:]
+        act = swiglu(gu, s.ffn)
         return x + self._linear(3, act, masks[3], mark)

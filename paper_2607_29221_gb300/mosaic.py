@@ -109,6 +109,8 @@ _SIGS = {
     "mosaic_unmask_planes": ([_PP, _I64, _I64, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
                               _INT, _P, _SZ, _P], _INT),
     "mosaic_selftest_wait": ([_I64, _P], _INT),
+    "mosaic_rmsnorm": ([_P, _I64, _I64, _I64, _F32, _P, _I64, _P], _INT),
+    "mosaic_swiglu": ([_P, _I64, _I64, _I64, _P, _I64, _P], _INT),
     "mosaic_freivalds_setup": ([_PP, _PK, _U64, _INT, _P, _I64, _I64, _I64, _P, _P, _P], _INT),
     "mosaic_freivalds_check": ([_INT, _P, _P, _I64, _I64, _I64, _P, _I64, _P, _I64, _P, _P, _P, _SZ,
                                 _P], _INT),
@@ -314,6 +316,14 @@ def mosaic_unmask_noalloc(params, l, m, Z, ldz, K_tm, L, S_idx, S_val, s_w, s_x,
     _call("mosaic_unmask_noalloc", ctypes.byref(params), l, m, _ptr(Z), ldz, _ptr(K_tm), _ptr(L),
           _ptr(S_idx), _ptr(S_val), _ptr(s_w), _ptr(s_x), _ptr(bias), _ptr(Y), _ptr(Yhat), ldy,
           variant, _stream(stream))
+
+
+def mosaic_rmsnorm(x, ldx, rows, n, eps, y, ldy, stream=None):
+    _call("mosaic_rmsnorm", _ptr(x), ldx, rows, n, eps, _ptr(y), ldy, _stream(stream))
+
+
+def mosaic_swiglu(gu, ldg, rows, ffn, out, ldo, stream=None):
+    _call("mosaic_swiglu", _ptr(gu), ldg, rows, ffn, _ptr(out), ldo, _stream(stream))
 
 
 def mosaic_freivalds_setup(params, key, matrix_id, k, Wm, ldw, m, n_pad, a, Ychk, stream=None):

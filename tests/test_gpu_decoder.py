@@ -84,6 +84,10 @@ def test_fp32_glue_matches_fp64_reference(name, l):
     qkv = wl.activations(l, s.qkv, seed=32)
     got_n = _np(D.rmsnorm(torch.from_numpy(x).cuda(), s.eps))
     assert _rel(got_n, ref_rmsnorm(x.astype(np.float64), s.eps)) < 1e-6
+    gu = wl.activations(l, 2 * s.ffn, seed=33) * 4.0
+    got_s = _np(D.swiglu(torch.from_numpy(gu).cuda(), s.ffn))
+    g, u = gu[:, :s.ffn].astype(np.float64), gu[:, s.ffn:].astype(np.float64)
+    assert _rel(got_s, g / (1.0 + np.exp(-g)) * u) < 1e-6
     got_a = _np(D.attention(torch.from_numpy(qkv).cuda(), s))
     ref_a = ref_attention(qkv.astype(np.float64), s.n_heads, s.n_kv, s.head_dim)
     assert np.max(np.abs(got_a - ref_a)) < 1e-5 * np.max(np.abs(ref_a)) + 1e-6
@@ -92,6 +96,28 @@ def test_fp32_glue_matches_fp64_reference(name, l):
     for h in (0, s.n_heads - 1):
         v0 = qkv[0, (s.n_heads + s.n_kv + h // g) * s.head_dim:(s.n_heads + s.n_kv + h // g + 1) * s.head_dim]
         assert np.allclose(got_a[0, h * s.head_dim:(h + 1) * s.head_dim], v0, rtol=1e-6, atol=1e-6)
+
+
+@pytest.mark.parametrize("rows,n,ld", [(3, 37, 41), (5, 4096, 4100), (1, 1, 1)])
+def test_glue_kernels_on_ragged_rows(rows, n, ld):
+    """RMSNorm and SwiGLU on widths that are not multiples of 4 and padded
+    leading dimensions (the scalar paths), against fp64; the padding is untouched."""
+    from paper_2607_29221_gb300 import decoder as D
+    x = wl.activations(rows, ld, seed=34)
+    xt = torch.from_numpy(x).cuda()
+    y = torch.full((rows, ld), 7.0, dtype=torch.float32, device="cuda")
+    M = __import__("paper_2607_29221_gb300.mosaic", fromlist=["x"])
+    M.mosaic_rmsnorm(xt, ld, rows, n, 1e-5, y, ld)
+    xv = x[:, :n].astype(np.float64)
+    want = xv / np.sqrt(np.mean(xv * xv, axis=1, keepdims=True) + 1e-5)
+    got = _np(y)
+    assert _rel(got[:, :n], want) < 1e-6 and np.all(got[:, n:] == 7.0)
+    gu = wl.activations(rows, 2 * n + 3, seed=35)
+    out = torch.full((rows, n + 2), 5.0, dtype=torch.float32, device="cuda")
+    M.mosaic_swiglu(torch.from_numpy(gu).cuda(), 2 * n + 3, rows, n, out, n + 2)
+    g, u = gu[:, :n].astype(np.float64), gu[:, n:2 * n].astype(np.float64)
+    got = _np(out)
+    assert _rel(got[:, :n], g / (1.0 + np.exp(-g)) * u) < 1e-6 and np.all(got[:, n:] == 5.0)
 
 
 @pytest.mark.parametrize("name,l", [("small", 96), ("gqa8", 160)])
