@@ -427,6 +427,34 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (lane == 0) mbar_arrive(acc_empty);
             ++chunk_count;
 
+            // Short products (no stream-K): one chunk before the tile is written,
+            // pull this lane's row of the added / subtracted inputs into L2, so
+            // that the write-out reads them from L2 instead of waiting on DRAM.
+            if (!a.split && nchunks >= 2 && c == nchunks - 2) {
+                const int tm0 = (int)(tile % a.tiles_m) * BM, ttn0 = (int)(tile / a.tiles_m) * BN;
+                const bool sec = ttn0 >= a.N1;
+                const int gr = tm0 + row;
+                const int col = ttn0 - (sec ? a.N1 : 0) + h * HB;
+                const uint32_t *pin = sec ? a.Cin2 : a.Cin;
+                const int64_t ldp = sec ? a.ldcin2 : a.ldcin;
+                const uint32_t *psub = sec ? nullptr : a.Csub;
+                // Whole 64-column pieces only, so that every prefetched byte lies in the row.
+                if (gr < a.M && col + HB <= (sec ? a.N - a.N1 : a.N1)) {
+                    if (pin) {
+                        const char *r0 = reinterpret_cast<const char *>(pin + (int64_t)gr * ldp + col);
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(r0));
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(r0 + 128));
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(r0 + 4 * HB - 4));
+                    }
+                    if (psub) {
+                        const char *r0 = reinterpret_cast<const char *>(psub + (int64_t)gr * a.ldcsub + col);
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(r0));
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(r0 + 128));
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(r0 + 4 * HB - 4));
+                    }
+                }
+            }
+
             if (c != nchunks - 1 && k != n0 - 1 && k != n_units - 1) continue;
             // End of this CTA's segment of the tile: write it out.
             const bool whole = k < n0 || ((s1b <= tile * nchunks) && (c == nchunks - 1));
