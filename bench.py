@@ -334,10 +334,7 @@ class DecoderLayerRun:
         self.masks = self.layer.init_x(l, 90_000)
 
     def step(self, x, i, mark=None):
-        mark = mark or _no_mark
-        mark("init_x")
-        masks = self.layer.init_x(self.l, 100_000 * self.rank + i, out=self.masks)
-        return self.layer.forward(x, masks, mark=mark)
+        return self.layer.forward_pass(x, 100_000 * self.rank + i, self.masks, mark=mark)
 
     def graph(self, x):
         """The layer's step captured as one CUDA graph (fresh masks per replay
@@ -352,16 +349,15 @@ class DecoderLayerRun:
         side.wait_stream(torch.cuda.current_stream())
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=side):
-            masks = self.layer.init_x(self.l, base, pass_dev=ctr, out=gm)
-            y = self.layer.forward(x, masks)
+            y = self.layer.forward_pass(x, base, gm, pass_dev=ctr)
             M.mosaic_advance_pass(ctr, 1, stream=side)
         torch.cuda.synchronize()
         return g, y
 
     def graph_e2e(self, X, X_host, Y_host):
         """The step with its host copies as one CUDA graph: the copy of X in
-        runs on a forked stream beside the four calls' Init X (independent of
-        X), the copy of Y out ends the graph."""
+        runs on a forked stream beside the four calls' Init X draws
+        (independent of X), the copy of Y out ends the graph."""
         import torch
         from paper_2607_29221_gb300 import mosaic as M
         base = 100_000 * self.rank + 70_000
@@ -375,9 +371,9 @@ class DecoderLayerRun:
             copy.wait_stream(side)
             with torch.cuda.stream(copy):
                 X.copy_(X_host, non_blocking=True)
-            masks = self.layer.init_x(self.l, base, pass_dev=ctr, out=gm)
-            side.wait_stream(copy)
-            y = self.layer.forward(X, masks)
+            # The draws of the pass start beside the copy of X; the layer
+            # (its first composition included) waits for X.
+            y = self.layer.forward_pass(X, base, gm, pass_dev=ctr, after=copy)
             M.mosaic_advance_pass(ctr, 1, stream=side)
             Y_host.copy_(y, non_blocking=True)
         torch.cuda.synchronize()

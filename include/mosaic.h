@@ -348,6 +348,29 @@ mosaic_status mosaic_mask_activation_ex(const mosaic_params *p, const mosaic_key
                                         uint32_t *Ux_tm, uint32_t *K_tm, int variant, void *ws,
                                         size_t ws_bytes, void *stream);
 
+
+/* Init X in two parts, for callers that overlap the draws with other work
+ * (Sec. 3.2 box, Init X step 1a is the draws; 1b-1c the compositions).  Same
+ * arguments and results as mosaic_mask_activation_ex, plus `phase`:
+ *   MOSAIC_INITX_DRAWS    R (and its digit planes), the T lists into ws and
+ *                         E_x into Ux_tm: one ALU-bound launch (ChaCha20);
+ *   MOSAIC_INITX_COMPOSE  the tensor-core product and the LPN gathers that
+ *                         turn them into U_x and K;
+ *   MOSAIC_INITX_ALL      both (mosaic_mask_activation_ex).
+ * A COMPOSE call must follow the DRAWS call of the same pass with the same
+ * arguments (p, key, pass id, shapes, C, J, cj_planes, Ux_tm, K_tm, variant)
+ * and the same workspace, untouched in between (the draws live there; make
+ * the COMPOSE stream wait for the DRAWS stream).  Each phase alone validates
+ * what the whole call validates. */
+#define MOSAIC_INITX_DRAWS 1
+#define MOSAIC_INITX_COMPOSE 2
+#define MOSAIC_INITX_ALL 3
+mosaic_status mosaic_mask_activation_phase(const mosaic_params *p, const mosaic_key *key, uint64_t pass_id,
+                                           const uint64_t *pass_dev, int64_t m, int64_t n_pad, int64_t l,
+                                           const uint32_t *C, const uint32_t *J, const uint16_t *cj_planes,
+                                           uint32_t *Ux_tm, uint32_t *K_tm, int variant, void *ws,
+                                           size_t ws_bytes, int phase, void *stream);
+
 /* *pass_dev += delta, enqueued on `stream` (one-thread kernel). */
 mosaic_status mosaic_advance_pass(uint64_t *pass_dev, uint64_t delta, void *stream);
 

@@ -543,8 +543,9 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
                                    const uint64_t *pass_dev, int64_t m, int64_t n_pad, int64_t l,
                                    const uint32_t *C, const uint32_t *J, const uint16_t *cj,
                                    uint32_t *Ux_tm, uint32_t *K_tm, int variant, void *ws,
-                                   size_t ws_bytes, void *stream) {
+                                   size_t ws_bytes, void *stream, int phase = MOSAIC_INITX_ALL) {
     RoleScope role("init_x");
+    if (phase < 1 || phase > MOSAIC_INITX_ALL) return MOSAIC_ERR_ARG;
     MOSAIC_TRY(check_params(p));
     if (!key) return MOSAIC_ERR_ARG;
     if (!npad_ok(n_pad) || m < 1 || l < 0 || l >= ((int64_t)1 << 20)) return MOSAIC_ERR_SHAPE;
@@ -594,8 +595,10 @@ mosaic_status mask_activation_impl(const mosaic_params *p, const mosaic_key *key
     for (uint32_t i = 1; i < d; i++)
         lines = lines && pgather_takes(n_pad, rT[i - 1], (int)tT[i - 1]) && pgather_takes(m, rT[i - 1], (int)tT[i - 1]);
     for (uint32_t i = 1; i < d; i++) lev[i - 1].lines = lines ? 1 : 0;
-    MOSAIC_TRY(prg_initx(k, R, pass_id, pass_dev, tag_of(MOSAIC_TAG_R, 0), l, rd, Rt, Rp, Kp, (int)d - 1, tagT, rT,
-                         tT, ti, tv, tag_of(MOSAIC_TAG_EX, 0), p->sigma, l * n_pad, Ux_tm, st, lines));
+    if (phase & MOSAIC_INITX_DRAWS)
+        MOSAIC_TRY(prg_initx(k, R, pass_id, pass_dev, tag_of(MOSAIC_TAG_R, 0), l, rd, Rt, Rp, Kp, (int)d - 1, tagT,
+                             rT, tT, ti, tv, tag_of(MOSAIC_TAG_EX, 0), p->sigma, l * n_pad, Ux_tm, st, lines));
+    if (!(phase & MOSAIC_INITX_COMPOSE)) return MOSAIC_OK;
     if (fused) {
         const uint16_t *B = cj;
         if (!B) {
@@ -663,6 +666,16 @@ mosaic_status mosaic_mask_activation_ex(const mosaic_params *p, const mosaic_key
     if (cj_planes && !aligned16(cj_planes)) return MOSAIC_ERR_ALIGN;
     return mask_activation_impl(p, key, pass_id, pass_dev, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm,
                                 variant, ws, ws_bytes, stream);
+}
+
+mosaic_status mosaic_mask_activation_phase(const mosaic_params *p, const mosaic_key *key, uint64_t pass_id,
+                                           const uint64_t *pass_dev, int64_t m, int64_t n_pad, int64_t l,
+                                           const uint32_t *C, const uint32_t *J, const uint16_t *cj_planes,
+                                           uint32_t *Ux_tm, uint32_t *K_tm, int variant, void *ws,
+                                           size_t ws_bytes, int phase, void *stream) {
+    if (cj_planes && !aligned16(cj_planes)) return MOSAIC_ERR_ALIGN;
+    return mask_activation_impl(p, key, pass_id, pass_dev, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm,
+                                variant, ws, ws_bytes, stream, phase);
 }
 
 mosaic_status mosaic_mask(int kind, const mosaic_params *p, const mosaic_key *key, uint64_t stream_id,

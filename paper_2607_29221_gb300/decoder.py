@@ -111,9 +111,14 @@ class SecureDecoderLayer:
         return [self.qkv, self.o, self.gu, self.down]
 
     def alloc(self, l: int) -> None:
-        """Preallocates every per-pass buffer of the four calls for l tokens."""
+        """Preallocates every per-pass buffer of the four calls for l tokens,
+        the Init X workspaces of the four calls (their draws stay there until
+        the compositions run, see forward_pass) and the stream of the draws."""
         dev = self.proto.device
         Sr = self.proto.sum_r
+        self.initx_ws = [torch.empty(max(lin.init_x_workspace_bytes(l), 256), dtype=torch.uint8, device=dev)
+                         for lin in self.linears()]
+        self.draw_stream = torch.cuda.Stream(device=dev)
         self.bufs = []
         for lin in self.linears():
             planes = lin.use_planes and l > M.STREAMW_MAX_M
@@ -135,9 +140,12 @@ class SecureDecoderLayer:
         return [lin.init_x(l, 1_000_000 * (i + 1) + pass_base, pass_dev=pass_dev, out=outs[i])
                 for i, lin in enumerate(self.linears())]
 
-    def _linear(self, i: int, x: torch.Tensor, mp, mark) -> torch.Tensor:
+    def _linear(self, i: int, x: torch.Tensor, mp, mark, compose=None) -> torch.Tensor:
         lin = self.linears()[i]
         b = self.bufs[i] if self.bufs is not None else {}
+        if compose is not None:
+            mark("init_x")
+            compose(i)
         mark("encode")
         Xp, s_x, Xpl = lin.mask_input(x, mp, b.get("Xp"), b.get("s_x"), b.get("Xpl"))
         mark("server")
@@ -147,10 +155,11 @@ class SecureDecoderLayer:
         mark("glue")
         return Y
 
-    def forward(self, x: torch.Tensor, masks=None, mark=None) -> torch.Tensor:
+    def forward(self, x: torch.Tensor, masks=None, mark=None, compose=None) -> torch.Tensor:
         """One pass over l tokens (x: l x hidden fp32).  `mark(part)`, if given,
         is called where each part of the pass begins (init_x, encode, server,
-        unmask, glue), e.g. to record CUDA events."""
+        unmask, glue), e.g. to record CUDA events.  With `compose`, call i's
+        Init X composition runs (compose(i)) right before its encode."""
         s = self.s
         mark = mark or _no_mark
         if masks is None:
@@ -158,8 +167,52 @@ class SecureDecoderLayer:
             masks = self.init_x(x.shape[0])
         mark("glue")
         h = rmsnorm(x, s.eps)
-        a = attention(self._linear(0, h, masks[0], mark), s)
-        x = x + self._linear(1, a, masks[1], mark)
-        gu = self._linear(2, rmsnorm(x, s.eps), masks[2], mark)
+        a = attention(self._linear(0, h, masks[0], mark, compose), s)
+        x = x + self._linear(1, a, masks[1], mark, compose)
+        gu = self._linear(2, rmsnorm(x, s.eps), masks[2], mark, compose)
         act = swiglu(gu, s.ffn)
-        return x + self._linear(3, act, masks[3], mark)
+        return x + self._linear(3, act, masks[3], mark, compose)
+
+    def forward_pass(self, x: torch.Tensor, pass_base: int, masks, pass_dev=None, mark=None,
+                     after=None) -> torch.Tensor:
+        """Init X and the layer of one pass, with the Init X draws (ALU-bound
+        ChaCha20 in blocks of 128 threads and 9 KB of shared memory) on a side
+        stream: call 0's draws at the start of the pass, the other three
+        calls' draws once call 0's composition is done, beside its encode,
+        server product, unmask and the attention; every composition (product
+        and gathers, which need the SM's shared memory) runs on the main
+        stream right before its call's encode.  Call 1's composition waits
+        for all three, so no draw runs beside an Init X gather.  Same pass ids
+        and results as init_x + forward (call i draws pass pass_base +
+        1_000_000 (i + 1), plus *pass_dev); `masks` are the four calls'
+        preallocated U_x / K buffers; `after`, a stream that the layer (not
+        the draws) waits for first, e.g. the copy of x.  Needs alloc."""
+        l = x.shape[0]
+        main = torch.cuda.current_stream()
+        side = self.draw_stream
+        side.wait_stream(main)
+        lins = self.linears()
+        pids = [1_000_000 * (i + 1) + pass_base for i in range(4)]
+
+        def draw(i):
+            lins[i].init_x(l, pids[i], pass_dev=pass_dev, out=masks[i], phase=M.INITX_DRAWS, ws=self.initx_ws[i])
+
+        first, rest = torch.cuda.Event(), torch.cuda.Event()
+        with torch.cuda.stream(side):
+            draw(0)
+            first.record(side)
+        if after is not None:
+            main.wait_stream(after)
+
+        def compose(i):
+            main.wait_event(first if i == 0 else rest)
+            lins[i].init_x(l, pids[i], pass_dev=pass_dev, out=masks[i], phase=M.INITX_COMPOSE,
+                           ws=self.initx_ws[i])
+            if i == 0:
+                side.wait_stream(main)
+                with torch.cuda.stream(side):
+                    for j in (1, 2, 3):
+                        draw(j)
+                    rest.record(side)
+
+        return self.forward(x, masks, mark=mark, compose=compose)

@@ -102,6 +102,8 @@ _SIGS = {
                                        _SZ, _P], _INT),
     "mosaic_mask_activation_ex": ([_PP, _PK, _U64, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _INT, _P, _SZ,
                                    _P], _INT),
+    "mosaic_mask_activation_phase": ([_PP, _PK, _U64, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _INT, _P, _SZ,
+                                      _INT, _P], _INT),
     "mosaic_advance_pass": ([_P, _U64, _P], _INT),
     "mosaic_mask": ([_INT, _PP, _PK, _U64, _I64, _I64, _I64, ctypes.POINTER(mosaic_mask_io), _INT, _P, _SZ,
                      _P], _INT),
@@ -365,6 +367,16 @@ def mosaic_mask_activation_ex(params, key, pass_id, pass_dev, m, n_pad, l, C, J,
     _call("mosaic_mask_activation_ex", ctypes.byref(params), ctypes.byref(key), pass_id, _ptr(pass_dev), m,
           n_pad, l, _ptr(C), _ptr(J), _ptr(cj_planes), _ptr(Ux_tm), _ptr(K_tm), variant, _ptr(ws),
           0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
+
+
+INITX_DRAWS, INITX_COMPOSE, INITX_ALL = 1, 2, 3
+
+
+def mosaic_mask_activation_phase(params, key, pass_id, pass_dev, m, n_pad, l, C, J, cj_planes, Ux_tm, K_tm,
+                                 variant, ws, phase, stream=None):
+    _call("mosaic_mask_activation_phase", ctypes.byref(params), ctypes.byref(key), pass_id, _ptr(pass_dev), m,
+          n_pad, l, _ptr(C), _ptr(J), _ptr(cj_planes), _ptr(Ux_tm), _ptr(K_tm), variant, _ptr(ws),
+          0 if ws is None else ws.numel() * ws.element_size(), phase, _stream(stream))
 
 
 def mosaic_mask(kind, params, key, stream_id, rows, n_pad, l, io: dict, variant=GEMM_AUTO, ws=None,

@@ -129,17 +129,28 @@ class SecureLinear:
             M.mosaic_prepare_unmask(p, m, self.L, self.L_planes)
 
     # Init X ---------------------------------------------------------------
-    def init_x(self, l: int, pass_id: int, pass_dev=None, out: PassMask | None = None) -> PassMask:
+    def init_x_workspace_bytes(self, l: int) -> int:
+        return M.mosaic_workspace_bytes(M.OP_MASK_ACTIVATION, self.m, self.n_pad, l, self.proto.params)
+
+    def init_x(self, l: int, pass_id: int, pass_dev=None, out: PassMask | None = None,
+               phase: int = M.INITX_ALL, ws=None) -> PassMask:
         """Init X for one pass.  pass_dev (a device int64 word, optional) is
         added to pass_id on the device, so that a captured CUDA graph draws a
-        fresh pass on every replay; `out` reuses preallocated U_x / K buffers."""
+        fresh pass on every replay; `out` reuses preallocated U_x / K buffers.
+        `phase` INITX_DRAWS / INITX_COMPOSE runs one part (the second call
+        with the same arguments and the same `ws`, left untouched between)."""
         p, dev = self.proto.params, self.proto.device
         Ux = _u32(l, self.n_pad, device=dev) if out is None else out.Ux
         K = _u32(l, self.m, device=dev) if out is None else out.K
-        ws = self.proto.workspace(
-            M.mosaic_workspace_bytes(M.OP_MASK_ACTIVATION, self.m, self.n_pad, l, p))
-        M.mosaic_mask_activation_ex(p, self.proto.key, pass_id, pass_dev, self.m, self.n_pad, l,
-                                    self.chains.C, self.J, self.cj_planes, Ux, K, self.proto.variant, ws)
+        if ws is None:
+            ws = self.proto.workspace(self.init_x_workspace_bytes(l))
+        if phase == M.INITX_ALL:
+            M.mosaic_mask_activation_ex(p, self.proto.key, pass_id, pass_dev, self.m, self.n_pad, l,
+                                        self.chains.C, self.J, self.cj_planes, Ux, K, self.proto.variant, ws)
+        else:
+            M.mosaic_mask_activation_phase(p, self.proto.key, pass_id, pass_dev, self.m, self.n_pad, l,
+                                           self.chains.C, self.J, self.cj_planes, Ux, K, self.proto.variant, ws,
+                                           phase)
         return PassMask(pass_id, l, Ux, K) if out is None else out
 
     # Online ---------------------------------------------------------------

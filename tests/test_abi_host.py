@@ -138,6 +138,12 @@ def test_validation_of_newer_entry_points(lib):
     bad = M.default_params(act_nested=2)
     assert _status("mosaic_mask_activation_ex", ctypes.byref(bad), ctypes.byref(key), 0, None, 8, 32, 4,
                    fake, fake, None, fake, fake, 0, None, 0, None) == 1
+    # Init X phases: 1 (draws), 2 (compositions), 3 (both); anything else is refused
+    for phase in (0, 4, -1):
+        assert _status("mosaic_mask_activation_phase", ctypes.byref(p), ctypes.byref(key), 0, None, 8, 32, 4,
+                       fake, fake, None, fake, fake, 0, None, 0, phase, None) == 1
+    assert _status("mosaic_mask_activation_phase", ctypes.byref(bad), ctypes.byref(key), 0, None, 8, 32, 4,
+                   fake, fake, None, fake, fake, 0, None, 0, 1, None) == 1
     # K above 2^20, rotation widths beyond 65536
     assert _status("mosaic_ring_gemm", fake, 1 << 21, fake, 1 << 21, fake, 8, 8, 8, (1 << 20) + 1, 3,
                    None, 0, None) == 2

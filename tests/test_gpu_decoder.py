@@ -182,3 +182,41 @@ def test_layer_graph_replays_match_eager_passes():
         assert np.array_equal(_np(y_g), eager[k]), k
     assert not np.array_equal(eager[0], eager[1])
     M.mosaic_device_status()
+
+
+@pytest.mark.parametrize("l", [64, 24])
+def test_overlapped_pass_matches_init_x_then_forward(l):
+    """forward_pass (the four calls' Init X draws on a side stream from the
+    start of the pass, each composition right before its call's encode) gives
+    the decoded output of init_x + forward with the same pass ids, bit for bit:
+    eager, and captured as one CUDA graph whose replays advance a device pass
+    counter.  l = 24 runs the streaming tensor-core server product."""
+    from paper_2607_29221_gb300 import decoder as D
+    from paper_2607_29221_gb300 import mosaic as M
+    from paper_2607_29221_gb300 import protocol as PR
+    s = D.LayerShape(**SHAPES["small"])
+    proto = PR.Protocol(wl.mask_key(), M.default_params(), variant=M.GEMM_AUTO)
+    layer = D.SecureDecoderLayer(proto, D.LayerWeights(s, seed=29))
+    layer.alloc(l)
+    x = torch.from_numpy(wl.activations(l, s.hidden, seed=6)).cuda()
+    base = 700
+    want = []
+    for k in range(3):
+        want.append(_np(layer.forward(x, layer.init_x(l, base + k))).copy())
+    masks = layer.init_x(l, 1)
+    got = _np(layer.forward_pass(x, base, masks)).copy()
+    assert np.array_equal(got, want[0])
+    ctr = torch.zeros(1, dtype=torch.int64, device="cuda")
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        y_g = layer.forward_pass(x, base, masks, pass_dev=ctr)
+        M.mosaic_advance_pass(ctr, 1, stream=side)
+    torch.cuda.synchronize()
+    for k in range(3):
+        g.replay()
+        torch.cuda.synchronize()
+        assert np.array_equal(_np(y_g), want[k]), k
+    M.mosaic_device_status()

@@ -81,3 +81,28 @@ def test_mosaic_mask_each_kind_matches_oracle(act_nested):
     xo = O.init_x(KEY, po, l, pass_id, Co, wo.J, n_pad)
     assert np.array_equal(_u32(Ux), xo.U_x.T)
     assert np.array_equal(_u32(K), xo.K.T)
+
+
+def test_init_x_in_two_phases_matches_one_call():
+    """mosaic_mask_activation_phase: the DRAWS call then the COMPOSE call on
+    the same workspace give U_x and K bit-identical to one
+    mosaic_mask_activation_ex call; the draws alone leave K untouched."""
+    import torch
+    from paper_2607_29221_gb300 import mosaic as M
+    from paper_2607_29221_gb300 import protocol as PR
+    from paper_2607_29221_gb300 import workloads as wl
+    proto = PR.Protocol(wl.mask_key(), M.default_params(d=3, r=[96, 64, 40], t=[0, 8, 4]), variant=M.GEMM_TC)
+    m, n, l = 200, 256, 96
+    ch = PR.Chains(proto, PR.pad_width(n))
+    layer = PR.SecureLinear(proto, torch.from_numpy(wl.weights(m, n, std=1.0)).cuda(), 4, ch)
+    one = layer.init_x(l, 42)
+    ws = torch.empty(layer.init_x_workspace_bytes(l), dtype=torch.uint8, device="cuda")
+    two = PR.PassMask(42, l, torch.empty_like(one.Ux), torch.full_like(one.K, 7))
+    layer.init_x(l, 42, out=two, phase=M.INITX_DRAWS, ws=ws)
+    torch.cuda.synchronize()
+    assert bool((two.K == 7).all())
+    layer.init_x(l, 42, out=two, phase=M.INITX_COMPOSE, ws=ws)
+    torch.cuda.synchronize()
+    assert torch.equal(one.Ux, two.Ux) and torch.equal(one.K, two.K)
+    with pytest.raises(M.MosaicError):
+        layer.init_x(l, 42, out=two, phase=0, ws=ws)
