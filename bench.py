@@ -292,27 +292,33 @@ class LinearChain:
         torch.cuda.synchronize()
         return g, y
 
-    def graph_e2e(self, X, X_host, Y_host):
+    def graph_e2e(self, X, X_host, Y_host_prev, Y_dev_prev, Y_dev_out):
         """The step with its host copies as one CUDA graph: the copy of X in
         runs on a forked stream beside every layer's Init X (which does not
-        depend on X), the copy of Y out ends the graph."""
+        depend on X); the previous step's result Y_dev_prev is read out to
+        Y_host_prev on another forked stream beside the whole step, and this
+        step's result ends in Y_dev_out (read out by the next step)."""
         import torch
         dev = X.device
         base = [1_000_000 * self.rank + 700_000 + 1000 * c for c in range(len(self.layers))]
         ctr = [torch.zeros(1, dtype=torch.int64, device=dev) for _ in self.layers]
         gmask = [ly.init_x(self.l, b) for ly, b in zip(self.layers, base)]
         torch.cuda.synchronize()
-        side, copy = torch.cuda.Stream(), torch.cuda.Stream()
+        side, copy, out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
         side.wait_stream(torch.cuda.current_stream())
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=side):
             copy.wait_stream(side)
+            out.wait_stream(side)
             with torch.cuda.stream(copy):
                 X.copy_(X_host, non_blocking=True)
+            with torch.cuda.stream(out):
+                Y_host_prev.copy_(Y_dev_prev, non_blocking=True)
             mps = [ly.init_x(self.l, base[c], pass_dev=ctr[c], out=gmask[c]) for c, ly in enumerate(self.layers)]
             side.wait_stream(copy)
             y = self._pass(X, mps, ctr, side)
-            Y_host.copy_(y, non_blocking=True)
+            Y_dev_out.copy_(y, non_blocking=True)
+            side.wait_stream(out)
         torch.cuda.synchronize()
         return g
 
@@ -360,28 +366,32 @@ class DecoderLayerRun:
         torch.cuda.synchronize()
         return g, y
 
-    def graph_e2e(self, X, X_host, Y_host):
+    def graph_e2e(self, X, X_host, Y_host_prev, Y_dev_prev, Y_dev_out):
         """The step with its host copies as one CUDA graph: the copy of X in
-        runs on a forked stream beside the four calls' Init X draws
-        (independent of X), the copy of Y out ends the graph."""
+        runs on a forked stream beside the first call's Init X draws
+        (independent of X); the previous step's result Y_dev_prev is read out
+        to Y_host_prev on another forked stream beside the whole step, and
+        this step's result ends in Y_dev_out (read out by the next step)."""
         import torch
         from paper_2607_29221_gb300 import mosaic as M
         base = 100_000 * self.rank + 70_000
         ctr = torch.zeros(1, dtype=torch.int64, device=X.device)
         gm = self.layer.init_x(self.l, base)
         torch.cuda.synchronize()
-        side, copy = torch.cuda.Stream(), torch.cuda.Stream()
+        side, copy, out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
         side.wait_stream(torch.cuda.current_stream())
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=side):
             copy.wait_stream(side)
+            out.wait_stream(side)
             with torch.cuda.stream(copy):
                 X.copy_(X_host, non_blocking=True)
-            # The draws of the pass start beside the copy of X; the layer
-            # (its first composition included) waits for X.
+            with torch.cuda.stream(out):
+                Y_host_prev.copy_(Y_dev_prev, non_blocking=True)
             y = self.layer.forward_pass(X, base, gm, pass_dev=ctr, after=copy)
             M.mosaic_advance_pass(ctr, 1, stream=side)
-            Y_host.copy_(y, non_blocking=True)
+            Y_dev_out.copy_(y, non_blocking=True)
+            side.wait_stream(out)
         torch.cuda.synchronize()
         return g
 
@@ -522,12 +532,23 @@ def run_mine(args, rank, world):
         Y = runner.step(X, 10_000 + i)
         Y_host.copy_(Y, non_blocking=True)
     e2e_eager_ms = _e2e(_eager_e2e)
-    ge = runner.graph_e2e(X, X_host, Y_host)
-    for i in range(3):
-        ge.replay()
+    # The graph form pipelines the read-out: step k copies X in and reads out
+    # step k - 1's result while it computes (two graphs alternate the device
+    # buffer of the result); the last step's result is read inside the last
+    # step's timed region.
+    Y_dev = [torch.empty(l, runner.m_out, dtype=torch.float32, device=dev) for _ in range(2)]
+    Y_hosts = [Y_host, torch.empty(l, runner.m_out, dtype=torch.float32).pin_memory()]
+    ges = [runner.graph_e2e(X, X_host, Y_hosts[1 - p], Y_dev[1 - p], Y_dev[p]) for p in (0, 1)]
+    for i in range(4):
+        ges[i % 2].replay()
     torch.cuda.synchronize()
-    e2e_ms = _e2e(lambda i: ge.replay())
-    del ge
+
+    def _graph_e2e(i):
+        ges[i % 2].replay()
+        if i == e2e_steps - 1:
+            Y_hosts[i % 2].copy_(Y_dev[i % 2], non_blocking=True)
+    e2e_ms = _e2e(_graph_e2e)
+    del ges
     clocks = sampler.stop()
     M.mosaic_device_status()
 
@@ -580,7 +601,8 @@ def run_mine(args, rank, world):
         "rooflines": rooflines,
         "e2e": {"value": round(world * l / (e2e_ms_max / 1e3), 1), "unit": "tokens/s",
                 "h2d_bytes_per_step": l * runner.n_in * 4, "d2h_bytes_per_step": l * runner.m_out * 4,
-                "launch": "one CUDA graph per step, the copy of X overlapping Init X",
+                "launch": "one CUDA graph per step: the copy of X in beside Init X, the previous step's "
+                          "result read out beside the whole step (the last step's inside its own timing)",
                 "value_eager": round(world * l / (e2e_eager_ms_max / 1e3), 1)},
         "gpu_launches": int(launches_timed),
         "kernel_ms_per_step": {k: round(v[1] / part_steps, 4) for k, v in sorted(ktimes.items())},

@@ -179,10 +179,11 @@ class SecureDecoderLayer:
         ChaCha20 in blocks of 128 threads and 9 KB of shared memory) on a side
         stream: call 0's draws at the start of the pass, the other three
         calls' draws once call 0's composition is done, beside its encode,
-        server product, unmask and the attention; every composition (product
-        and gathers, which need the SM's shared memory) runs on the main
-        stream right before its call's encode.  Call 1's composition waits
-        for all three, so no draw runs beside an Init X gather.  Same pass ids
+        server product, unmask and the attention.  Call 0's composition
+        (product and gathers, which need the SM's shared memory) runs first,
+        before the layer waits for `after`; the others on the main stream
+        right before their call's encode.  Call 1's composition waits for all
+        three draws, so no draw runs beside an Init X gather.  Same pass ids
         and results as init_x + forward (call i draws pass pass_base +
         1_000_000 (i + 1), plus *pass_dev); `masks` are the four calls'
         preallocated U_x / K buffers; `after`, a stream that the layer (not
@@ -201,18 +202,24 @@ class SecureDecoderLayer:
         with torch.cuda.stream(side):
             draw(0)
             first.record(side)
+        # Call 0's composition does not depend on x either: it runs before
+        # the layer waits for `after`.
+        (mark or _no_mark)("init_x")
+        main.wait_event(first)
+        lins[0].init_x(l, pids[0], pass_dev=pass_dev, out=masks[0], phase=M.INITX_COMPOSE, ws=self.initx_ws[0])
+        side.wait_stream(main)
+        with torch.cuda.stream(side):
+            for j in (1, 2, 3):
+                draw(j)
+            rest.record(side)
         if after is not None:
             main.wait_stream(after)
 
         def compose(i):
-            main.wait_event(first if i == 0 else rest)
+            if i == 0:
+                return
+            main.wait_event(rest)
             lins[i].init_x(l, pids[i], pass_dev=pass_dev, out=masks[i], phase=M.INITX_COMPOSE,
                            ws=self.initx_ws[i])
-            if i == 0:
-                side.wait_stream(main)
-                with torch.cuda.stream(side):
-                    for j in (1, 2, 3):
-                        draw(j)
-                    rest.record(side)
 
         return self.forward(x, masks, mark=mark, compose=compose)
