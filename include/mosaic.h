@@ -99,9 +99,11 @@ uint64_t mosaic_kernel_launches(void);
  * mosaic_kernel_times waits for every recorded pair, adds the durations to
  * per-key totals and writes up to `cap` of them to `out` (cap may be 0); the
  * key is "<role>:<kernel>", role naming the entry point that launched the
- * kernel (init_x, encode, server, unmask, init_w, ...).  With `reset` the
- * totals start again from zero after being written.  Returns the number of
- * keys, or -1 if an event could not be read (the records are dropped). */
+ * kernel (init_x, encode, ring_gemm, unmask, init_w, glue, ...).  With
+ * `reset` the totals start again from zero after being written.  Returns the
+ * number of keys, or -1 if an event could not be read (the records are
+ * dropped).  Recorded pairs (and their events) stay held until this call
+ * reads them. */
 typedef struct {
     char name[64];
     uint64_t launches;
