@@ -509,6 +509,12 @@ def run_mine(args, rank, world):
     torch.cuda.synchronize()
     M.mosaic_kernel_timing(False)
     ktimes = M.mosaic_kernel_times(reset=True)
+    # The device's rate of the ChaCha20 add / xor / rotate mix: the draws' ALU peak.
+    mix_scratch = torch.empty(8 * 256 * 256, dtype=torch.int32, device=dev)
+    alu_rate = M.mosaic_int_mix_rate(mix_scratch)
+    # ... and its conflict-free shared-memory read rate: the gathers' peak.
+    smem_rate = M.mosaic_smem_read_rate(mix_scratch)
+    del mix_scratch
 
     # End to end through the public API with host buffers: the copy of X in
     # and of Y out inside the timed region, every step.
@@ -582,7 +588,8 @@ def run_mine(args, rank, world):
                   "traffic": None, "bytes_per_step": enc_bytes, "ms_per_step": round(enc_ms, 4),
                   "peak_source": f"{peak_src} copy bandwidth"}]
     rooflines += _client_rooflines(ktimes, part_steps, runner.layers, proto, l, bf16, peak_src,
-                                   float(clocks.get("sm_mhz") or clocks.get("sm_max_mhz") or 2070.0))
+                                   float(clocks.get("sm_mhz") or clocks.get("sm_max_mhz") or 2070.0), alu_rate,
+                                   smem_rate)
     out = {
         "metric": METRIC, "value": round(tokens_s, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms_max, 4),
@@ -625,7 +632,7 @@ SMEM_BYTES_PER_CLK_SM = 128
 CHACHA_OPS_PER_BLOCK = 20 * 4 * 12 + 16   # 80 quarter rounds of 12 add/xor/rotate, 16 final adds
 
 
-def _client_rooflines(kt, steps, layers, proto, l, bf16, peak_src, sm_mhz):
+def _client_rooflines(kt, steps, layers, proto, l, bf16, peak_src, sm_mhz, alu_measured=None, smem_measured=None):
     """Rooflines of the client kernels from the library's per-kernel event
     times (`kt`: {"<role>:<kernel>": (launches, ms)} over `steps` eager steps).
     Algorithmic work per step, summed over the step's secure linears:
@@ -646,18 +653,28 @@ def _client_rooflines(kt, steps, layers, proto, l, bf16, peak_src, sm_mhz):
     w_lv = list(range(1, d))
     clk = sm_mhz * 1e6
     alu_peak = GB300_SMS * INT_OPS_PER_CLK_SM * clk / 1e12
+    alu_src = "derived int32 ALU peak"
+    if alu_measured:
+        # The device's measured rate of the same add / xor / rotate mix.
+        alu_peak = alu_measured / 1e12
+        alu_src = "measured ChaCha20 mix rate (mosaic_int_mix_rate)"
     smem_peak = GB300_SMS * SMEM_BYTES_PER_CLK_SM * clk / 1e9
+    smem_src = "derived shared-memory wavefront peak"
+    if smem_measured:
+        # The device's measured conflict-free 16-byte shared-memory read rate.
+        smem_peak = smem_measured / 1e9
+        smem_src = "measured shared-memory read rate (mosaic_smem_read_rate)"
     blocks = sum(-(-l * r_act // 16) + len(act_lv) * l * 32 + -(-l * ly.n_pad // 8) for ly in layers)
     gx = sum(l * (ly.n_pad + ly.m) * t[i] for ly in layers for i in act_lv)
     gu = sum(ly.m * l * t[i] for ly in layers for i in w_lv)
     fx = sum(20 * l * (ly.n_pad + ly.m) * r_act for ly in layers)
     fu = sum(20 * l * ly.m * r[d - 1] for ly in layers)
     rows = [("init_x:initx_draw", "initx_draw_kernel (Init X draws: R, T lists, E_x; ChaCha20)", "alu",
-             blocks * CHACHA_OPS_PER_BLOCK / 1e12, alu_peak, "Tops/s", "derived int32 ALU peak"),
+             blocks * CHACHA_OPS_PER_BLOCK / 1e12, alu_peak, "Tops/s", alu_src),
             ("init_x:pgather", "pgather_kernel (Init X LPN terms of U_x and K)", "smem",
-             gx * 4 / 1e9, smem_peak, "GB/s", "derived shared-memory wavefront peak"),
+             gx * 4 / 1e9, smem_peak, "GB/s", smem_src),
             ("unmask:pgather", "pgather_kernel (unmask LPN terms + decode)", "smem",
-             gu * 4 / 1e9, smem_peak, "GB/s", "derived shared-memory wavefront peak"),
+             gu * 4 / 1e9, smem_peak, "GB/s", smem_src),
             ("init_x:ring_gemm_tc", "ring_gemm_tc_kernel (Init X: R [C_d; J_d]^T, K = r_d)", "tensor",
              fx / 1e12, bf16, "TFLOP/s", f"{peak_src} bf16 dense burst"),
             ("unmask:ring_gemm_tc", "ring_gemm_tc_kernel (unmask: Y' - K - Q_d L^T, K = r_d)", "tensor",

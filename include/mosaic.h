@@ -112,6 +112,24 @@ typedef struct {
 int mosaic_kernel_timing(int enable);
 int mosaic_kernel_times(mosaic_kernel_time *out, int cap, int reset);
 
+/* Rate of the ChaCha20 integer mix (add, xor, rotate) on the current device,
+ * in operations per second, for the draws' roofline (not part of the
+ * method): one launch of 8 blocks of 256 threads per SM, each thread running
+ * 2000 double rounds on 16 independent words, timed with CUDA events; waits
+ * for the launch.  `scratch` is a device buffer of at least 8192 bytes per SM
+ * (one word per thread is written there).  About 2 ms of GPU time. */
+mosaic_status mosaic_int_mix_rate(uint32_t *scratch, size_t scratch_bytes, double *ops_per_second, void *stream);
+
+/* Shared-memory read rate of the current device in bytes per second, for the
+ * gathers' roofline (not part of the method), with the tiled gather's access:
+ * two blocks of 512 threads and 64 KB per SM, each group of 8 lanes reading a
+ * whole 128-byte line per 16-byte load instruction (four scattered lines per
+ * warp access), 4000 x 8 volatile loads a thread, timed with CUDA events;
+ * waits for the launch.  `scratch` is a device buffer of at least 4096 bytes
+ * per SM.  About 1 ms of GPU time. */
+mosaic_status mosaic_smem_read_rate(uint32_t *scratch, size_t scratch_bytes, double *bytes_per_second,
+                                    void *stream);
+
 /* Human-readable name of a status code (static string). */
 const char *mosaic_status_string(mosaic_status s);
 

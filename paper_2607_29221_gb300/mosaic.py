@@ -71,6 +71,8 @@ _SIGS = {
     "mosaic_default_params": ([_PP], None),
     "mosaic_kernel_launches": ([], ctypes.c_uint64),
     "mosaic_kernel_timing": ([_INT], _INT),
+    "mosaic_int_mix_rate": ([_P, _SZ, ctypes.POINTER(ctypes.c_double), _P], _INT),
+    "mosaic_smem_read_rate": ([_P, _SZ, ctypes.POINTER(ctypes.c_double), _P], _INT),
     "mosaic_kernel_times": ([ctypes.POINTER(mosaic_kernel_time), _INT, _INT], _INT),
     "mosaic_status_string": ([_INT], ctypes.c_char_p),
     "mosaic_qmax": ([_I64, _U32], ctypes.c_int32),
@@ -204,6 +206,22 @@ def mosaic_kernel_times(reset: bool = True) -> dict:
     if n < 0:
         raise MosaicError("mosaic_kernel_times", -1)
     return {buf[i].name.decode(): (int(buf[i].launches), float(buf[i].ms)) for i in range(min(n, len(buf)))}
+
+
+def mosaic_int_mix_rate(scratch, stream=None) -> float:
+    """Measured ChaCha20 mix (add / xor / rotate) rate of the device, ops/s."""
+    out = ctypes.c_double(0.0)
+    _call("mosaic_int_mix_rate", _ptr(scratch), scratch.numel() * scratch.element_size(), ctypes.byref(out),
+          _stream(stream))
+    return float(out.value)
+
+
+def mosaic_smem_read_rate(scratch, stream=None) -> float:
+    """Measured conflict-free shared-memory read rate of the device, bytes/s."""
+    out = ctypes.c_double(0.0)
+    _call("mosaic_smem_read_rate", _ptr(scratch), scratch.numel() * scratch.element_size(), ctypes.byref(out),
+          _stream(stream))
+    return float(out.value)
 
 
 def mosaic_qmax(n_pad: int, qbits: int = 16) -> int:

@@ -158,6 +158,11 @@ def test_validation_of_newer_entry_points(lib):
                    fake, fake, fake, None, fake, None, 8, 3, None, 0, None) == 3
 
 
+def test_rate_probes_need_an_output(lib):
+    assert _status("mosaic_int_mix_rate", None, 0, None, None) == 1
+    assert _status("mosaic_smem_read_rate", None, 0, None, None) == 1
+
+
 def test_selftest_wait_validates_its_limit(lib):
     assert _status("mosaic_selftest_wait", 0, None) == 1
     assert _status("mosaic_selftest_wait", 1000001, None) == 1

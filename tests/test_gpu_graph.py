@@ -128,3 +128,30 @@ def test_kernel_timing_records_eager_launches_only():
     g.replay()
     torch.cuda.synchronize()
     del g
+
+
+def test_int_mix_rate_is_measured_and_validated():
+    """mosaic_int_mix_rate: a positive rate of the ChaCha20 mix within the
+    bounds one GB300-class part allows, and a refusal of a scratch buffer
+    that is too small."""
+    from paper_2607_29221_gb300 import mosaic as M
+    scratch = torch.empty(8 * 256 * 256, dtype=torch.int32, device="cuda")
+    rate = M.mosaic_int_mix_rate(scratch)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    # between 16 and 256 32-bit ops per clock per SM at 0.5 to 3 GHz
+    assert sms * 16 * 0.5e9 < rate < sms * 256 * 3.0e9, rate
+    with pytest.raises(M.MosaicError):
+        M.mosaic_int_mix_rate(torch.empty(16, dtype=torch.int32, device="cuda"))
+
+
+def test_smem_read_rate_is_measured_and_validated():
+    """mosaic_smem_read_rate: a positive shared-memory read rate no higher than
+    a few lines per clock per SM, and a refusal of a scratch buffer that is
+    too small."""
+    from paper_2607_29221_gb300 import mosaic as M
+    scratch = torch.empty(8 * 256 * 256, dtype=torch.int32, device="cuda")
+    rate = M.mosaic_smem_read_rate(scratch)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    assert sms * 16 * 0.5e9 < rate < sms * 512 * 3.0e9, rate
+    with pytest.raises(M.MosaicError):
+        M.mosaic_smem_read_rate(torch.empty(16, dtype=torch.int32, device="cuda"))

@@ -83,16 +83,20 @@ def test_mosaic_mask_each_kind_matches_oracle(act_nested):
     assert np.array_equal(_u32(K), xo.K.T)
 
 
-def test_init_x_in_two_phases_matches_one_call():
+@pytest.mark.parametrize("l,nested", [(96, 1), (12, 1), (96, 0)])
+def test_init_x_in_two_phases_matches_one_call(l, nested):
     """mosaic_mask_activation_phase: the DRAWS call then the COMPOSE call on
     the same workspace give U_x and K bit-identical to one
-    mosaic_mask_activation_ex call; the draws alone leave K untouched."""
+    mosaic_mask_activation_ex call (tensor-core product, the streaming
+    product at 12 tokens, and the LWE-only activation mask); the draws alone
+    leave K untouched."""
     import torch
     from paper_2607_29221_gb300 import mosaic as M
     from paper_2607_29221_gb300 import protocol as PR
     from paper_2607_29221_gb300 import workloads as wl
-    proto = PR.Protocol(wl.mask_key(), M.default_params(d=3, r=[96, 64, 40], t=[0, 8, 4]), variant=M.GEMM_TC)
-    m, n, l = 200, 256, 96
+    proto = PR.Protocol(wl.mask_key(), M.default_params(d=3, r=[96, 64, 40], t=[0, 8, 4], act_nested=nested),
+                        variant=M.GEMM_TC)
+    m, n = 200, 256
     ch = PR.Chains(proto, PR.pad_width(n))
     layer = PR.SecureLinear(proto, torch.from_numpy(wl.weights(m, n, std=1.0)).cuda(), 4, ch)
     one = layer.init_x(l, 42)
