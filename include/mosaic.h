@@ -513,12 +513,10 @@ mosaic_status mosaic_device_status(void *stream);
  *    MOSAIC_ERR_WORKSPACE and enqueue nothing.
  *  - Every GPU that loads the library holds the 16 MiB array until the
  *    process exits.
- *  - The first call on a device looks up the array's device address
- *    (cudaGetSymbolAddress) with that device current; make that first call
- *    before any stream capture.  The address is kept for the life of the
- *    process: after cudaDeviceReset (or anything else that destroys the
- *    device's primary context) it is stale, so do not call this entry point
- *    on that device again in the same process.
+ *  - Every call looks up the array's device address (cudaGetSymbolAddress)
+ *    on the current device; nothing is cached, so the entry point stays
+ *    valid after cudaDeviceReset.  Make the first call on a device before
+ *    any stream capture (it may load the module).
  *  - Speed: the array holds the l x m scratch first and then whichever
  *    optional parts of mosaic_unmask still fit (digit planes of Q_d, tile
  *    images of the Q_i, line-offset copies of the S lists).  Beyond small

@@ -12,34 +12,23 @@
 // The array is a file-scope __device__ variable, so every GPU that loads the
 // library holds it (16 MiB) until the process exits.  Host code cannot use the
 // array's name as a device address (on the host it names a stand-in object),
-// so the first call on each device looks the address up with
-// cudaGetSymbolAddress while that device is current, and later calls reuse it.
-#include <mutex>
+// so every call looks the address up with cudaGetSymbolAddress on the current
+// device (cheap once the module is loaded).  Nothing is cached: after a device
+// or context reset the module reloads and the array may sit elsewhere.
 
 #include "mosaic_internal.cuh"
 
 namespace {
 
 constexpr int64_t kScratchWords = (int64_t)1 << 22;   // 16 MiB of uint32: l * m <= 2^22
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) uint32_t g_unmask_scratch[kScratchWords];
 
-std::mutex g_setup_mutex;
-void *g_scratch_addr[kMaxDevices];   // device address of g_unmask_scratch, per device ordinal
-
-// Device address of the scratch array on the current device (set up once per device).
+// Device address of the scratch array on the current device.
 mosaic_status scratch_address(void **out) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MOSAIC_ERR_CUDA;
-    std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (g_scratch_addr[dev] == nullptr) {
-        void *addr = nullptr;
-        if (cudaGetSymbolAddress(&addr, g_unmask_scratch) != cudaSuccess || addr == nullptr)
-            return MOSAIC_ERR_CUDA;
-        g_scratch_addr[dev] = addr;
-    }
-    *out = g_scratch_addr[dev];
+    void *addr = nullptr;
+    if (cudaGetSymbolAddress(&addr, g_unmask_scratch) != cudaSuccess || addr == nullptr) return MOSAIC_ERR_CUDA;
+    *out = addr;
     return MOSAIC_OK;
 }
 
