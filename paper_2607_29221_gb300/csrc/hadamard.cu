@@ -140,6 +140,47 @@ __device__ __forceinline__ void store_planes(uint16_t *p, int64_t plane_stride, 
     }
 }
 
+// Stages h = 32 .. 512 of a row held 32 values a thread, lane L of a warp
+// holding elements 32 L + e (e = 0 .. 31) of the warp's block of 1024.  The
+// warp transposes its 32 x 32 block through its own 4 KB of shared memory at
+// `wb` (16-byte aligned): lane L's values go to words [32 L, 32 L + 32) with
+// their 16-byte pieces XOR-permuted by L & 7, so the 16-byte stores and the
+// 4-byte loads back are conflict-free.  Lane L then holds elements 32 e + L,
+// and the five stages run between registers.  Each pair, its order and its
+// rounding are those of the shuffle form (lower p + q, upper p - q), so the
+// results are identical; 40 shared-memory instructions replace 160 shuffles.
+// Lane L writes only its own 32 words, so the caller's last reads of them need
+// no barrier; on return the warp has finished reading the block.
+__device__ __forceinline__ void warp_transpose_stages(float (&v)[32], uint32_t wb, int lane) {
+    const uint32_t l = (uint32_t)lane;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const uint32_t addr = wb + 4u * (32u * l + 4u * ((uint32_t)q ^ (l & 7u)));
+        asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v[4 * q]), "f"(v[4 * q + 1]),
+                     "f"(v[4 * q + 2]), "f"(v[4 * q + 3])
+                     : "memory");
+    }
+    __syncwarp();
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+        const uint32_t addr = wb + 4u * (32u * (uint32_t)e + 4u * ((l >> 2) ^ ((uint32_t)e & 7u)) + (l & 3u));
+        asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v[e]) : "r"(addr) : "memory");
+    }
+    __syncwarp();
+#pragma unroll
+    for (int h = 1; h < 32; h <<= 1) {
+#pragma unroll
+        for (int i = 0; i < 32; i += 2 * h) {
+#pragma unroll
+            for (int j = i; j < i + h; j++) {
+                const float p = v[j], q = v[j + h];
+                v[j] = __fadd_rn(p, q);
+                v[j + h] = __fsub_rn(p, q);
+            }
+        }
+    }
+}
+
 template <int E, int T>
 struct Cfg {
     static constexpr int N = E * T;
@@ -225,17 +266,25 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
                 }
             }
         }
-        // Phase 2: h = E .. 16E across lanes.
-        // The lower lane of a pair keeps v + o, the upper o - v: one fused
+        // Phase 2: h = E .. 16E across lanes.  With 32 values a thread (and a
+        // shared-memory row) the warp transposes its block in its own part of
+        // the row buffer, words [1056 w, 1056 w + 1024), which is where its
+        // phase-3 stores land, so no other warp touches them.  Otherwise: the
+        // lower lane of a pair keeps v + o, the upper o - v, one fused
         // multiply-add by +-1 (the product is exact, so the single rounding is
         // that of the plain sum or difference).
+        if constexpr (E == 32 && WN > 1) {
+            warp_transpose_stages(
+                v, (uint32_t)__cvta_generic_to_shared(smem + rb * C::SMEM_ROW + 1056 * (lt >> 5)), lane);
+        } else {
 #pragma unroll
-        for (int hl = 1; hl < 32; hl <<= 1) {
-            const float sgn = (lane & hl) ? -1.0f : 1.0f;
+            for (int hl = 1; hl < 32; hl <<= 1) {
+                const float sgn = (lane & hl) ? -1.0f : 1.0f;
 #pragma unroll
-            for (int e = 0; e < E; e++) {
-                const float o = __shfl_xor_sync(0xffffffffu, v[e], hl);
-                v[e] = __fmaf_rn(v[e], sgn, o);
+                for (int e = 0; e < E; e++) {
+                    const float o = __shfl_xor_sync(0xffffffffu, v[e], hl);
+                    v[e] = __fmaf_rn(v[e], sgn, o);
+                }
             }
         }
     }
@@ -245,8 +294,14 @@ __global__ void __launch_bounds__(T * Cfg<E, T>::RPB) fwht_kernel(FwhtArgs a) {
     // layout below is the same in both cases.
     if constexpr (WN > 1) {
         float *buf = smem + rb * C::SMEM_ROW;
+        if (E == 32 && a.rotate) {
+            // After the warp transpose v[e] is element 1024 w + 32 e + lane.
 #pragma unroll
-        for (int e = 0; e < E; e++) buf[pad_idx(base + e)] = v[e];
+            for (int e = 0; e < E; e++) buf[pad_idx(1024 * (lt >> 5) + 32 * e + lane)] = v[e];
+        } else {
+#pragma unroll
+            for (int e = 0; e < E; e++) buf[pad_idx(base + e)] = v[e];
+        }
         __syncthreads();
 #pragma unroll
         for (int j = 0; j < WN; j++)
@@ -426,6 +481,8 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
             tma_load_3d(reinterpret_cast<uint8_t *>(xbuf) + (size_t)c * C::BOX_CHUNKS * 128, &tmx, bar_x, 0,
                         c * C::BOX_CHUNKS, (int)row);
     };
+    // The sign bits of this thread's 32 values are the same for every row.
+    const uint32_t sign_w = (a.rotate && a.signs) ? a.signs[base >> 5] : 0u;
     int64_t row = blockIdx.x;
     if (lt == 0 && row < a.rows) issue_x(row);
     uint32_t ph = 0;
@@ -437,6 +494,10 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
         }
         __syncthreads();
         if (*abort_flag) break;
+        // The encode adds this row's mask words at the end: ask L2 for them now
+        // (lane L: the warp's 128-byte line of run L).
+        if (a.mode == 1 && a.mask)
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(a.mask + row * a.ldm + lane * 1024 + 32 * (lt >> 5)));
         // This thread's 32 values: chunk lt, 16-byte piece q at q ^ (lt & 7).
         float v[E];
         {
@@ -452,10 +513,9 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
         }
         if (a.rotate) {
             if (a.signs) {
-                const uint32_t w = a.signs[base >> 5] >> (base & 31);
 #pragma unroll
                 for (int e = 0; e < E; e++)
-                    if ((w >> e) & 1u) v[e] = -v[e];
+                    if ((sign_w >> e) & 1u) v[e] = -v[e];
             }
 #pragma unroll
             for (int h = 1; h < E; h <<= 1) {
@@ -469,19 +529,19 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
                     }
                 }
             }
-#pragma unroll
-            for (int hl = 1; hl < 32; hl <<= 1) {
-                const float sgn = (lane & hl) ? -1.0f : 1.0f;
-#pragma unroll
-                for (int e = 0; e < E; e++) {
-                    const float o = __shfl_xor_sync(0xffffffffu, v[e], hl);
-                    v[e] = __fmaf_rn(v[e], sgn, o);
-                }
-            }
+            // Stages h = 32 .. 512 through this warp's 4 KB of the input
+            // buffer, which only this warp has read.
+            warp_transpose_stages(v, smem_u32(xbuf) + 4096u * (uint32_t)(lt >> 5), lane);
         }
         __syncthreads();   // every thread has read the input buffer
+        if (a.rotate) {
+            // v[e] is element 1024 w + 32 e + lane after the warp transpose.
 #pragma unroll
-        for (int e = 0; e < E; e++) tbuf[pad_idx(base + e)] = v[e];
+            for (int e = 0; e < E; e++) tbuf[pad_idx(1024 * (lt >> 5) + 32 * e + lane)] = v[e];
+        } else {
+#pragma unroll
+            for (int e = 0; e < E; e++) tbuf[pad_idx(base + e)] = v[e];
+        }
         __syncthreads();
 #pragma unroll
         for (int j = 0; j < WN; j++)
@@ -670,6 +730,8 @@ __global__ void __launch_bounds__(kPairT, 2) fwht_pair_kernel(const __grid_const
             tma_load_3d(reinterpret_cast<uint8_t *>(xbuf) + (size_t)c * kPairBox * 128, &tmx, bar_x, 0,
                         c * kPairBox, (int)row);
     };
+    // The sign bits of this thread's 32 values are the same for every row.
+    const uint32_t sign_w = (a.rotate && a.signs) ? a.signs[base >> 5] : 0u;
     int64_t row = blockIdx.x;
     if (lt == 0 && row < a.rows) issue_x(row);
     uint32_t ph = 0;
@@ -681,6 +743,11 @@ __global__ void __launch_bounds__(kPairT, 2) fwht_pair_kernel(const __grid_const
         }
         __syncthreads();
         if (*abort_flag) break;
+        // The encode adds this row's mask words at the end: ask L2 for them now
+        // (lane L: line L & 1 of the warp's 256 bytes of run L / 2).
+        if (a.mode == 1 && a.mask)
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(a.mask + row * a.ldm + (lane >> 1) * 1024 + 64 * (lt >> 5) +
+                                                       32 * (lane & 1)));
         float v[E];
         {
             const uint32_t rb = smem_u32(xbuf) + (uint32_t)lt * 128u;
@@ -695,10 +762,9 @@ __global__ void __launch_bounds__(kPairT, 2) fwht_pair_kernel(const __grid_const
         }
         if (a.rotate) {
             if (a.signs) {
-                const uint32_t w = a.signs[base >> 5] >> (base & 31);
 #pragma unroll
                 for (int e = 0; e < E; e++)
-                    if ((w >> e) & 1u) v[e] = -v[e];
+                    if ((sign_w >> e) & 1u) v[e] = -v[e];
             }
 #pragma unroll
             for (int h = 1; h < E; h <<= 1) {
@@ -712,19 +778,19 @@ __global__ void __launch_bounds__(kPairT, 2) fwht_pair_kernel(const __grid_const
                     }
                 }
             }
-#pragma unroll
-            for (int hl = 1; hl < 32; hl <<= 1) {
-                const float sgn = (lane & hl) ? -1.0f : 1.0f;
-#pragma unroll
-                for (int e = 0; e < E; e++) {
-                    const float o = __shfl_xor_sync(0xffffffffu, v[e], hl);
-                    v[e] = __fmaf_rn(v[e], sgn, o);
-                }
-            }
+            // Stages h = 32 .. 512 through this warp's 4 KB of the input
+            // buffer, which only this warp has read.
+            warp_transpose_stages(v, smem_u32(xbuf) + 4096u * (uint32_t)(lt >> 5), lane);
         }
         __syncthreads();   // every thread has read the input buffer
+        if (a.rotate) {
+            // v[e] is element 1024 w + 32 e + lane after the warp transpose.
 #pragma unroll
-        for (int e = 0; e < E; e++) xbuf[pad_idx(base + e)] = v[e];
+            for (int e = 0; e < E; e++) xbuf[pad_idx(1024 * (lt >> 5) + 32 * e + lane)] = v[e];
+        } else {
+#pragma unroll
+            for (int e = 0; e < E; e++) xbuf[pad_idx(base + e)] = v[e];
+        }
         __syncthreads();
 #pragma unroll
         for (int j = 0; j < WN; j++)
