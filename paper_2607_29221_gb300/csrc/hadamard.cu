@@ -140,18 +140,15 @@ __device__ __forceinline__ void store_planes(uint16_t *p, int64_t plane_stride, 
     }
 }
 
-// Stages h = 32 .. 512 of a row held 32 values a thread, lane L of a warp
-// holding elements 32 L + e (e = 0 .. 31) of the warp's block of 1024.  The
-// warp transposes its 32 x 32 block through its own 4 KB of shared memory at
-// `wb` (16-byte aligned): lane L's values go to words [32 L, 32 L + 32) with
-// their 16-byte pieces XOR-permuted by L & 7, so the 16-byte stores and the
-// 4-byte loads back are conflict-free.  Lane L then holds elements 32 e + L,
-// and the five stages run between registers.  Each pair, its order and its
-// rounding are those of the shuffle form (lower p + q, upper p - q), so the
-// results are identical; 40 shared-memory instructions replace 160 shuffles.
-// Lane L writes only its own 32 words, so the caller's last reads of them need
-// no barrier; on return the warp has finished reading the block.
-__device__ __forceinline__ void warp_transpose_stages(float (&v)[32], uint32_t wb, int lane) {
+// A row held 32 values a thread, lane L of a warp holding elements 32 L + e
+// (e = 0 .. 31) of the warp's block of 1024: the warp transposes its 32 x 32
+// block through its own 4 KB of shared memory at `wb` (16-byte aligned):
+// lane L's values go to words [32 L, 32 L + 32) with their 16-byte pieces
+// XOR-permuted by L & 7, so the 16-byte stores and the 4-byte loads back are
+// conflict-free.  On return lane L holds elements 32 e + L, and the warp has
+// finished reading the block.  Lane L writes only its own 32 words, so the
+// caller's last reads of them need no barrier.
+__device__ __forceinline__ void warp_transpose32(float (&v)[32], uint32_t wb, int lane) {
     const uint32_t l = (uint32_t)lane;
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
@@ -167,6 +164,12 @@ __device__ __forceinline__ void warp_transpose_stages(float (&v)[32], uint32_t w
         asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v[e]) : "r"(addr) : "memory");
     }
     __syncwarp();
+}
+// Stages h = 32 .. 512 between the registers of the transposed block (v[e] =
+// element 32 e + L).  Each pair, its order and its rounding are those of the
+// shuffle form (lower p + q, upper p - q), so the results are identical; with
+// the transpose, 40 shared-memory instructions replace 160 shuffles.
+__device__ __forceinline__ void reg_stages32(float (&v)[32]) {
 #pragma unroll
     for (int h = 1; h < 32; h <<= 1) {
 #pragma unroll
@@ -179,6 +182,10 @@ __device__ __forceinline__ void warp_transpose_stages(float (&v)[32], uint32_t w
             }
         }
     }
+}
+__device__ __forceinline__ void warp_transpose_stages(float (&v)[32], uint32_t wb, int lane) {
+    warp_transpose32(v, wb, lane);
+    reg_stages32(v);
 }
 
 template <int E, int T>
@@ -910,6 +917,243 @@ mosaic_status launch_pair(const FwhtArgs &a, cudaStream_t st) {
 }
 
 // ---------------------------------------------------------------------------
+// Rotation alone (mosaic_hadamard) of rows of 16384 and 32768 whose length n
+// is a multiple of 32.  Without the encode's long per-row tail (quantise, mask
+// words, digit planes) to hide it, the copy of a block's next row has to start
+// early: these kernels refill the input buffer in two halves, each on its own
+// barrier, the first as soon as every thread has read the row and the second
+// once phase 2 is done, and run the exchange between warps for phase 3 in a
+// buffer of its own (R, plus P for 32768).  Warps whose part of the input
+// buffer is being refilled transpose their blocks for phase 2 in R instead.
+// Rows arrive as for the kernels above (the 3-D {32 values, chunks, rows} view
+// with the 128-byte swizzle); stage order and roundings are those of
+// fwht_kernel, so the results are identical.  The TMA waits are bounded (abort
+// flag + g_fwht_error).
+//
+// 16384 (two 512-thread CTAs per SM, 64 registers): phase 3 holds
+// v[2 j + u] = element 1024 j + 512 u + t (t the thread), i.e. register
+// 16 u + w of warp j, same lane, so the exchange runs through R (32 KB) in two
+// rounds, one per half of the registers, and no thread holds more than 32
+// values.
+// 32768 (one 1024-thread CTA per SM): phase 3 holds v[j] = element
+// 1024 j + t, register w of warp j, same lane; in round 0 every warp stores
+// v[0..15] in R (64 KB) and warps 0-15 park v[16..31] in P (32 KB) before
+// reading their 32 values from R; in round 1 warps 16-31 store v[16..31] in R
+// and read theirs from R and P.
+// ---------------------------------------------------------------------------
+constexpr int kRotRowBox = 256;   // chunks of 32 values per TMA box (32 KB)
+
+template <int T>
+struct RotCfg {
+    static_assert(T == 512 || T == 1024, "rows of 16384 or 32768");
+    static constexpr int E = 32;
+    static constexpr int N = E * T;
+    static constexpr int WN = T / 32;
+    static constexpr int BOXES = N / 32 / kRotRowBox;        // 2 or 4, half of them per half-row copy
+    static constexpr size_t XBUF = (size_t)N * 4;            // the row as it lands
+    static constexpr size_t RBUF = (size_t)N / 2 * 4;        // R: 16 registers x WN warps x 32 lanes
+    static constexpr size_t PBUF = T == 1024 ? (size_t)N / 4 * 4 : 0;   // P: 16 registers x 16 warps x 32 lanes
+    static constexpr size_t SMEM = 1024 + XBUF + RBUF + PBUF + 64;
+};
+
+template <int T>
+__global__ void __launch_bounds__(T, T == 512 ? 2 : 1) rot_kernel(const __grid_constant__ CUtensorMap tmx, FwhtArgs a) {
+    using C = RotCfg<T>;
+    constexpr int E = C::E, N = C::N, WN = C::WN;
+    extern __shared__ uint8_t raw[];
+    uint8_t *base_ptr = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~(uintptr_t)1023);
+    float *xbuf = reinterpret_cast<float *>(base_ptr);
+    float *rbuf = reinterpret_cast<float *>(base_ptr + C::XBUF);
+    float *pbuf = reinterpret_cast<float *>(base_ptr + C::XBUF + C::RBUF);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(base_ptr + C::XBUF + C::RBUF + C::PBUF);   // one per half
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar + 2);
+
+    const int lt = threadIdx.x, lane = lt & 31, w = lt >> 5;
+    const int base = lt * E;
+    if (lt == 0) {
+        mbar_init(&bar[0], 1);
+        mbar_init(&bar[1], 1);
+        *abort_flag = 0;
+        mbar_init_fence();
+    }
+    __syncthreads();
+    // Half h of row `row`: boxes [h BOXES / 2, (h + 1) BOXES / 2).
+    auto issue_half = [&](int64_t row, int h) {
+        mbar_expect_tx(&bar[h], (uint32_t)(N * 2));
+#pragma unroll
+        for (int c = h * (C::BOXES / 2); c < (h + 1) * (C::BOXES / 2); ++c)
+            tma_load_3d(reinterpret_cast<uint8_t *>(xbuf) + (size_t)c * kRotRowBox * 128, &tmx, &bar[h], 0,
+                        c * kRotRowBox, (int)row);
+    };
+    // The sign bits of this thread's 32 values are the same for every row.
+    const uint32_t sign_w = (a.rotate && a.signs) ? a.signs[base >> 5] : 0u;
+    // This warp's 4 KB for its block transpose: R for the warps of the lower
+    // half (refilled first), its own part of the upper half of the input
+    // buffer for the others.
+    const uint32_t wb = w < WN / 2 ? smem_u32(rbuf) + 4096u * (uint32_t)w : smem_u32(xbuf) + 4096u * (uint32_t)w;
+    int64_t row = blockIdx.x;
+    if (lt == 0 && row < a.rows) {
+        issue_half(row, 0);
+        issue_half(row, 1);
+    }
+    uint32_t ph = 0;
+    for (; row < a.rows; row += gridDim.x, ph ^= 1u) {
+        const int64_t next = row + gridDim.x;
+        if (!mbar_wait(&bar[0], ph, abort_flag) || !mbar_wait(&bar[1], ph, abort_flag)) {
+            *abort_flag = 1;
+            atomicExch(&g_fwht_error, 1u);
+        }
+        __syncthreads();
+        if (*abort_flag) break;
+        // This thread's 32 values: chunk lt, 16-byte piece q at q ^ (lt & 7).
+        float v[E];
+        {
+            const uint32_t rb = smem_u32(xbuf) + (uint32_t)lt * 128u;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const uint32_t addr = rb + (uint32_t)((q ^ (lt & 7)) * 16);
+                asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                             : "=f"(v[4 * q]), "=f"(v[4 * q + 1]), "=f"(v[4 * q + 2]), "=f"(v[4 * q + 3])
+                             : "r"(addr)
+                             : "memory");
+            }
+        }
+        __syncthreads();   // every thread has read the row
+        if (lt == 0 && next < a.rows) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            issue_half(next, 0);
+        }
+        if (a.rotate) {
+            if (a.signs) {
+#pragma unroll
+                for (int e = 0; e < E; e++)
+                    if ((sign_w >> e) & 1u) v[e] = -v[e];
+            }
+#pragma unroll
+            for (int h = 1; h < E; h <<= 1) {
+#pragma unroll
+                for (int i = 0; i < E; i += 2 * h) {
+#pragma unroll
+                    for (int j = i; j < i + h; j++) {
+                        const float p = v[j], q = v[j + h];
+                        v[j] = __fadd_rn(p, q);
+                        v[j + h] = __fsub_rn(p, q);
+                    }
+                }
+            }
+        }
+        // v[e] becomes element 1024 w + 32 e + lane (with or without rotation,
+        // so that the layout below is the same), then stages h = 32 .. 512.
+        warp_transpose32(v, wb, lane);
+        if (a.rotate) reg_stages32(v);
+        __syncthreads();   // R and the upper half of the input buffer are free
+        if (lt == 0 && next < a.rows) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            issue_half(next, 1);
+        }
+        if constexpr (T == 512) {
+            float t[E];
+            // R word (e * 16 + warp) * 32 + lane holds register 16 u + e in
+            // round u; thread (w, lane) reads its 16 values of round u at e = w.
+#pragma unroll
+            for (int e = 0; e < 16; e++) rbuf[(e * 16 + w) * 32 + lane] = v[e];
+            __syncthreads();
+#pragma unroll
+            for (int j = 0; j < WN; j++) t[2 * j] = rbuf[(w * 16 + j) * 32 + lane];
+            __syncthreads();
+#pragma unroll
+            for (int e = 0; e < 16; e++) rbuf[(e * 16 + w) * 32 + lane] = v[16 + e];
+            __syncthreads();
+#pragma unroll
+            for (int j = 0; j < WN; j++) t[2 * j + 1] = rbuf[(w * 16 + j) * 32 + lane];
+#pragma unroll
+            for (int e = 0; e < E; e++) v[e] = t[e];
+        } else {
+            // R word (e * 32 + warp) * 32 + lane holds register 16 r + e of
+            // round r; P word (e * 16 + warp) * 32 + lane register 16 + e of
+            // warps 0-15.
+#pragma unroll
+            for (int e = 0; e < 16; e++) rbuf[(e * 32 + w) * 32 + lane] = v[e];
+            if (w < 16) {
+#pragma unroll
+                for (int e = 0; e < 16; e++) pbuf[(e * 16 + w) * 32 + lane] = v[16 + e];
+            }
+            __syncthreads();
+            if (w < 16) {
+#pragma unroll
+                for (int j = 0; j < WN; j++) v[j] = rbuf[(w * 32 + j) * 32 + lane];
+            }
+            __syncthreads();
+            if (w >= 16) {
+#pragma unroll
+                for (int e = 0; e < 16; e++) rbuf[(e * 32 + w) * 32 + lane] = v[16 + e];
+            }
+            __syncthreads();
+            if (w >= 16) {
+#pragma unroll
+                for (int j = 0; j < 16; j++) v[j] = pbuf[((w - 16) * 16 + j) * 32 + lane];
+#pragma unroll
+                for (int j = 16; j < WN; j++) v[j] = rbuf[((w - 16) * 32 + j) * 32 + lane];
+            }
+        }
+        // Phase 3 (h = 1024 .. N / 2): v[U j + u] is element 1024 j + 512 u + lt
+        // (U = 2 for 16384; U = 1, u = 0 for 32768).
+        constexpr int U = E / WN;
+        if (a.rotate) {
+#pragma unroll
+            for (int hj = 1; hj < WN; hj <<= 1) {
+#pragma unroll
+                for (int i = 0; i < WN; i += 2 * hj) {
+#pragma unroll
+                    for (int j = i; j < i + hj; j++) {
+#pragma unroll
+                        for (int u = 0; u < U; u++) {
+                            const float p = v[U * j + u], q = v[U * (j + hj) + u];
+                            v[U * j + u] = __fadd_rn(p, q);
+                            v[U * (j + hj) + u] = __fsub_rn(p, q);
+                        }
+                    }
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < E; e++) v[e] = __fmul_rn(v[e], a.inv_sqrt);
+        }
+        // v[e] is element T e + lt.
+        float *yr = a.y + row * a.ldy;
+#pragma unroll
+        for (int e = 0; e < E; e++) yr[T * e + lt] = v[e];
+    }
+    // After a normal exit every issued copy has been waited for; after an
+    // expired wait, let the copies still in flight land (bounded) first.
+    if (lt == 0 && *abort_flag) {
+        mbar_drain(&bar[0], ph);
+        mbar_drain(&bar[1], ph);
+    }
+    __syncthreads();
+}
+
+template <int T>
+mosaic_status launch_rot(const FwhtArgs &a, cudaStream_t st) {
+    using C = RotCfg<T>;
+    CUtensorMap tmx;
+    if (!make_chunk_map(&tmx, a.x, a.n, a.rows, a.ldx, true)) return MOSAIC_ERR_CUDA;
+    static std::atomic<unsigned long long> attr_set{0};
+    int dev = 0, sms = 0, per_sm = 0;
+    if (!ensure_smem_limit(attr_set, rot_kernel<T>, C::SMEM, &dev) ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1 ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rot_kernel<T>, T, C::SMEM) != cudaSuccess ||
+        per_sm < 1)
+        return MOSAIC_ERR_CUDA;
+    const int64_t slots = (int64_t)sms * per_sm;
+    const int64_t grid = a.rows < slots ? a.rows : slots;
+    {
+        KernelSpan span("fwht_rot", st);
+        rot_kernel<T><<<(unsigned)grid, T, C::SMEM, st>>>(tmx, a);
+    }
+    return launch_status();
+}
+
+// ---------------------------------------------------------------------------
 // Rows of 65536: the first 15 stages (h = 1 .. 16384) run on the two halves
 // as rows of 32768 (split mode, unscaled, into y or into `out` used as fp32
 // scratch); the last stage h = 32768 pairs the halves elementwise here, then
@@ -1056,8 +1300,12 @@ mosaic_status fwht_encode(const float *x, int64_t ldx, int64_t rows, int64_t n, 
         case 2048: return launch<16, 128>(a, st);
         case 4096: return launch<16, 256>(a, st);
         case 8192: return launch<32, 256>(a, st);
-        case 16384: return stream_ok(a) ? launch_pair(a, st) : launch<32, 512>(a, st);
-        case 32768: return stream_ok(a) ? launch_stream<1024>(a, st) : launch<32, 1024>(a, st);
+        case 16384:
+            if (!stream_ok(a)) return launch<32, 512>(a, st);
+            return a.mode == 0 ? launch_rot<512>(a, st) : launch_pair(a, st);
+        case 32768:
+            if (!stream_ok(a)) return launch<32, 1024>(a, st);
+            return a.mode == 0 ? launch_rot<1024>(a, st) : launch_stream<1024>(a, st);
         default: return MOSAIC_ERR_SHAPE;
     }
 }
