@@ -254,9 +254,12 @@ struct SparseLevel {
     const uint32_t *tiled = nullptr;   // tile images of src's segment (build_tile_image), or null
     int lines = 0;                     // idx holds pg_line(position) (lists drawn for the tiled gather)
 };
-// Line offset of position p in a staged tile of the tiled gather: 128-byte
-// line p, the permutation bits ((p >> 2) & 7) in the 16-byte chunk field.
-__host__ __device__ __forceinline__ uint32_t pg_line(uint32_t p) { return (p << 7) + ((p << 2) & 0x70u); }
+// Chunk permutation of line p in a staged tile of the tiled gather: rows
+// 4c .. 4c+3 sit in 16-byte chunk c ^ pg_perm(p), an even number.
+__host__ __device__ __forceinline__ uint32_t pg_perm(uint32_t p) { return ((p >> 2) & 3u) << 1; }
+// Line offset of position p in a staged tile: 128-byte line p, the
+// permutation bits in the 16-byte chunk field.
+__host__ __device__ __forceinline__ uint32_t pg_line(uint32_t p) { return (p << 7) + (pg_perm(p) << 4); }
 // True when the tiled gather takes lists of weight t over segments of r words
 // staged in g_count rows (16-byte aligned lists assumed).
 bool pgather_takes(int64_t g_count, uint32_t r, int t);

@@ -197,45 +197,47 @@ __global__ void __launch_bounds__(GW * 32) gather_kernel(GatherArgs a) {
 //
 // A tile is 32 rows g of the level's segment, staged TRANSPOSED: the 32 rows'
 // words at position p form one 128-byte line (line p at byte 128 p), whose
-// eight 16-byte chunks are XOR-permuted by (p >> 2) & 7: rows 4c .. 4c+3 sit
-// in chunk c ^ ((p >> 2) & 7).  A warp serves four list entities at a time,
-// eight lanes each; lane i of an entity reads rows 4i .. 4i+3 at position p
-// with one 16-byte load, so the eight lanes of an entity read one whole line
-// (all 32 banks) and every 16-byte access phase is conflict-free.
+// eight 16-byte chunks are XOR-permuted by f(p) = 2 ((p >> 2) & 3), an even
+// number: rows 4c .. 4c+3 sit in chunk c ^ f(p).  A warp serves eight list
+// entities at a time, four lanes each; lane i of an entity owns rows
+// 8i .. 8i+7 (chunks 2i and 2i+1) and reads them at position p with two
+// 16-byte loads.  The even entities of a warp read their even chunk first and
+// the odd ones their odd chunk, and f(p) keeps a chunk's parity, so in each
+// 16-byte access phase (two entities, eight lanes) the two entities' four
+// chunks fall in distinct halves of the 32 banks whatever their positions:
+// every load is conflict-free.  Each lane accumulates the two loads apart and
+// puts the rows back in order when it writes the unit out.
 // Staging: a warp loads 4 rows x 32 positions (four 128-byte segments, one
-// 16-byte load a lane) and each of its four 4-byte stores hits 32 distinct
-// banks thanks to the permutation.
-// The (position, value) lists stream through a per-warp ring in rounds of
-// 16 pairs (cp.async one or two rounds ahead, zero-filled past the end of a
-// list).  Lists already given as line addresses (`lines`: drawn that way, or
-// converted once per call) are used as they are; otherwise, once a round has
-// landed, each lane rewrites two of its entity's positions into line
-// addresses with the permutation bits in place (clamping positions of caller
-// lists to r - 1), so that the gather loop needs one XOR per pair.  Work
-// units are (tile, 64 entities), numbered tile-major and split evenly over a
-// persistent grid, so a CTA stages each of its one or two tiles once; with a
-// second job (`two`: another source and output on the same lists) its units
-// follow the first job's.  Each unit's a - b operands are loaded when it
-// starts and its outputs written when its last round is done (16-byte
+// 16-byte load a lane) and stores each word in its line.
+// The (position, value) lists stream through a per-warp ring of two slots in
+// rounds of 16 pairs (cp.async one round ahead, zero-filled past the end of a
+// list).  A slot holds the round's positions then its values, quad q of
+// entity e at word 32 q + 4 e, so one 16-byte load of quad q serves all eight
+// entities from the 32 banks at once.  Lists already given as line addresses
+// (`lines`: drawn that way, or converted once per call) are used as they
+// are; otherwise, once a round has landed, each lane rewrites four positions
+// into line addresses with the permutation bits in place (clamping positions
+// of caller lists to r - 1), so that the gather loop needs one XOR per load.
+// Work units are (tile, 128 entities), numbered tile-major and split evenly
+// over a persistent grid, so a CTA stages each of its one or two tiles once;
+// with a second job (`two`: another source and output on the same lists) its
+// units follow the first job's.  Each unit's a - b operands are loaded when it
+// starts and its outputs written when its last round is done (32-byte
 // accesses where the output rows are the list entities and the layout
-// allows).
+// allows; eight consecutive entities, 32 bytes, per output row otherwise).
 // ---------------------------------------------------------------------------
 constexpr int kPgRows = 32;
 constexpr int kPgWarps = 16;
-constexpr int kPgEnts = 4 * kPgWarps;       // entities per unit
-constexpr int kPgSlot = 4 * 36;             // words per ring slot: 4 entities x (16 idx + 16 val + 4 pad)
-constexpr uint32_t kPgMaxR = 1568;          // stage + three-slot rings + barrier + alignment within 227 KB
-
-// Ring slots per warp: three (lists two rounds ahead) where the outputs are
-// rows of the list entities; two where they are columns, whose scattered
-// a / b reads gain more from the L1 space left beside shared memory.
-template <bool LIST_IS_COL>
-__host__ __device__ constexpr int pg_ring() { return LIST_IS_COL ? 2 : 3; }
+constexpr int kPgEPW = 8;                   // entities per warp
+constexpr int kPgEnts = kPgEPW * kPgWarps;  // entities per unit
+constexpr int kPgRing = 2;                  // ring slots per warp
+constexpr int kPgSlot = 2 * 16 * kPgEPW;    // words per ring slot: 16 positions + 16 values per entity
+constexpr uint32_t kPgMaxR = 1536;          // stage + rings + barrier + alignment within 227 KB
 
 // Stage, rings, the staging barrier and abort flag (16 bytes), + 128 bytes
 // to align the stage to a line.
-size_t pgather_smem(uint32_t r, int ring) {
-    return (size_t)((r + 31) / 32 * 32) * kPgRows * 4 + (size_t)kPgWarps * ring * kPgSlot * 4 + 16 + 128;
+size_t pgather_smem(uint32_t r) {
+    return (size_t)((r + 31) / 32 * 32) * kPgRows * 4 + (size_t)kPgWarps * kPgRing * kPgSlot * 4 + 16 + 128;
 }
 
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
@@ -249,16 +251,19 @@ __device__ __forceinline__ uint4 lds128(uint32_t addr) {
 __device__ __forceinline__ void sts32(uint32_t addr, uint32_t v) {
     asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
 }
+__device__ __forceinline__ void sts128(uint32_t addr, uint4 v) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
 
 constexpr int kPgStageBatch = 12;  // 16-byte loads a lane keeps in flight while staging
 
 template <bool LIST_IS_COL, bool CLAMP>
 __global__ void __launch_bounds__(kPgWarps * 32, 1)
     pgather_kernel(GatherArgs a, int units, int units0, int chunks, int vec_src, int vec_ab) {
-    constexpr int kPgRing = pg_ring<LIST_IS_COL>();
     extern __shared__ __align__(16) uint32_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int grp = lane >> 3, li = lane & 7;
+    const int grp = lane >> 2, li = lane & 3;
     const int r = (int)a.r, rp = (r + 31) / 32 * 32, t = a.t;
     const uint32_t sm_base = ((uint32_t)__cvta_generic_to_shared(sm) + 127u) & ~127u;
     const uint32_t ring_base = sm_base + 4u * (uint32_t)(rp * kPgRows + warp * (kPgRing * kPgSlot));
@@ -277,22 +282,30 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
     const int R = (t + 15) >> 4;
     const int steps = (u_end - u_begin) * R;
     const uint32_t rlast = a.r - 1;
-    const uint32_t lane_chunk = 16u * (uint32_t)li;   // rows 4 li .. 4 li + 3 of a line, before permutation
+    // Byte offsets of this lane's two chunks in a line, in load order (before
+    // the permutation): chunk 2 li + par first, par = 1 for the odd entities.
+    const int par = grp & 1;
+    const uint32_t chunk0 = 16u * (uint32_t)(2 * li + par);
+    const uint32_t chunk1 = 16u * (uint32_t)(2 * li + (par ^ 1));
 
-    // List rounds: lane (grp, li) copies 16 bytes of round rr of entity
-    // (chunk, warp, grp): positions 4 li .. (li < 4) or values 4 (li - 4) ..
-    const uint32_t *lbase = li < 4 ? a.idx : a.val;
-    const int qoff = (li & 3) * 4;
-    const uint32_t st_off = 4u * (uint32_t)(grp * 36 + (li < 4 ? 0 : 16) + qoff);
+    // List rounds: lane (grp, li) copies quad li of round rr of entity
+    // (chunk, warp, grp), positions and values, to slot words 32 li + 4 grp
+    // and 128 + 32 li + 4 grp.
+    const uint32_t st_idx = 4u * (uint32_t)(li * 32 + grp * 4);
+    const uint32_t st_val = st_idx + 4u * 128u;
     int i_chunk = u_begin % chunks, i_rr = 0, i_s = 0;
     auto issue = [&]() {
         if (i_s < steps) {
-            const int64_t e = (int64_t)i_chunk * kPgEnts + warp * 4 + grp;
-            const int q = i_rr * 16 + qoff;
+            const int64_t e = (int64_t)i_chunk * kPgEnts + warp * kPgEPW + grp;
+            const int q = i_rr * 16 + li * 4;
             const bool ok = e < a.nlist && q < t;
-            const uint32_t dst = ring_base + 4u * (uint32_t)((i_s % kPgRing) * kPgSlot) + st_off;
-            asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst),
-                         "l"(lbase + (ok ? e * t + q : 0)), "r"(ok ? 16 : 0)
+            const int64_t off = ok ? e * t + q : 0;
+            const uint32_t dst = ring_base + 4u * (uint32_t)((i_s % kPgRing) * kPgSlot);
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst + st_idx), "l"(a.idx + off),
+                         "r"(ok ? 16 : 0)
+                         : "memory");
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst + st_val), "l"(a.val + off),
+                         "r"(ok ? 16 : 0)
                          : "memory");
             if (++i_rr == R) {
                 i_rr = 0;
@@ -305,9 +318,8 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
 
     // Transposed, permuted copy of rows tile*32 .. +31 (zeros past the ends).
     // Lane (gl, pq) of a warp loads words p .. p+3 (p = 32 b + 4 pq) of row
-    // 4 j + gl and stores word p+k in line p+k, chunk j ^ (((p+k) >> 2) & 7):
-    // for each k the 32 stores fall in 32 distinct banks.  Each lane keeps
-    // kPgStageBatch 16-byte loads in flight.
+    // 4 j + gl and stores word p+k in line p+k, chunk j ^ f(p+k).  Each lane
+    // keeps kPgStageBatch 16-byte loads in flight.
     // Tile images (a.tiled) hold exactly this layout: one bulk copy per 32 KB,
     // all threads wait (bounded) for the barrier.  Returns false if the copy
     // did not land in time (error word raised).
@@ -363,7 +375,7 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
 #pragma unroll
                     for (int k = 0; k < 4; k++) {
                         const uint32_t pp = (uint32_t)(p + k);
-                        sts32(sm_base + (pp << 7) + ((((uint32_t)g >> 2) ^ (pp >> 2)) & 7u) * 16u +
+                        sts32(sm_base + (pp << 7) + ((((uint32_t)g >> 2) ^ pg_perm(pp)) & 7u) * 16u +
                                   4u * (uint32_t)(g & 3),
                               v[k]);
                     }
@@ -397,27 +409,30 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
                 break;
             }
         }
-        const int64_t e = (int64_t)chunk * kPgEnts + warp * 4 + grp;
-        const int64_t g = tile * kPgRows + li * 4;
+        const int64_t e = (int64_t)chunk * kPgEnts + warp * kPgEPW + grp;
+        const int64_t g = tile * kPgRows + li * 8;
         const bool e_ok = e < a.nlist;
-        // a - b of the unit's outputs: row e, columns g .. g+3 (or the transpose).
-        const bool vec = vec_ab && !LIST_IS_COL && g + 4 <= g_count;
+        // a - b of the unit's outputs: row e, columns g .. g+7 (or the transpose).
+        const bool vec = vec_ab && !LIST_IS_COL && g + 8 <= g_count;
         const uint32_t *ja = j1 ? a.a2 : a.a;
         const int64_t jlda = j1 ? a.lda2 : a.lda;
-        uint32_t ab[4] = {0u, 0u, 0u, 0u};
+        uint32_t ab[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
         if (e_ok) {
             if (vec) {
-                if (ja) {
-                    const uint4 x = __ldg(reinterpret_cast<const uint4 *>(ja + e * jlda + g));
-                    ab[0] = x.x; ab[1] = x.y; ab[2] = x.z; ab[3] = x.w;
-                }
-                if (a.b) {
-                    const uint4 x = __ldg(reinterpret_cast<const uint4 *>(a.b + e * a.ldb + g));
-                    ab[0] -= x.x; ab[1] -= x.y; ab[2] -= x.z; ab[3] -= x.w;
+#pragma unroll
+                for (int h = 0; h < 2; h++) {
+                    if (ja) {
+                        const uint4 x = __ldg(reinterpret_cast<const uint4 *>(ja + e * jlda + g + 4 * h));
+                        ab[4 * h] = x.x; ab[4 * h + 1] = x.y; ab[4 * h + 2] = x.z; ab[4 * h + 3] = x.w;
+                    }
+                    if (a.b) {
+                        const uint4 x = __ldg(reinterpret_cast<const uint4 *>(a.b + e * a.ldb + g + 4 * h));
+                        ab[4 * h] -= x.x; ab[4 * h + 1] -= x.y; ab[4 * h + 2] -= x.z; ab[4 * h + 3] -= x.w;
+                    }
                 }
             } else {
 #pragma unroll
-                for (int c = 0; c < 4; c++) {
+                for (int c = 0; c < 8; c++) {
                     if (g + c >= g_count) break;
                     const int64_t row = LIST_IS_COL ? g + c : e;
                     const int64_t col = LIST_IS_COL ? e : g + c;
@@ -428,54 +443,62 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
                 }
             }
         }
-        uint32_t acc0 = 0u, acc1 = 0u, acc2 = 0u, acc3 = 0u;
+        // x*: the rows of the first load (chunk 2 li + par), y*: of the second.
+        uint32_t x0 = 0u, x1 = 0u, x2 = 0u, x3 = 0u, y0 = 0u, y1 = 0u, y2 = 0u, y3 = 0u;
         for (int rr = 0; rr < R; rr++, s++) {
             issue();
             asm volatile("cp.async.wait_group %0;" ::"n"(kPgRing - 1) : "memory");
             __syncwarp();
-            const uint32_t slot = ring_base + 4u * (uint32_t)((s % kPgRing) * kPgSlot + grp * 36);
+            const uint32_t slot = ring_base + 4u * (uint32_t)((s % kPgRing) * kPgSlot);
             if (!a.lines) {
-                // Positions 2 li, 2 li + 1 of the round -> line offset | permutation bits.
-                uint32_t p0, p1;
-                asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(p0), "=r"(p1) : "r"(slot + 8u * li) : "memory");
+                // Positions 4 lane .. 4 lane + 3 of the round -> line offset | permutation bits.
+                uint4 P = lds128(slot + 16u * (uint32_t)lane);
                 if (CLAMP) {
-                    p0 = min(p0, rlast);
-                    p1 = min(p1, rlast);
+                    P.x = min(P.x, rlast);
+                    P.y = min(P.y, rlast);
+                    P.z = min(P.z, rlast);
+                    P.w = min(P.w, rlast);
                 }
-                p0 = pg_line(p0);
-                p1 = pg_line(p1);
-                asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(slot + 8u * li), "r"(p0), "r"(p1) : "memory");
+                sts128(slot + 16u * (uint32_t)lane, make_uint4(pg_line(P.x), pg_line(P.y), pg_line(P.z), pg_line(P.w)));
                 __syncwarp();
             }
 #pragma unroll
-            for (int u4 = 0; u4 < 4; u4++) {
-                const uint4 I = lds128(slot + 16u * u4);
-                const uint4 V = lds128(slot + 64u + 16u * u4);
+            for (int q = 0; q < 4; q++) {
+                const uint4 I = lds128(slot + 4u * (uint32_t)(q * 32 + grp * 4));
+                const uint4 V = lds128(slot + 4u * (uint32_t)(128 + q * 32 + grp * 4));
                 const uint32_t pi[4] = {I.x, I.y, I.z, I.w};
                 const uint32_t vi[4] = {V.x, V.y, V.z, V.w};
 #pragma unroll
                 for (int c = 0; c < 4; c++) {
-                    const uint4 x = lds128(sm_base + (pi[c] ^ lane_chunk));
-                    acc0 += vi[c] * x.x;
-                    acc1 += vi[c] * x.y;
-                    acc2 += vi[c] * x.z;
-                    acc3 += vi[c] * x.w;
+                    const uint4 dx = lds128(sm_base + (pi[c] ^ chunk0));
+                    const uint4 dy = lds128(sm_base + (pi[c] ^ chunk1));
+                    x0 += vi[c] * dx.x;
+                    x1 += vi[c] * dx.y;
+                    x2 += vi[c] * dx.z;
+                    x3 += vi[c] * dx.w;
+                    y0 += vi[c] * dy.x;
+                    y1 += vi[c] * dy.y;
+                    y2 += vi[c] * dy.z;
+                    y3 += vi[c] * dy.w;
                 }
             }
             __syncwarp();
         }
         if (e_ok) {
-            const uint32_t acc[4] = {acc0, acc1, acc2, acc3};
-            uint32_t res[4];
+            // Rows g .. g+3 come from the even chunk, g+4 .. g+7 from the odd one.
+            const uint32_t acc[8] = {par ? y0 : x0, par ? y1 : x1, par ? y2 : x2, par ? y3 : x3,
+                                     par ? x0 : y0, par ? x1 : y1, par ? x2 : y2, par ? x3 : y3};
+            uint32_t res[8];
 #pragma unroll
-            for (int c = 0; c < 4; c++) res[c] = (a.sgn >= 0 ? acc[c] : 0u - acc[c]) + ab[c];
+            for (int c = 0; c < 8; c++) res[c] = (a.sgn >= 0 ? acc[c] : 0u - acc[c]) + ab[c];
             uint32_t *jout = j1 ? a.out2 : a.out;
             const int64_t jldo = j1 ? a.ldo2 : a.ldo;
             if (vec && jout && !a.decode) {
                 *reinterpret_cast<uint4 *>(jout + e * jldo + g) = make_uint4(res[0], res[1], res[2], res[3]);
+                *reinterpret_cast<uint4 *>(jout + e * jldo + g + 4) = make_uint4(res[4], res[5], res[6], res[7]);
             } else {
 #pragma unroll
-                for (int c = 0; c < 4; c++) {
+                for (int c = 0; c < 8; c++) {
                     if (g + c >= g_count) break;
                     const int64_t row = LIST_IS_COL ? g + c : e;
                     const int64_t col = LIST_IS_COL ? e : g + c;
@@ -498,7 +521,7 @@ __global__ void __launch_bounds__(kPgWarps * 32, 1)
 
 template <bool LIST_IS_COL, bool CLAMP>
 mosaic_status launch_pgather(const GatherArgs &a, cudaStream_t st) {
-    const size_t smem = pgather_smem(a.r, pg_ring<LIST_IS_COL>());
+    const size_t smem = pgather_smem(a.r);
     auto kern = pgather_kernel<LIST_IS_COL, CLAMP>;
     static std::atomic<unsigned long long> attr_set{0};   // one bit per device ordinal
     int dev = 0, sms = 0, per_sm = 0;
@@ -770,7 +793,7 @@ __global__ void digit_split_kernel(const uint32_t *a, int64_t lda, int64_t rows,
 // Tile images for the tiled gather: image t holds rows 32 t .. 32 t + 31 of
 // the segment src[:, col0 .. col0 + r) exactly as pgather_kernel stages them
 // (line p = the 32 rows' words at position p, 16-byte chunk c holding rows
-// 4 (c ^ ((p >> 2) & 7)) .. + 3; zeros past the rows and positions), so that
+// 4 (c ^ pg_perm(p)) .. + 3; zeros past the rows and positions), so that
 // a whole tile is one contiguous copy.  Block (p-block, tile): 32 positions.
 __device__ __forceinline__ void tile_image_block(const uint32_t *src, int64_t lds, int64_t col0, int r,
                                                  int64_t g_count, int rp, uint32_t *img, int64_t tile, int p0,
@@ -785,7 +808,7 @@ __device__ __forceinline__ void tile_image_block(const uint32_t *src, int64_t ld
     const int c = tx >> 2, w = tx & 3;
     for (int k = ty; k < 32; k += 8) {
         const int p = p0 + k;
-        const int g = ((c ^ ((p >> 2) & 7)) << 2) | w;
+        const int g = ((c ^ (int)pg_perm((uint32_t)p)) << 2) | w;
         img[((size_t)tile * rp + p) * 32 + tx] = t[g][k];
     }
 }

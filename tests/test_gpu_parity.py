@@ -311,8 +311,8 @@ def test_layer_tiled_gather_shapes(r, t):
     """Hamming weights that are multiples of 4 take the tiled gather: ragged
     row tiles (m = 131, l = 67), segments that are not multiples of 32, a
     segment offset that is not 16-byte aligned (r_1 = 98), the longest
-    segment it stages (1568 words, from prepared tile images for Init X and
-    per-call images of Q for the unmask) and a longer one (1600) that falls
+    segment it stages (1536 words, from prepared tile images for Init X and
+    per-call images of Q for the unmask) and longer ones (1544-1600) that fall
     back to the row-staged gather."""
     for variant in _variants():
         g, ref, op, m, l = _run_layer(3, r, t, m=131, n=300, l=67, variant=variant)
