@@ -432,9 +432,10 @@ mosaic_status launch(const FwhtArgs &a, cudaStream_t st) {
 }
 
 // ---------------------------------------------------------------------------
-// Rows of 32768 whose length n is a multiple of 32: a persistent grid (one
-// block per SM) that fetches each block's NEXT input row by TMA while the
-// current row is transformed and stored.  In the kernel above an SM
+// Encode of rows of 32768 whose length n is a multiple of 32 (the rotation
+// alone runs rot_kernel below): a persistent grid (one block per SM) that
+// fetches each block's NEXT input row by TMA while the current row is
+// transformed and stored.  In the kernel above an SM
 // holds a single row at a time (32 values per thread in registers, a 512- or
 // 1024-thread block), so its loads, butterflies and stores never overlap.
 // The row arrives as a 3-D tensor {32 values, chunks, rows} with the 128-byte
@@ -580,12 +581,6 @@ __global__ void __launch_bounds__(T, 1) fwht_stream_kernel(const __grid_constant
             for (int e = 0; e < E; e++) v[e] = __fmul_rn(v[e], a.inv_sqrt);
         }
         auto elem = [&](int run) -> int { return run * 32 * E + lt * CS; };
-        if (a.mode == 0) {
-            float *yr = a.y + row * a.ldy;
-#pragma unroll
-            for (int run = 0; run < RUNS; run++) store_f32<CS>(yr + elem(run), v + run * CS);
-            continue;
-        }
         float mx = 0.0f;
         int ok = 1;
 #pragma unroll
@@ -689,7 +684,8 @@ bool stream_ok(const FwhtArgs &a) {
 }
 
 // ---------------------------------------------------------------------------
-// Rows of 16384 (length n a multiple of 32), two rows in flight per SM.  Each
+// Encode of rows of 16384 (length n a multiple of 32; the rotation alone runs
+// rot_kernel below), two rows in flight per SM.  Each
 // CTA (512 threads, 32 values a thread, at most 64 registers so that two CTAs
 // share an SM) transforms one row at a time with the stage order and roundings
 // of fwht_kernel, so the results are identical.  The row arrives by TMA in the
@@ -830,7 +826,7 @@ __global__ void __launch_bounds__(kPairT, 2) fwht_pair_kernel(const __grid_const
 #pragma unroll
             for (int e = 0; e < E; e++) v[e] = __fmul_rn(v[e], a.inv_sqrt);
         }
-        if (a.mode == 0) {
+        if (a.mode == 0) {   // rotation alone (launched as rot_kernel; kept for direct use)
             float *yr = a.y + row * a.ldy;
 #pragma unroll
             for (int run = 0; run < RUNS; run++) store_f32<CS>(yr + elem(run), v + run * CS);
