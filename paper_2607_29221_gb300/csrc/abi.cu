@@ -519,11 +519,36 @@ mosaic_status mosaic_mask_weight(const mosaic_params *p, const mosaic_key *key, 
         lev[i - 1] = SparseLevel{S_idx + soff, S_val + soff, (int)t, off_r(p, i), ri};
         soff += m * t;
     }
-    // W' = (W_hat + E_w) + L P_d + sum_i S_{i+1} P_i.
-    MOSAIC_TRY(gemm_u32(variant, cv, L, rd, 1, P + od * n_pad, 1, n_pad, Wp, n_pad, WE, n_pad, 1, m,
-                        n_pad, rd, st));
-    if (d > 1)
-        MOSAIC_TRY(sparse_rowgather(P, n_pad, lev, (int)d - 1, m, n_pad, Wp, n_pad, Wp, n_pad, st));
+    // W' = (W_hat + E_w) + L P_d + sum_i S_{i+1} P_i.  With room in the
+    // workspace (the J product's digit planes are released by now), L P_d
+    // runs against P_d^T (K-major, so the tensor cores can take it) and the
+    // sparse terms run on the tiled gather with the rows of P^T as its staged
+    // rows; otherwise the product reads P_d strided and a plain row gather
+    // reads P.
+    {
+        const size_t mark = cv.used;
+        uint32_t *PdT = cv.take<uint32_t>((size_t)(n_pad * rd));
+        if (PdT) {
+            MOSAIC_TRY(transpose_u32(P + od * n_pad, n_pad, rd, n_pad, PdT, rd, st));
+            MOSAIC_TRY(gemm_u32(variant, cv, L, rd, 1, PdT, rd, 1, Wp, n_pad, WE, n_pad, 1, m, n_pad, rd, st));
+        } else {
+            MOSAIC_TRY(gemm_u32(variant, cv, L, rd, 1, P + od * n_pad, 1, n_pad, Wp, n_pad, WE, n_pad, 1, m,
+                                n_pad, rd, st));
+        }
+        cv.used = mark;
+    }
+    if (d > 1) {
+        const size_t mark = cv.used;
+        uint32_t *PT = cv.take<uint32_t>((size_t)(n_pad * od));   // rows [0, od) of P = P_1 .. P_{d-1}
+        if (PT && od % 4 == 0) {
+            MOSAIC_TRY(transpose_u32(P, n_pad, od, n_pad, PT, od, st));
+            MOSAIC_TRY(sparse_gather(PT, od, 0, od, n_pad, m, false, lev, (int)d - 1, Wp, n_pad, nullptr, 0, 1,
+                                     Wp, n_pad, st));
+        } else {
+            MOSAIC_TRY(sparse_rowgather(P, n_pad, lev, (int)d - 1, m, n_pad, Wp, n_pad, Wp, n_pad, st));
+        }
+        cv.used = mark;
+    }
     // The server operand carries the public chains below W'.
     if (cudaMemcpyAsync(Wp + m * n_pad, P, sizeof(uint32_t) * (size_t)(Sr * n_pad),
                         cudaMemcpyDeviceToDevice, st) != cudaSuccess)
