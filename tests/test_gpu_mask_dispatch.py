@@ -110,3 +110,45 @@ def test_init_x_in_two_phases_matches_one_call(l, nested):
     assert torch.equal(one.Ux, two.Ux) and torch.equal(one.K, two.K)
     with pytest.raises(M.MosaicError):
         layer.init_x(l, 42, out=two, phase=0, ws=ws)
+
+
+def test_weight_mask_workspace_sizes_match_oracle():
+    """Init W with three workspaces: the full size (tensor-core products, P_d^T
+    and P^T carved for the L P_d product and the tiled gather of the sparse
+    terms), room for the transposes only (CUDA-core products against P_d^T,
+    tiled gather), and the minimum (CUDA-core products reading P_d strided,
+    row gather of P).  W' and J are bit-identical to the oracle for all three."""
+    from paper_2607_29221_gb300 import mosaic as M
+    p = M.default_params()
+    po = O.Params()
+    key = M.make_key(KEY)
+    m, n, n_pad, matrix_id = 300, 500, 512, 13
+    Sr, rd = sum(po.r), po.r[-1]
+    od = Sr - rd
+    full = M.mosaic_workspace_bytes(M.OP_MASK_WEIGHT, m, n_pad, 0, p)
+    ws_c = torch.empty(M.mosaic_workspace_bytes(M.OP_MASK_CHAINS, m, n_pad, 0, p), dtype=torch.uint8,
+                       device="cuda")
+    P, C, CT = _i32(Sr, n_pad), _i32(n_pad, Sr), _i32(Sr, n_pad)
+    M.mosaic_mask(M.MASK_CHAINS, p, key, n_pad, 0, n_pad, 0, dict(P=P, C=C, CT=CT), M.GEMM_AUTO, ws_c)
+    Po, Co = O.chains(KEY, po, n_pad)
+    W = wl.weights(m, n, seed=78)
+    wo = O.init_w(KEY, po, W, matrix_id, Po, Co, n_pad)
+
+    def up(v):
+        return (v + 255) // 256 * 256
+
+    minimum = up(m * n_pad * 4)
+    sizes = [full, minimum + up(n_pad * max(rd, od) * 4), minimum]
+    assert sizes[0] > sizes[1] > sizes[2]
+    for size in sizes:
+        ws = torch.empty(size, dtype=torch.uint8, device="cuda")
+        sw, s_w, L = _i32(n_pad // 32), torch.empty(m, dtype=torch.float32, device="cuda"), _i32(m, rd)
+        nsp = sum(po.t) * m
+        S_idx, S_val, Wp, J = _i32(nsp), _i32(nsp), _i32(m + Sr, n_pad), _i32(m, Sr)
+        M.mosaic_mask(M.MASK_WEIGHT, p, key, matrix_id, m, n_pad, 0,
+                      dict(W=torch.from_numpy(W).cuda(), ldw=n, n=n, P=P, CT=CT, sign_words=sw, s_w=s_w, L=L,
+                           S_idx=S_idx, S_val=S_val, Wp=Wp, J=J), M.GEMM_AUTO, ws)
+        M.mosaic_device_status()
+        assert np.array_equal(_u32(Wp)[:m], wo.W_masked), size
+        assert np.array_equal(_u32(Wp)[m:], np.vstack(Po)), size
+        assert np.array_equal(_u32(J), np.hstack(wo.J)), size
