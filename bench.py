@@ -661,7 +661,8 @@ def _client_rooflines(kt, steps, layers, proto, l, bf16, peak_src, sm_mhz, alu_m
     smem_peak = GB300_SMS * SMEM_BYTES_PER_CLK_SM * clk / 1e9
     smem_src = "derived shared-memory wavefront peak"
     if smem_measured:
-        # The device's measured conflict-free 16-byte shared-memory read rate.
+        # The device's measured shared-memory read rate with the gather's access
+        # (whole 128-byte lines, 16-byte loads, several lines a warp access).
         smem_peak = smem_measured / 1e9
         smem_src = "measured shared-memory read rate (mosaic_smem_read_rate)"
     blocks = sum(-(-l * r_act // 16) + len(act_lv) * l * 32 + -(-l * ly.n_pad // 8) for ly in layers)

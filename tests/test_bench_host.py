@@ -72,3 +72,26 @@ def test_client_rooflines_count_the_work_of_the_7b_step():
     tcu = row("unmask: Y'")
     assert abs(tcu["achieved"] - 20 * 512 * 4096 * 652 / 2e-6 / 1e12) < 0.01
     assert all(abs(r["frac"] / (r["achieved"] / r["peak"]) - 1) < 1e-3 for r in rows)
+
+
+def test_client_rooflines_take_the_measured_peaks():
+    """With the device's measured ChaCha20 mix rate and shared-memory read rate
+    the draw and gather rows use them as their peaks (and say so); the tensor
+    rows keep the bf16 figure."""
+    sys.path.insert(0, ROOT)
+    import types
+    import bench
+    from paper_2607_29221_gb300 import mosaic as M
+    proto = types.SimpleNamespace(params=M.default_params())
+    layer = types.SimpleNamespace(m=4096, n_pad=4096)
+    kt = {"init_x:initx_draw": (2, 4e-3), "init_x:pgather": (4, 8e-3), "unmask:pgather": (4, 8e-3),
+          "init_x:ring_gemm_tc": (2, 4e-3), "unmask:ring_gemm_tc": (2, 4e-3)}
+    rows = bench._client_rooflines(kt, 2, [layer], proto, 512, 1910.6, "measured", 2070.0,
+                                   alu_measured=29.088e12, smem_measured=39794.3e9)
+    by = {r["kernel"].split(" (")[0] + ":" + r["bound"]: r for r in rows}
+    assert abs(by["initx_draw_kernel:alu"]["peak"] - 29.088) < 1e-9
+    assert "mosaic_int_mix_rate" in by["initx_draw_kernel:alu"]["peak_source"]
+    gathers = [r for r in rows if r["bound"] == "smem"]
+    assert len(gathers) == 2
+    assert all(abs(r["peak"] - 39794.3) < 1e-6 and "mosaic_smem_read_rate" in r["peak_source"] for r in gathers)
+    assert all(r["peak"] == 1910.6 for r in rows if r["bound"] == "tensor")
