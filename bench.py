@@ -509,10 +509,11 @@ def run_mine(args, rank, world):
     torch.cuda.synchronize()
     M.mosaic_kernel_timing(False)
     ktimes = M.mosaic_kernel_times(reset=True)
-    # The device's rate of the ChaCha20 add / xor / rotate mix: the draws' ALU peak.
+    # The device's rate of the ChaCha20 add / xor / rotate mix: the draws' ALU peak
+    # (8 x 256 threads per SM, one scratch word each; 256 SMs' worth) ...
     mix_scratch = torch.empty(8 * 256 * 256, dtype=torch.int32, device=dev)
     alu_rate = M.mosaic_int_mix_rate(mix_scratch)
-    # ... and its conflict-free shared-memory read rate: the gathers' peak.
+    # ... and its shared-memory read rate with the gather's access: the gathers' peak.
     smem_rate = M.mosaic_smem_read_rate(mix_scratch)
     del mix_scratch
 

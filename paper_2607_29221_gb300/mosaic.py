@@ -217,7 +217,8 @@ def mosaic_int_mix_rate(scratch, stream=None) -> float:
 
 
 def mosaic_smem_read_rate(scratch, stream=None) -> float:
-    """Measured conflict-free shared-memory read rate of the device, bytes/s."""
+    """Measured shared-memory read rate of the device with the tiled gather's
+    access (whole 128-byte lines, 16-byte loads), bytes/s."""
     out = ctypes.c_double(0.0)
     _call("mosaic_smem_read_rate", _ptr(scratch), scratch.numel() * scratch.element_size(), ctypes.byref(out),
           _stream(stream))
